@@ -1,0 +1,374 @@
+#!/usr/bin/env python
+"""Benchmark of the 1.5-SPSA parameter-space step on GB300.
+
+One step = the whole hot path over one batch of synthetic inputs:
+K x (perturb +eps, perturb -2 eps, perturb +eps) over every weight tensor,
+the probe-space preconditioner on K seeded loss triples, and the fused
+K-probe update (lr = eps). Default workload: the OPT-30B-shaped fp16
+parameter set (772 tensors, 29.97e9 weights, 60 GB), K = 256.
+
+Metric: Gparam*probe/s = d * K / step time, whole job over all ranks.
+Prints one JSON line (rank 0). Multi-GPU runs (torchrun) are independent
+replicas: every rank trains its own copy; nothing is exchanged.
+
+--impl reference times the CPU oracle instead (rank 0 only), on a bounded
+prefix sample of the same workload.
+"""
+import argparse
+import hashlib
+import json
+import os
+import platform
+import statistics
+import subprocess
+import sys
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+import numpy as np  # noqa: E402
+
+from paper_2609_38095_gb300 import workloads as W  # noqa: E402
+
+METRIC = "Gparam·probe/s and HBM GB/s vs peak, fused K-probe update, OPT-30B shape"
+UNIT = "Gparam·probe/s"
+NOMINAL_HBM_GBS = 7900.0
+FALLBACK_HBM_GBS = 6800.0
+LANES_PER_SM = 128
+
+
+def parse_args():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=2)
+    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--impl", choices=["zo", "reference"], default="zo")
+    ap.add_argument("--config", default="opt-30b", choices=sorted(W.BY_KEY))
+    ap.add_argument("--cpu-seconds", type=float, default=12.0, help="target CPU time of the oracle sample")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-e2e", action="store_true")
+    return ap.parse_args()
+
+
+def measured_peaks():
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(p):
+        with open(p) as f:
+            return json.load(f), "measured"
+    return {"hbm_gbs": FALLBACK_HBM_GBS, "sm_max_mhz": 2070.0}, "fallback"
+
+
+def kernel_source_hash():
+    h = hashlib.sha256()
+    for f in ("zo_device.cuh", "zo_stream_kernels.cu"):
+        with open(os.path.join(ROOT, "paper_2609_38095_gb300", "csrc", f), "rb") as fh:
+            h.update(fh.read())
+    return h.hexdigest()[:16]
+
+
+def committed_traffic(kernel, config_key):
+    """DRAM bytes per launch from the committed ncu summary, or None when the
+    summary is missing or was taken on a different kernel source."""
+    p = os.path.join(ROOT, "profiles", "ncu_traffic.txt")
+    if not os.path.exists(p):
+        return None
+    want = kernel_source_hash()
+    for line in open(p):
+        parts = line.split()
+        if len(parts) >= 4 and parts[0] == kernel and parts[1] == config_key and parts[2] == want:
+            return float(parts[3])
+    return None
+
+
+# ----------------------------------------------------------------- clocks
+class ClockSampler:
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, device_id):
+        self.proc = None
+        self.path = os.path.join(ROOT, "gpurun_out", f"clocks_{os.getpid()}.csv")
+        self.device_id = device_id
+
+    def start(self):
+        try:
+            os.makedirs(os.path.dirname(self.path), exist_ok=True)
+            self.fh = open(self.path, "w")
+            cmd = ["nvidia-smi", f"--query-gpu={self.FIELDS}", "--format=csv,noheader,nounits", "-lms", "200"]
+            if self.device_id:
+                cmd += ["-i", self.device_id]
+            self.proc = subprocess.Popen(cmd, stdout=self.fh, stderr=subprocess.DEVNULL)
+        except (OSError, FileNotFoundError):
+            self.proc = None
+
+    def stop(self):
+        if self.proc is None:
+            return None
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except subprocess.TimeoutExpired:
+            self.proc.kill()
+        self.fh.close()
+        sm, mx, reasons = [], [], set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for line in open(self.path):
+            f = [x.strip() for x in line.split(",")]
+            if len(f) < 9:
+                continue
+            try:
+                sm.append(float(f[1]))
+                mx.append(float(f[2]))
+            except ValueError:
+                continue
+            for n, v in zip(names, f[5:9]):
+                if v.lower().startswith("active"):
+                    reasons.add(n)
+        if not sm:
+            return None
+        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": max(mx), "reasons": sorted(reasons),
+                "samples": len(sm)}
+
+
+# ------------------------------------------------------------- oracle arm
+def oracle_step(ps, M, step, host_theta):
+    """One step of the workload restricted to its first M weights (a prefix of
+    the first tensor), computed by the CPU oracle."""
+    import oracle
+    K, eps = ps.K, ps.eps
+    seed = W.step_seed(step)
+    for k in range(K):
+        for s in (eps, -2 * eps, eps):
+            oracle.perturb(host_theta, [ps.dtype], seed, k, s)
+    rc, c, _, _ = oracle.precondition(W.synthetic_losses(K, step), eps)
+    assert rc == 0
+    oracle.update(host_theta, [ps.dtype], seed, c, eps)
+
+
+def oracle_sample_size(ps, target_s):
+    rng = np.random.default_rng(0)
+    M0 = 2048
+    th = [W.random_storage(rng, M0, ps.dtype)]
+    t0 = time.perf_counter()
+    oracle_step(ps, M0, 0, th)
+    dt = time.perf_counter() - t0
+    M = int(M0 * target_s / max(dt, 1e-6))
+    return max(16, min(M, ps.numels[0]) // 16 * 16)
+
+
+def time_oracle(ps, target_s, steps=1, warmup=0):
+    import oracle
+    oracle.lib()
+    M = oracle_sample_size(ps, target_s)
+    rng = np.random.default_rng(1)
+    th = [W.random_storage(rng, M, ps.dtype)]
+    for s in range(warmup):
+        oracle_step(ps, M, s, th)
+    t0 = time.perf_counter()
+    for s in range(steps):
+        oracle_step(ps, M, warmup + s, th)
+    dt = (time.perf_counter() - t0) / steps
+    value = M * ps.K / dt / 1e9
+    sample = (f"first {M} weights of the first tensor ({ps.shapes[0][0]}) of the {ps.name} set, K={ps.K}: "
+              f"{3 * ps.K} perturb passes + preconditioner + fused update per step, single-threaded oracle")
+    return value, dt, M, sample
+
+
+def run_reference(args):
+    rank = int(os.environ.get("RANK", "0"))
+    if rank != 0:
+        return
+    ps = W.BY_KEY[args.config]
+    value, dt, M, sample = time_oracle(ps, args.cpu_seconds / 2, steps=args.steps, warmup=args.warmup)
+    line = {
+        "impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": args.gpus,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": dt * 1e3, "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "f32", "data": "synthetic",
+        "config": {"workload": ps.name, "K": ps.K, "d": ps.d, "sample_weights": M},
+        "cpu_baseline": {"value": value, "unit": UNIT, "cores": 1, "kind": "oracle", "sample": sample},
+        "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(line), flush=True)
+
+
+# ---------------------------------------------------------------- GPU arm
+def run_zo(args):
+    import torch
+    import torch.distributed as dist
+
+    import paper_2609_38095_gb300 as zo
+
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    if world > 1:
+        dist.init_process_group("nccl", device_id=dev)
+
+    def barrier():
+        if world > 1:
+            dist.barrier()
+        torch.cuda.synchronize()
+
+    def max_over_ranks(x):
+        if world == 1:
+            return x
+        t = torch.tensor([x], dtype=torch.float64, device=dev)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        return float(t.item())
+
+    ps = W.BY_KEY[args.config]
+    K, eps, d = ps.K, ps.eps, ps.d
+    params = W.allocate_params(ps, device=dev)
+    plist = zo.ParamList(params)
+    n_steps_total = args.warmup + args.steps + (0 if args.no_e2e else args.steps)
+    losses_host = [W.synthetic_losses(K, s) for s in range(n_steps_total)]
+    losses_dev = [torch.tensor(L, device=dev) for L in losses_host]
+    c = torch.empty(K, dtype=torch.float64, device=dev)
+    status = torch.zeros(1, dtype=torch.int32, device=dev)
+    stream = torch.cuda.current_stream(dev)
+    chunks = (len(params) + 1023) // 1024
+
+    timing = {"perturb": [], "update": [], "precondition": []}
+
+    def step(s, losses_d, record):
+        seed = W.step_seed(s)
+        for k in range(K):
+            for sc in (eps, -2 * eps, eps):
+                if record:
+                    e0 = torch.cuda.Event(enable_timing=True)
+                    e1 = torch.cuda.Event(enable_timing=True)
+                    e0.record(stream)
+                    zo.perturb(plist, seed, k, sc)
+                    e1.record(stream)
+                    timing["perturb"].append((e0, e1))
+                else:
+                    zo.perturb(plist, seed, k, sc)
+        if record:
+            e0, e1, e2 = (torch.cuda.Event(enable_timing=True) for _ in range(3))
+            e0.record(stream)
+        zo.precondition(losses_d, eps, out=(c, status))
+        if record:
+            e1.record(stream)
+        zo.update(plist, seed, c, eps, status=status)
+        if record:
+            e2.record(stream)
+            timing["precondition"].append((e0, e1))
+            timing["update"].append((e1, e2))
+
+    for s in range(args.warmup):
+        step(s, losses_dev[s], record=False)
+
+    # ---- timed region: inputs resident in HBM
+    dev_uuid = None
+    try:
+        dev_uuid = "GPU-" + str(torch.cuda.get_device_properties(dev).uuid)
+    except Exception:
+        pass
+    clocks = ClockSampler(dev_uuid)
+    clocks.start()
+    barrier()
+    t_start = torch.cuda.Event(enable_timing=True)
+    t_end = torch.cuda.Event(enable_timing=True)
+    t_start.record(stream)
+    for i in range(args.steps):
+        s = args.warmup + i
+        step(s, losses_dev[s], record=True)
+    t_end.record(stream)
+    barrier()
+    clk = clocks.stop()
+    elapsed_ms = max_over_ranks(t_start.elapsed_time(t_end))
+    ms_per_step = elapsed_ms / args.steps
+    launches = args.steps * (3 * K * chunks + 1 + chunks)
+
+    def avg_ms(key):
+        v = [a.elapsed_time(b) for a, b in timing[key]]
+        return sum(v) / len(v)
+
+    perturb_ms = max_over_ranks(avg_ms("perturb"))
+    update_ms = max_over_ranks(avg_ms("update"))
+    precond_ms = max_over_ranks(avg_ms("precondition"))
+
+    # ---- end to end through the public API with host buffers
+    e2e = None
+    if not args.no_e2e:
+        pinned = [torch.from_numpy(L).pin_memory() for L in losses_host]
+        c_host = torch.empty(K, dtype=torch.float64).pin_memory()
+        st_host = torch.empty(1, dtype=torch.int32).pin_memory()
+        staging = torch.empty(K, 3, dtype=torch.float64, device=dev)
+        barrier()
+        t0 = time.perf_counter()
+        for i in range(args.steps):
+            s = args.warmup + args.steps + i
+            staging.copy_(pinned[s], non_blocking=True)
+            step(s, staging, record=False)
+            c_host.copy_(c, non_blocking=True)
+            st_host.copy_(status, non_blocking=True)
+            stream.synchronize()
+            if int(st_host[0]) != 0:
+                raise RuntimeError("preconditioner reported non-finite losses")
+        barrier()
+        e2e_s = max_over_ranks((time.perf_counter() - t0) / args.steps)
+        e2e = {"value": world * d * K / e2e_s / 1e9, "unit": UNIT, "h2d_bytes_per_step": K * 3 * 8,
+               "d2h_bytes_per_step": K * 8 + 4, "ms_per_step": e2e_s * 1e3}
+
+    peaks, peak_kind = measured_peaks()
+    hbm_peak = float(peaks.get("hbm_gbs", FALLBACK_HBM_GBS))
+    perturb_bytes = 2.0 * d * ps.bytes_per_elem       # read + write every weight once
+    achieved = perturb_bytes / (perturb_ms * 1e-3) / 1e9
+    traffic = committed_traffic("perturb_kernel", args.config)
+    sms = torch.cuda.get_device_properties(dev).multi_processor_count
+    sm_mhz = (clk or {}).get("sm_mhz") or float(peaks.get("sm_max_mhz", 2070.0))
+    alu_peak = sms * LANES_PER_SM * sm_mhz * 1e6 / 1e9    # Gparam*probe/s at one instruction per pair
+    upd_rate = d * K / (update_ms * 1e-3) / 1e9
+    value = world * d * K / (ms_per_step * 1e-3) / 1e9
+
+    if rank != 0:
+        return
+    cpu = None
+    if world == 1 and not args.no_cpu_baseline:
+        v, dt, M, sample = time_oracle(ps, args.cpu_seconds)
+        cpu = {"value": v, "unit": UNIT, "cores": 1, "kind": "oracle", "sample": sample}
+    line = {
+        "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": ms_per_step, "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": "f32", "data": "synthetic",
+        "config": {"workload": ps.name, "K": K, "d": d, "tensors": len(params), "storage": "fp16" if
+                   ps.dtype == W.DT_F16 else ("bf16" if ps.dtype == W.DT_BF16 else "fp32"),
+                   "eps": eps, "lr": eps, "parallelism": f"replicas{world}",
+                   "l2": "inputs larger than L2 (every pass streams the whole parameter set)"},
+        "roofline": {"bound": "hbm", "kernel": "perturb_kernel", "achieved": achieved, "peak": hbm_peak,
+                     "unit": "GB/s", "frac": achieved / hbm_peak, "traffic": traffic,
+                     "peak_source": f"{peak_kind} hbm_gbs", "bytes_per_launch": perturb_bytes},
+        "kernels": {
+            "perturb": {"ms": perturb_ms, "GB/s": achieved, "frac_of_measured_hbm": achieved / hbm_peak,
+                        "frac_of_nominal_hbm": achieved / NOMINAL_HBM_GBS, "launches_per_step": 3 * K * chunks},
+            "update": {"ms": update_ms, "gparam_probe_per_s": upd_rate, "bound": "alu",
+                       "peak_gparam_probe_per_s_1instr": alu_peak, "frac_alu_1instr": upd_rate / alu_peak,
+                       "GB/s": perturb_bytes / (update_ms * 1e-3) / 1e9},
+            "precondition": {"ms": precond_ms},
+        },
+        "e2e": e2e,
+        "gpu_launches": launches,
+        "clocks": clk,
+        "cpu_baseline": cpu,
+        "host": platform.machine(),
+    }
+    print(json.dumps(line), flush=True)
+    if world > 1:
+        dist.destroy_process_group()
+
+
+def main():
+    args = parse_args()
+    if args.impl == "reference":
+        run_reference(args)
+    else:
+        run_zo(args)
+
+
+if __name__ == "__main__":
+    main()

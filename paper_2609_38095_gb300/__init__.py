@@ -1,1 +1,14 @@
-"""placeholder"""
+"""GB300 (sm_103a) parameter-space hot path of 1.5-SPSA: probe generation,
+fused perturb, probe-space preconditioner and fused K-probe update, behind the
+C ABI of include/zo.h. The shared library is loaded on first use; a missing
+library raises (there is no fallback).
+"""
+from .zo import (ZO_ERR_ALIGN, ZO_ERR_ARG, ZO_ERR_CUDA, ZO_ERR_DTYPE, ZO_ERR_NONFINITE, ZO_ERR_TOO_MANY_PROBES,
+                 ZO_ERR_WORKSPACE, ZO_MAX_PROBES, ZO_OK, ParamList, ZoError, perturb, precondition, probe_bytes,
+                 probe_signs, quadratic_loss, quadratic_loss_workspace_size, status_string, update,
+                 update_sequential, version)
+
+__all__ = ["ParamList", "ZoError", "perturb", "precondition", "update", "update_sequential", "probe_bytes",
+           "probe_signs", "quadratic_loss", "quadratic_loss_workspace_size", "status_string", "version",
+           "ZO_OK", "ZO_ERR_ARG", "ZO_ERR_DTYPE", "ZO_ERR_ALIGN", "ZO_ERR_NONFINITE", "ZO_ERR_CUDA",
+           "ZO_ERR_TOO_MANY_PROBES", "ZO_ERR_WORKSPACE", "ZO_MAX_PROBES"]

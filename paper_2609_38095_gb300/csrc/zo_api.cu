@@ -1,0 +1,321 @@
+// zo_api.cu -- the extern "C" entry points declared in include/zo.h: argument
+// validation, Philox key expansion, tensor-table planning and launch sizing.
+// Everything here runs on the host and only enqueues kernels.
+#include <cmath>
+#include <cstdio>
+#include <cstring>
+#include <mutex>
+
+#include <cuda_runtime.h>
+
+#include "zo.h"
+#include "zo_launch.h"
+
+namespace {
+
+using zo::PerturbParams;
+using zo::RoundKeys;
+using zo::TensorTable;
+using zo::UpdateParams;
+
+thread_local char g_last_cuda_error[256] = "";
+
+int cuda_fail(cudaError_t e, const char* where) {
+  std::snprintf(g_last_cuda_error, sizeof(g_last_cuda_error), "%s: %s (%s)", where, cudaGetErrorName(e),
+                cudaGetErrorString(e));
+  return ZO_ERR_CUDA;
+}
+
+// Philox4x32 key schedule: round r uses (lo + r * W0, hi + r * W1) mod 2^32.
+RoundKeys expand_keys(uint64_t seed) {
+  RoundKeys k;
+  uint32_t k0 = static_cast<uint32_t>(seed), k1 = static_cast<uint32_t>(seed >> 32);
+  for (int r = 0; r < 10; ++r) {
+    k.k0[r] = k0;
+    k.k1[r] = k1;
+    k0 += 0x9E3779B9u;
+    k1 += 0xBB67AE85u;
+  }
+  return k;
+}
+
+int elem_size(int32_t dtype) { return dtype == ZO_F32 ? 4 : 2; }
+
+// Per-device launch facts, filled once per device.
+struct DeviceInfo {
+  int sms = 0;
+  int perturb_bps = 0;                    // resident perturb blocks per SM
+  int update_bps[zo::kMaxGroups + 1] = {};  // by probe-group count
+};
+constexpr int kMaxDevices = 64;
+DeviceInfo g_dev[kMaxDevices];
+std::mutex g_dev_mu;
+
+int device_info(DeviceInfo** out) {
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return cuda_fail(e, "cudaGetDevice");
+  if (dev < 0 || dev >= kMaxDevices) return ZO_ERR_ARG;
+  std::lock_guard<std::mutex> lock(g_dev_mu);
+  DeviceInfo& d = g_dev[dev];
+  if (d.sms == 0) {
+    int sms = 0;
+    e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+    if (e != cudaSuccess) return cuda_fail(e, "cudaDeviceGetAttribute");
+    int bps = 0;
+    e = zo::perturb_blocks_per_sm(&bps);
+    if (e != cudaSuccess) return cuda_fail(e, "occupancy(perturb)");
+    d.perturb_bps = bps > 0 ? bps : 1;
+    d.sms = sms;
+  }
+  *out = &d;
+  return ZO_OK;
+}
+
+int update_blocks_per_sm(DeviceInfo* d, int groups, int* out) {
+  std::lock_guard<std::mutex> lock(g_dev_mu);
+  if (d->update_bps[groups] == 0) {
+    int bps = 0;
+    cudaError_t e = zo::update_blocks_per_sm(groups, &bps);
+    if (e != cudaSuccess) return cuda_fail(e, "occupancy(update)");
+    d->update_bps[groups] = bps > 0 ? bps : 1;
+  }
+  *out = d->update_bps[groups];
+  return ZO_OK;
+}
+
+int validate_params(const zo_tensor* params, int32_t n) {
+  if (n < 0) return ZO_ERR_ARG;
+  if (n > 0 && params == nullptr) return ZO_ERR_ARG;
+  int64_t blocks = 0;
+  for (int32_t t = 0; t < n; ++t) {
+    const zo_tensor& p = params[t];
+    if (p.numel < 0 || p.reserved != 0) return ZO_ERR_ARG;
+    if (p.dtype != ZO_F32 && p.dtype != ZO_BF16 && p.dtype != ZO_F16) return ZO_ERR_DTYPE;
+    if (p.numel > 0 && p.ptr == nullptr) return ZO_ERR_ARG;
+    if (reinterpret_cast<uintptr_t>(p.ptr) % static_cast<uintptr_t>(elem_size(p.dtype)) != 0) return ZO_ERR_ALIGN;
+    const int64_t nb = (p.numel + 15) / 16;
+    if (nb > (INT64_C(1) << 58) - blocks) return ZO_ERR_ARG;  // virtual index space
+    blocks += nb;
+  }
+  return ZO_OK;
+}
+
+// Fill `tab` with tensors [t0, t1) whose first virtual block is blk_begin.
+// Returns the number of blocks the launch covers.
+int64_t fill_table(TensorTable& tab, const zo_tensor* params, int32_t t0, int32_t t1, int64_t blk_begin) {
+  tab.n = t1 - t0;
+  tab.pad_ = 0;
+  tab.blk_begin = blk_begin;
+  int64_t b = blk_begin;
+  for (int32_t t = t0; t < t1; ++t) {
+    const zo_tensor& p = params[t];
+    const int i = t - t0;
+    b += (p.numel + 15) / 16;
+    tab.blk_end[i] = b;
+    tab.ptr[i] = reinterpret_cast<uint64_t>(p.ptr);
+    tab.numel[i] = p.numel;
+    uint8_t fl = static_cast<uint8_t>(p.dtype);
+    if (reinterpret_cast<uintptr_t>(p.ptr) % 32 == 0) fl |= zo::kVec32;
+    tab.flags[i] = fl;
+  }
+  return b - blk_begin;
+}
+
+int grid_for(int64_t blocks, int sms, int bps) {
+  const int64_t want = (blocks + zo::kThreads - 1) / zo::kThreads;
+  const int64_t cap = static_cast<int64_t>(sms) * bps;
+  const int64_t g = want < cap ? want : cap;
+  return static_cast<int>(g < 1 ? 1 : g);
+}
+
+// Enqueue perturb launches over the whole parameter list.
+int run_perturb(const zo_tensor* params, int32_t n, PerturbParams& pp, DeviceInfo* d, cudaStream_t s) {
+  int64_t blk = 0;
+  for (int32_t t0 = 0; t0 < n; t0 += zo::kMaxTensorsPerLaunch) {
+    const int32_t t1 = (n - t0 > zo::kMaxTensorsPerLaunch) ? t0 + zo::kMaxTensorsPerLaunch : n;
+    const int64_t nb = fill_table(pp.tab, params, t0, t1, blk);
+    if (nb > 0) {
+      cudaError_t e = zo::launch_perturb(pp, grid_for(nb, d->sms, d->perturb_bps), s);
+      if (e != cudaSuccess) return cuda_fail(e, "perturb_kernel");
+    }
+    blk += nb;
+  }
+  return ZO_OK;
+}
+
+thread_local PerturbParams tl_perturb;
+thread_local UpdateParams tl_update;
+
+}  // namespace
+
+extern "C" {
+
+const char* zo_status_string(int status) {
+  switch (status) {
+    case ZO_OK: return "ZO_OK";
+    case ZO_ERR_ARG: return "ZO_ERR_ARG: invalid argument";
+    case ZO_ERR_DTYPE: return "ZO_ERR_DTYPE: unknown dtype";
+    case ZO_ERR_ALIGN: return "ZO_ERR_ALIGN: pointer not aligned to its element size";
+    case ZO_ERR_NONFINITE: return "ZO_ERR_NONFINITE: non-finite loss, curvature or coefficient";
+    case ZO_ERR_CUDA: return "ZO_ERR_CUDA: CUDA runtime error";
+    case ZO_ERR_TOO_MANY_PROBES: return "ZO_ERR_TOO_MANY_PROBES: K exceeds ZO_MAX_PROBES";
+    case ZO_ERR_WORKSPACE: return "ZO_ERR_WORKSPACE: workspace missing or too small";
+    default: return "unknown zo_status";
+  }
+}
+
+const char* zo_last_cuda_error(void) { return g_last_cuda_error; }
+
+int zo_version(void) { return 10000; }
+
+int zo_perturb(const zo_tensor* params, int32_t n_tensors, uint64_t seed, uint32_t probe, float scale,
+               void* stream) {
+  int rc = validate_params(params, n_tensors);
+  if (rc != ZO_OK) return rc;
+  if (!std::isfinite(scale)) return ZO_ERR_ARG;
+  if (n_tensors == 0) return ZO_OK;
+  DeviceInfo* d = nullptr;
+  if ((rc = device_info(&d)) != ZO_OK) return rc;
+  PerturbParams& pp = tl_perturb;
+  pp.keys = expand_keys(seed);
+  pp.probe = probe;
+  pp.scale = scale;
+  pp.coef = nullptr;
+  pp.coef_mul = 0.0;
+  pp.status = nullptr;
+  return run_perturb(params, n_tensors, pp, d, static_cast<cudaStream_t>(stream));
+}
+
+static int check_update_args(const zo_tensor* params, int32_t n, const double* c, int32_t K, double lr) {
+  int rc = validate_params(params, n);
+  if (rc != ZO_OK) return rc;
+  if (K < 1) return ZO_ERR_ARG;
+  if (K > ZO_MAX_PROBES) return ZO_ERR_TOO_MANY_PROBES;
+  if (c == nullptr || !std::isfinite(lr)) return ZO_ERR_ARG;
+  return ZO_OK;
+}
+
+int zo_update(const zo_tensor* params, int32_t n_tensors, uint64_t seed, const double* c, int32_t K, double lr,
+              const int32_t* status, void* stream) {
+  int rc = check_update_args(params, n_tensors, c, K, lr);
+  if (rc != ZO_OK || n_tensors == 0) return rc;
+  DeviceInfo* d = nullptr;
+  if ((rc = device_info(&d)) != ZO_OK) return rc;
+  UpdateParams& up = tl_update;
+  up.keys = expand_keys(seed);
+  up.coef = c;
+  up.coef_mul = -(lr / static_cast<double>(K));
+  up.K = K;
+  up.groups = (K + 7) / 8;
+  up.status = status;
+  int bps = 1;
+  if ((rc = update_blocks_per_sm(d, up.groups, &bps)) != ZO_OK) return rc;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  int64_t blk = 0;
+  for (int32_t t0 = 0; t0 < n_tensors; t0 += zo::kMaxTensorsPerLaunch) {
+    const int32_t t1 = (n_tensors - t0 > zo::kMaxTensorsPerLaunch) ? t0 + zo::kMaxTensorsPerLaunch : n_tensors;
+    const int64_t nb = fill_table(up.tab, params, t0, t1, blk);
+    if (nb > 0) {
+      cudaError_t e = zo::launch_update(up, grid_for(nb, d->sms, bps), s);
+      if (e != cudaSuccess) return cuda_fail(e, "update_kernel");
+    }
+    blk += nb;
+  }
+  return ZO_OK;
+}
+
+int zo_update_sequential(const zo_tensor* params, int32_t n_tensors, uint64_t seed, const double* c, int32_t K,
+                         double lr, const int32_t* status, void* stream) {
+  int rc = check_update_args(params, n_tensors, c, K, lr);
+  if (rc != ZO_OK || n_tensors == 0) return rc;
+  DeviceInfo* d = nullptr;
+  if ((rc = device_info(&d)) != ZO_OK) return rc;
+  PerturbParams& pp = tl_perturb;
+  pp.keys = expand_keys(seed);
+  pp.scale = 0.0f;
+  pp.coef = c;
+  pp.coef_mul = -(lr / static_cast<double>(K));
+  pp.status = status;
+  for (int32_t k = 0; k < K; ++k) {
+    pp.probe = static_cast<uint32_t>(k);
+    if ((rc = run_perturb(params, n_tensors, pp, d, static_cast<cudaStream_t>(stream))) != ZO_OK) return rc;
+  }
+  return ZO_OK;
+}
+
+static int check_precondition_args(const double* losses, int32_t K, double eps, double alpha, double lambda_reg,
+                                   const double* c, const int32_t* status) {
+  if (K < 1) return ZO_ERR_ARG;
+  if (K > ZO_MAX_PROBES) return ZO_ERR_TOO_MANY_PROBES;
+  if (losses == nullptr || c == nullptr || status == nullptr) return ZO_ERR_ARG;
+  if (!(eps > 0.0) || !std::isfinite(eps)) return ZO_ERR_ARG;
+  if (!(alpha >= 0.0) || !(alpha <= 1.0)) return ZO_ERR_ARG;
+  if (!(lambda_reg > 0.0) || !std::isfinite(lambda_reg)) return ZO_ERR_ARG;
+  return ZO_OK;
+}
+
+int zo_precondition_ex(const double* losses, int32_t K, double eps, double alpha, double lambda_reg,
+                       int32_t one_sided, double* c, double* w, double* curv, int32_t* status, void* stream) {
+  int rc = check_precondition_args(losses, K, eps, alpha, lambda_reg, c, status);
+  if (rc != ZO_OK) return rc;
+  cudaError_t e = zo::launch_precondition(losses, K, eps, alpha, lambda_reg, one_sided != 0, c, w, curv, status,
+                                          static_cast<cudaStream_t>(stream));
+  return e == cudaSuccess ? ZO_OK : cuda_fail(e, "precondition_kernel");
+}
+
+int zo_precondition(const double* losses, int32_t K, double eps, double* c, int32_t* status, void* stream) {
+  return zo_precondition_ex(losses, K, eps, 0.1, 1.0, 0, c, nullptr, nullptr, status, stream);
+}
+
+static int probe_view_grid(int64_t blocks, int* grid) {
+  DeviceInfo* d = nullptr;
+  int rc = device_info(&d);
+  if (rc != ZO_OK) return rc;
+  *grid = grid_for(blocks, d->sms, 8);
+  return ZO_OK;
+}
+
+int zo_probe_bytes(uint64_t seed, uint32_t probe, int64_t first, int64_t n, uint8_t* out, void* stream) {
+  if (first < 0 || n < 0 || (n > 0 && out == nullptr)) return ZO_ERR_ARG;
+  if (n > (INT64_C(1) << 58) - first) return ZO_ERR_ARG;
+  if (n == 0) return ZO_OK;
+  int grid = 1;
+  int rc = probe_view_grid((n + 1) / 2 + 1, &grid);
+  if (rc != ZO_OK) return rc;
+  cudaError_t e = zo::launch_probe_bytes(expand_keys(seed), probe, first, n, out, grid,
+                                         static_cast<cudaStream_t>(stream));
+  return e == cudaSuccess ? ZO_OK : cuda_fail(e, "probe_bytes_kernel");
+}
+
+int zo_probe_signs(uint64_t seed, uint32_t probe, int64_t first, int64_t n, int8_t* out, void* stream) {
+  if (first < 0 || n < 0 || (n > 0 && out == nullptr)) return ZO_ERR_ARG;
+  if (n > (INT64_C(1) << 58) - first) return ZO_ERR_ARG;
+  if (n == 0) return ZO_OK;
+  int grid = 1;
+  int rc = probe_view_grid(n / 16 + 2, &grid);
+  if (rc != ZO_OK) return rc;
+  cudaError_t e = zo::launch_probe_signs(expand_keys(seed), probe, first, n, out, grid,
+                                         static_cast<cudaStream_t>(stream));
+  return e == cudaSuccess ? ZO_OK : cuda_fail(e, "probe_signs_kernel");
+}
+
+int64_t zo_quadratic_loss_workspace_size(int64_t n) {
+  (void)n;
+  return static_cast<int64_t>(zo::kMaxLossPartials) * static_cast<int64_t>(sizeof(double));
+}
+
+int zo_quadratic_loss(const float* theta, const float* a, int64_t n, double* out, void* workspace,
+                      int64_t workspace_bytes, void* stream) {
+  if (n < 0 || out == nullptr || (n > 0 && (theta == nullptr || a == nullptr))) return ZO_ERR_ARG;
+  if (workspace == nullptr || workspace_bytes < zo_quadratic_loss_workspace_size(n)) return ZO_ERR_WORKSPACE;
+  if (reinterpret_cast<uintptr_t>(workspace) % sizeof(double) != 0) return ZO_ERR_ALIGN;
+  DeviceInfo* d = nullptr;
+  int rc = device_info(&d);
+  if (rc != ZO_OK) return rc;
+  cudaError_t e = zo::launch_quadratic_loss(theta, a, n, out, static_cast<double*>(workspace), zo::kMaxLossPartials,
+                                            d->sms, static_cast<cudaStream_t>(stream));
+  return e == cudaSuccess ? ZO_OK : cuda_fail(e, "quadratic_loss");
+}
+
+}  // extern "C"

@@ -1,0 +1,30 @@
+// zo_launch.h -- host-side launch wrappers shared between the kernel files and
+// the C ABI layer (not part of the public interface).
+#pragma once
+
+#include <cuda_runtime.h>
+
+#include "zo_device.cuh"
+
+namespace zo {
+
+constexpr int kStatusNonFinite = -4;  // ZO_ERR_NONFINITE
+constexpr int kThreads = 256;         // threads per block of the streaming kernels
+constexpr int kMaxLossPartials = 2048;
+
+cudaError_t launch_perturb(const PerturbParams& p, int grid, cudaStream_t stream);
+cudaError_t launch_update(const UpdateParams& p, int grid, cudaStream_t stream);
+size_t update_smem_bytes(int groups);
+cudaError_t perturb_blocks_per_sm(int* out);
+cudaError_t update_blocks_per_sm(int groups, int* out);
+cudaError_t launch_probe_bytes(const RoundKeys& keys, uint32_t probe, int64_t first, int64_t n, uint8_t* out,
+                               int grid, cudaStream_t stream);
+cudaError_t launch_probe_signs(const RoundKeys& keys, uint32_t probe, int64_t first, int64_t n, int8_t* out,
+                               int grid, cudaStream_t stream);
+cudaError_t launch_precondition(const double* losses, int K, double eps, double alpha, double lambda_reg,
+                                int one_sided, double* c, double* w, double* curv, int32_t* status,
+                                cudaStream_t stream);
+cudaError_t launch_quadratic_loss(const float* theta, const float* a, int64_t n, double* out, double* partial,
+                                  int max_partials, int num_sms, cudaStream_t stream);
+
+}  // namespace zo

@@ -1,0 +1,289 @@
+// zo_stream_kernels.cu -- the HBM-streaming kernels of the 1.5-SPSA step:
+// fused perturb (Algorithm 1, ApplyPackedPerturbation), fused K-probe update
+// (Sec. 4.2, Eqs. 5-6) and the debug views of a probe.
+//
+// Work unit: one thread owns one 16-element Philox block at a time (grid-
+// stride over the virtual block space of the launch's tensor table). A block
+// of a 16-bit tensor is 32 bytes: one 256-bit load and one 256-bit store when
+// the tensor is 32-byte aligned, element-wise access otherwise or for a
+// tensor's last, partial block.
+#include "zo_device.cuh"
+
+namespace zo {
+
+// ---------------------------------------------------------------------------
+// Perturb: theta <- rn(fp32(theta) + scale * z_k) in place.
+//
+// z_k[g] is bit (k mod 8) of byte (g mod 16) of Philox(b = g/16, q = k/8).
+// Byte m sits at bits 8(m mod 4).. of word m/4; shifting the word left by
+// 31 - 8(m mod 4) - (k mod 8) puts the probe bit in the sign position, which
+// then flips -scale into +scale (bit 1 -> z = +1). The product scale * z is
+// exact, so the element result is one fp32 add and one rounding to storage.
+// ---------------------------------------------------------------------------
+// Probe bit of element i (0..15) of a block, moved to bit 31.
+__device__ __forceinline__ uint32_t sign_bit(const uint4& x, int i, uint32_t j) {
+  return (word_of(x, i >> 2) << (31u - 8u * static_cast<uint32_t>(i & 3) - j)) & 0x80000000u;
+}
+
+template <uint8_t DT>
+__device__ __forceinline__ void perturb_block_vec(void* base, int64_t e0, const uint4& x, uint32_t nscale_bits,
+                                                  uint32_t j) {
+  if constexpr (DT == kF32) {
+    float* p = static_cast<float*>(base) + e0;
+#pragma unroll
+    for (int half = 0; half < 2; ++half) {
+      uint32_t v[8];
+      ld256(p + 8 * half, v);
+#pragma unroll
+      for (int r = 0; r < 8; ++r) {
+        const int i = 8 * half + r;  // element within the block
+        const float d = __uint_as_float(nscale_bits ^ sign_bit(x, i, j));
+        v[r] = __float_as_uint(__fadd_rn(__uint_as_float(v[r]), d));
+      }
+      st256(p + 8 * half, v);
+    }
+  } else {
+    uint16_t* p = static_cast<uint16_t*>(base) + e0;
+    uint32_t v[8];
+    ld256(p, v);
+#pragma unroll
+    for (int r = 0; r < 8; ++r) {
+      const float2 f = unpack2<DT>(v[r]);
+      const float r0 = __fadd_rn(f.x, __uint_as_float(nscale_bits ^ sign_bit(x, 2 * r, j)));
+      const float r1 = __fadd_rn(f.y, __uint_as_float(nscale_bits ^ sign_bit(x, 2 * r + 1, j)));
+      v[r] = pack2<DT>(r0, r1);
+    }
+    st256(p, v);
+  }
+}
+
+__global__ void __launch_bounds__(256) perturb_kernel(const __grid_constant__ PerturbParams P) {
+  if (P.status != nullptr && *P.status != 0) return;
+  float scale = P.scale;
+  if (P.coef != nullptr) scale = __double2float_rn(P.coef_mul * P.coef[P.probe]);
+  const uint32_t nscale_bits = __float_as_uint(scale) ^ 0x80000000u;  // -scale
+  const uint32_t j = P.probe & 7u;
+  const uint32_t q = P.probe >> 3;
+
+  const TensorTable& tab = P.tab;
+  const int64_t blk_total = tab.blk_end[tab.n - 1];
+  const int64_t stride = static_cast<int64_t>(gridDim.x) * blockDim.x;
+  int t = 0;
+  for (int64_t b = tab.blk_begin + static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; b < blk_total;
+       b += stride) {
+    t = advance_tensor(tab, t, b);
+    const int64_t e0 = (b - tensor_blk_begin(tab, t)) * 16;
+    const int64_t cnt = min(static_cast<int64_t>(16), tab.numel[t] - e0);
+    const uint8_t fl = tab.flags[t];
+    const uint8_t dt = fl & kDtypeMask;
+    void* base = reinterpret_cast<void*>(tab.ptr[t]);
+    const uint4 x = philox10(static_cast<uint32_t>(b), static_cast<uint32_t>(static_cast<uint64_t>(b) >> 32), q, 0u,
+                             P.keys);
+    if (cnt == 16 && (fl & kVec32)) {
+      if (dt == kBF16)
+        perturb_block_vec<kBF16>(base, e0, x, nscale_bits, j);
+      else if (dt == kF16)
+        perturb_block_vec<kF16>(base, e0, x, nscale_bits, j);
+      else
+        perturb_block_vec<kF32>(base, e0, x, nscale_bits, j);
+    } else {
+      for (int i = 0; i < cnt; ++i) {
+        const float th = load_elem(base, dt, e0 + i);
+        store_elem(base, dt, e0 + i, __fadd_rn(th, __uint_as_float(nscale_bits ^ sign_bit(x, i, j))));
+      }
+    }
+  }
+}
+
+// ---------------------------------------------------------------------------
+// Fused K-probe update: theta <- rn(fp32(theta) + sum_k a_k z_k[g]).
+//
+// Byte m of Philox(b, q) holds the signs of probes 8q..8q+7 for element
+// 16b + m. Its low nibble indexes a 16-entry table of the fp32 partial sums
+//   T[n] = ((s0 a_{4h} + s1 a_{4h+1}) + s2 a_{4h+2}) + s3 a_{4h+3},
+//   s_j = +1 if bit j of n is set, else -1,
+// for probe quad h = 2q, the high nibble the table of quad 2q + 1. Each
+// element adds the two looked-up partials to its fp32 accumulator, quads in
+// increasing order: one shared-memory load and one add per four probes
+// instead of a select and an add per probe. Probes K..8*groups-1 have a = 0.
+// ---------------------------------------------------------------------------
+__device__ __forceinline__ void accumulate_block(float (&acc)[16], int64_t b, const UpdateParams& P,
+                                                 const float* __restrict__ lut) {
+  const uint32_t blo = static_cast<uint32_t>(b), bhi = static_cast<uint32_t>(static_cast<uint64_t>(b) >> 32);
+  for (int q = 0; q < P.groups; ++q) {
+    const uint4 x = philox10(blo, bhi, static_cast<uint32_t>(q), 0u, P.keys);
+    const float* tlo = lut + 32 * q;
+    const float* thi = tlo + 16;
+#pragma unroll
+    for (int m = 0; m < 16; ++m) {
+      const uint32_t byte = (word_of(x, m >> 2) >> (8 * (m & 3))) & 0xFFu;
+      acc[m] = __fadd_rn(acc[m], tlo[byte & 0xFu]);
+      acc[m] = __fadd_rn(acc[m], thi[byte >> 4]);
+    }
+  }
+}
+
+template <uint8_t DT>
+__device__ __forceinline__ void apply_block_vec(void* base, int64_t e0, const float (&acc)[16]) {
+  if constexpr (DT == kF32) {
+    float* p = static_cast<float*>(base) + e0;
+#pragma unroll
+    for (int half = 0; half < 2; ++half) {
+      uint32_t v[8];
+      ld256(p + 8 * half, v);
+#pragma unroll
+      for (int r = 0; r < 8; ++r) v[r] = __float_as_uint(__fadd_rn(__uint_as_float(v[r]), acc[8 * half + r]));
+      st256(p + 8 * half, v);
+    }
+  } else {
+    uint16_t* p = static_cast<uint16_t*>(base) + e0;
+    uint32_t v[8];
+    ld256(p, v);
+#pragma unroll
+    for (int r = 0; r < 8; ++r) {
+      const float2 f = unpack2<DT>(v[r]);
+      v[r] = pack2<DT>(__fadd_rn(f.x, acc[2 * r]), __fadd_rn(f.y, acc[2 * r + 1]));
+    }
+    st256(p, v);
+  }
+}
+
+__global__ void __launch_bounds__(256) update_kernel(const __grid_constant__ UpdateParams P) {
+  extern __shared__ float smem[];
+  float* a_s = smem;                 // 8 * groups coefficients (zero padded)
+  float* lut = smem + 8 * P.groups;  // 2 * groups tables of 16 partial sums
+  __shared__ int skip;
+  if (threadIdx.x == 0) skip = (P.status != nullptr && *P.status != 0);
+  const int npad = 8 * P.groups;
+  for (int k = threadIdx.x; k < npad; k += blockDim.x)
+    a_s[k] = k < P.K ? __double2float_rn(P.coef_mul * P.coef[k]) : 0.0f;
+  __syncthreads();
+  if (skip) return;
+  for (int e = threadIdx.x; e < 32 * P.groups; e += blockDim.x) {
+    const int h = e >> 4, n = e & 15;
+    const float* a = a_s + 4 * h;
+    float s = (n & 1) ? a[0] : -a[0];
+    s = __fadd_rn(s, (n & 2) ? a[1] : -a[1]);
+    s = __fadd_rn(s, (n & 4) ? a[2] : -a[2]);
+    s = __fadd_rn(s, (n & 8) ? a[3] : -a[3]);
+    lut[e] = s;
+  }
+  __syncthreads();
+
+  const TensorTable& tab = P.tab;
+  const int64_t blk_total = tab.blk_end[tab.n - 1];
+  const int64_t stride = static_cast<int64_t>(gridDim.x) * blockDim.x;
+  int t = 0;
+  for (int64_t b = tab.blk_begin + static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; b < blk_total;
+       b += stride) {
+    t = advance_tensor(tab, t, b);
+    float acc[16];
+#pragma unroll
+    for (int m = 0; m < 16; ++m) acc[m] = 0.0f;
+    accumulate_block(acc, b, P, lut);
+    const int64_t e0 = (b - tensor_blk_begin(tab, t)) * 16;
+    const int64_t cnt = min(static_cast<int64_t>(16), tab.numel[t] - e0);
+    const uint8_t fl = tab.flags[t];
+    const uint8_t dt = fl & kDtypeMask;
+    void* base = reinterpret_cast<void*>(tab.ptr[t]);
+    if (cnt == 16 && (fl & kVec32)) {
+      if (dt == kBF16)
+        apply_block_vec<kBF16>(base, e0, acc);
+      else if (dt == kF16)
+        apply_block_vec<kF16>(base, e0, acc);
+      else
+        apply_block_vec<kF32>(base, e0, acc);
+    } else {
+#pragma unroll
+      for (int i = 0; i < 16; ++i) {
+        if (i < cnt) store_elem(base, dt, e0 + i, __fadd_rn(load_elem(base, dt, e0 + i), acc[i]));
+      }
+    }
+  }
+}
+
+// ---------------------------------------------------------------------------
+// Debug views: probe k packed one bit per element (Appendix F layout) and the
+// unpacked int8 signs, over a range of the virtual index space.
+// ---------------------------------------------------------------------------
+__global__ void probe_bytes_kernel(RoundKeys keys, uint32_t probe, int64_t first, int64_t n, uint8_t* out) {
+  const uint32_t j = probe & 7u, q = probe >> 3;
+  const int64_t b_first = first >> 1, b_last = (first + n - 1) >> 1;  // packed bytes 2b, 2b+1 <- block b
+  const int64_t stride = static_cast<int64_t>(gridDim.x) * blockDim.x;
+  for (int64_t b = b_first + static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; b <= b_last; b += stride) {
+    const uint4 x = philox10(static_cast<uint32_t>(b), static_cast<uint32_t>(static_cast<uint64_t>(b) >> 32), q, 0u,
+                             keys);
+#pragma unroll
+    for (int half = 0; half < 2; ++half) {
+      const int64_t jb = 2 * b + half;
+      if (jb < first || jb >= first + n) continue;
+      uint32_t v = 0;
+#pragma unroll
+      for (int i = 0; i < 8; ++i) {
+        const int m = 8 * half + i;
+        v |= ((word_of(x, m >> 2) >> (8 * (m & 3) + j)) & 1u) << i;
+      }
+      out[jb - first] = static_cast<uint8_t>(v);
+    }
+  }
+}
+
+__global__ void probe_signs_kernel(RoundKeys keys, uint32_t probe, int64_t first, int64_t n, int8_t* out) {
+  const uint32_t j = probe & 7u, q = probe >> 3;
+  const int64_t b_first = first >> 4, b_last = (first + n - 1) >> 4;
+  const int64_t stride = static_cast<int64_t>(gridDim.x) * blockDim.x;
+  for (int64_t b = b_first + static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; b <= b_last; b += stride) {
+    const uint4 x = philox10(static_cast<uint32_t>(b), static_cast<uint32_t>(static_cast<uint64_t>(b) >> 32), q, 0u,
+                             keys);
+#pragma unroll
+    for (int m = 0; m < 16; ++m) {
+      const int64_t g = 16 * b + m;
+      if (g < first || g >= first + n) continue;
+      const uint32_t bit = (word_of(x, m >> 2) >> (8 * (m & 3) + j)) & 1u;
+      out[g - first] = bit ? static_cast<int8_t>(1) : static_cast<int8_t>(-1);
+    }
+  }
+}
+
+}  // namespace zo
+
+// ---------------------------------------------------------------------------
+// Launch wrappers.
+// ---------------------------------------------------------------------------
+#include "zo_launch.h"
+
+namespace zo {
+
+cudaError_t launch_perturb(const PerturbParams& p, int grid, cudaStream_t stream) {
+  perturb_kernel<<<grid, kThreads, 0, stream>>>(p);
+  return cudaGetLastError();
+}
+
+size_t update_smem_bytes(int groups) { return static_cast<size_t>(groups) * 40 * sizeof(float); }
+
+cudaError_t launch_update(const UpdateParams& p, int grid, cudaStream_t stream) {
+  update_kernel<<<grid, kThreads, update_smem_bytes(p.groups), stream>>>(p);
+  return cudaGetLastError();
+}
+
+cudaError_t perturb_blocks_per_sm(int* out) {
+  return cudaOccupancyMaxActiveBlocksPerMultiprocessor(out, perturb_kernel, kThreads, 0);
+}
+
+cudaError_t update_blocks_per_sm(int groups, int* out) {
+  return cudaOccupancyMaxActiveBlocksPerMultiprocessor(out, update_kernel, kThreads, update_smem_bytes(groups));
+}
+
+cudaError_t launch_probe_bytes(const RoundKeys& keys, uint32_t probe, int64_t first, int64_t n, uint8_t* out,
+                               int grid, cudaStream_t stream) {
+  probe_bytes_kernel<<<grid, kThreads, 0, stream>>>(keys, probe, first, n, out);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_probe_signs(const RoundKeys& keys, uint32_t probe, int64_t first, int64_t n, int8_t* out,
+                               int grid, cudaStream_t stream) {
+  probe_signs_kernel<<<grid, kThreads, 0, stream>>>(keys, probe, first, n, out);
+  return cudaGetLastError();
+}
+
+}  // namespace zo

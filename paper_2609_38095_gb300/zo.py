@@ -1,0 +1,243 @@
+"""Python binding of libzo.so (include/zo.h): argument marshalling only.
+
+Every numeric step runs in the library's CUDA kernels; this module turns torch
+CUDA tensors into pointers, passes the current torch stream, and raises on a
+non-zero status. There is no CPU path: if libzo.so is missing, every call
+raises.
+"""
+import ctypes
+import os
+
+import torch
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(_HERE, "libzo.so")
+
+ZO_OK = 0
+ZO_ERR_ARG = -1
+ZO_ERR_DTYPE = -2
+ZO_ERR_ALIGN = -3
+ZO_ERR_NONFINITE = -4
+ZO_ERR_CUDA = -5
+ZO_ERR_TOO_MANY_PROBES = -6
+ZO_ERR_WORKSPACE = -7
+ZO_MAX_PROBES = 1024
+
+DTYPE_CODE = {torch.float32: 0, torch.bfloat16: 1, torch.float16: 2}
+
+EXPORTS = ["zo_status_string", "zo_last_cuda_error", "zo_version", "zo_perturb", "zo_precondition",
+           "zo_precondition_ex", "zo_update", "zo_update_sequential", "zo_probe_bytes", "zo_probe_signs",
+           "zo_quadratic_loss_workspace_size", "zo_quadratic_loss"]
+
+
+class zo_tensor(ctypes.Structure):
+    _fields_ = [("ptr", ctypes.c_void_p), ("numel", ctypes.c_int64), ("dtype", ctypes.c_int32),
+                ("reserved", ctypes.c_int32)]
+
+
+class ZoError(RuntimeError):
+    def __init__(self, fn, status):
+        msg = f"{fn}: {status_string(status)}"
+        if status == ZO_ERR_CUDA:
+            msg += f" [{_lib().zo_last_cuda_error().decode()}]"
+        super().__init__(msg)
+        self.status = status
+
+
+_L = None
+
+
+def _lib():
+    global _L
+    if _L is None:
+        if not os.path.exists(LIB_PATH):
+            raise RuntimeError(f"{LIB_PATH} is not built; run paper_2609_38095_gb300.build.build() "
+                               "(there is no fallback implementation)")
+        L = ctypes.CDLL(LIB_PATH)
+        c = ctypes
+        vp, i32, i64, u32, u64, f32, f64 = c.c_void_p, c.c_int32, c.c_int64, c.c_uint32, c.c_uint64, c.c_float, c.c_double
+        sig = {
+            "zo_status_string": ([c.c_int], c.c_char_p),
+            "zo_last_cuda_error": ([], c.c_char_p),
+            "zo_version": ([], c.c_int),
+            "zo_perturb": ([vp, i32, u64, u32, f32, vp], c.c_int),
+            "zo_precondition": ([vp, i32, f64, vp, vp, vp], c.c_int),
+            "zo_precondition_ex": ([vp, i32, f64, f64, f64, i32, vp, vp, vp, vp, vp], c.c_int),
+            "zo_update": ([vp, i32, u64, vp, i32, f64, vp, vp], c.c_int),
+            "zo_update_sequential": ([vp, i32, u64, vp, i32, f64, vp, vp], c.c_int),
+            "zo_probe_bytes": ([u64, u32, i64, i64, vp, vp], c.c_int),
+            "zo_probe_signs": ([u64, u32, i64, i64, vp, vp], c.c_int),
+            "zo_quadratic_loss_workspace_size": ([i64], i64),
+            "zo_quadratic_loss": ([vp, vp, i64, vp, vp, i64, vp], c.c_int),
+        }
+        for name, (args, res) in sig.items():
+            f = getattr(L, name)
+            f.argtypes = args
+            f.restype = res
+        _L = L
+    return _L
+
+
+def status_string(status: int) -> str:
+    return _lib().zo_status_string(int(status)).decode()
+
+
+def version() -> int:
+    return _lib().zo_version()
+
+
+def _check(fn, rc):
+    if rc != ZO_OK:
+        raise ZoError(fn, rc)
+
+
+def _stream(device):
+    return ctypes.c_void_p(torch.cuda.current_stream(device).cuda_stream)
+
+
+def _dev_ptr(t, dtype=None, what="tensor"):
+    if not isinstance(t, torch.Tensor) or not t.is_cuda:
+        raise TypeError(f"{what} must be a CUDA tensor")
+    if not t.is_contiguous():
+        raise ValueError(f"{what} must be contiguous")
+    if dtype is not None and t.dtype != dtype:
+        raise TypeError(f"{what} must be {dtype}, got {t.dtype}")
+    return ctypes.c_void_p(t.data_ptr())
+
+
+class ParamList:
+    """The parameter list of a training step: a fixed, ordered list of CUDA
+    tensors, each updated in place. Build it once and pass it to every call of
+    every step: the probes are defined by each element's position in it."""
+
+    def __init__(self, tensors):
+        self.tensors = list(tensors)
+        n = len(self.tensors)
+        arr = (zo_tensor * max(n, 1))()
+        dev = None
+        for i, t in enumerate(self.tensors):
+            if not isinstance(t, torch.Tensor) or not t.is_cuda:
+                raise TypeError("parameters must be CUDA tensors")
+            if not t.is_contiguous():
+                raise ValueError("parameters must be contiguous")
+            if t.dtype not in DTYPE_CODE:
+                raise TypeError(f"unsupported parameter dtype {t.dtype}")
+            if dev is None:
+                dev = t.device
+            elif t.device != dev:
+                raise ValueError("all parameters must live on one device")
+            arr[i].ptr = t.data_ptr()
+            arr[i].numel = t.numel()
+            arr[i].dtype = DTYPE_CODE[t.dtype]
+            arr[i].reserved = 0
+        self._arr = arr
+        self.n = n
+        self.device = dev if dev is not None else torch.device("cuda", torch.cuda.current_device())
+
+    @property
+    def numels(self):
+        return [t.numel() for t in self.tensors]
+
+    def __len__(self):
+        return self.n
+
+
+def _plist(params):
+    return params if isinstance(params, ParamList) else ParamList(params)
+
+
+def perturb(params, seed: int, probe: int, scale: float):
+    """theta <- theta + scale * z_probe in place (zo_perturb)."""
+    p = _plist(params)
+    with torch.cuda.device(p.device):
+        _check("zo_perturb", _lib().zo_perturb(p._arr, p.n, seed, probe, scale, _stream(p.device)))
+
+
+def precondition(losses, eps: float, alpha: float = 0.1, lambda_reg: float = 1.0, one_sided: bool = False,
+                 out=None, with_weights: bool = False):
+    """losses: CUDA float64 tensor (K, 3) of rows (L+, L-, L0).
+    Returns (c, status) -- or (c, status, w, curv) with with_weights -- as CUDA
+    tensors; status[0] is ZO_OK or ZO_ERR_NONFINITE once the kernel has run."""
+    if losses.dim() != 2 or losses.shape[1] != 3:
+        raise ValueError("losses must have shape (K, 3)")
+    lp = _dev_ptr(losses, torch.float64, "losses")
+    K = losses.shape[0]
+    dev = losses.device
+    if out is None:
+        c = torch.empty(K, dtype=torch.float64, device=dev)
+        status = torch.empty(1, dtype=torch.int32, device=dev)
+    else:
+        c, status = out
+    w = curv = None
+    if with_weights:
+        w = torch.empty(K, dtype=torch.float64, device=dev)
+        curv = torch.empty(K, dtype=torch.float64, device=dev)
+    with torch.cuda.device(dev):
+        rc = _lib().zo_precondition_ex(lp, K, eps, alpha, lambda_reg, int(one_sided),
+                                       _dev_ptr(c, torch.float64, "c"),
+                                       _dev_ptr(w, torch.float64) if w is not None else None,
+                                       _dev_ptr(curv, torch.float64) if curv is not None else None,
+                                       _dev_ptr(status, torch.int32, "status"), _stream(dev))
+    _check("zo_precondition", rc)
+    return (c, status, w, curv) if with_weights else (c, status)
+
+
+def update(params, seed: int, c, lr: float, status=None):
+    """theta <- theta - (lr / K) * sum_k c_k z_k in one pass (zo_update)."""
+    p = _plist(params)
+    st = _dev_ptr(status, torch.int32, "status") if status is not None else None
+    with torch.cuda.device(p.device):
+        rc = _lib().zo_update(p._arr, p.n, seed, _dev_ptr(c, torch.float64, "c"), c.numel(), lr, st,
+                              _stream(p.device))
+    _check("zo_update", rc)
+
+
+def update_sequential(params, seed: int, c, lr: float, status=None):
+    """Algorithm 1's K-pass application, the comparator (zo_update_sequential)."""
+    p = _plist(params)
+    st = _dev_ptr(status, torch.int32, "status") if status is not None else None
+    with torch.cuda.device(p.device):
+        rc = _lib().zo_update_sequential(p._arr, p.n, seed, _dev_ptr(c, torch.float64, "c"), c.numel(), lr, st,
+                                         _stream(p.device))
+    _check("zo_update_sequential", rc)
+
+
+def probe_bytes(seed: int, probe: int, first: int, n: int, device=None):
+    """Probe `probe` packed one bit per element (bytes first..first+n-1)."""
+    out = torch.empty(n, dtype=torch.uint8, device=device or "cuda")
+    with torch.cuda.device(out.device):
+        rc = _lib().zo_probe_bytes(seed, probe, first, n, ctypes.c_void_p(out.data_ptr()), _stream(out.device))
+    _check("zo_probe_bytes", rc)
+    return out
+
+
+def probe_signs(seed: int, probe: int, first: int, n: int, device=None):
+    """z_probe[g] as int8 for g = first..first+n-1."""
+    out = torch.empty(n, dtype=torch.int8, device=device or "cuda")
+    with torch.cuda.device(out.device):
+        rc = _lib().zo_probe_signs(seed, probe, first, n, ctypes.c_void_p(out.data_ptr()), _stream(out.device))
+    _check("zo_probe_signs", rc)
+    return out
+
+
+def quadratic_loss_workspace_size(n: int) -> int:
+    return _lib().zo_quadratic_loss_workspace_size(n)
+
+
+def quadratic_loss(theta, a, out=None, workspace=None):
+    """f = 1/2 sum a_i theta_i^2 in fp64, into out (a CUDA float64 tensor of
+    one element, returned)."""
+    n = theta.numel()
+    if a.numel() != n:
+        raise ValueError("theta and a differ in size")
+    dev = theta.device
+    if out is None:
+        out = torch.empty(1, dtype=torch.float64, device=dev)
+    if workspace is None:
+        workspace = torch.empty(quadratic_loss_workspace_size(n), dtype=torch.uint8, device=dev)
+    with torch.cuda.device(dev):
+        rc = _lib().zo_quadratic_loss(_dev_ptr(theta, torch.float32, "theta"), _dev_ptr(a, torch.float32, "a"), n,
+                                      ctypes.c_void_p(out.data_ptr()), ctypes.c_void_p(workspace.data_ptr()),
+                                      workspace.numel(), _stream(dev))
+    _check("zo_quadratic_loss", rc)
+    return out

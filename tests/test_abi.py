@@ -1,0 +1,118 @@
+"""C-ABI checks that need no GPU: the library builds, loads, exports every
+entry point declared in include/zo.h, and rejects bad arguments on the host
+before touching CUDA."""
+import ctypes
+import os
+import re
+
+import pytest
+
+from paper_2609_38095_gb300 import build as zo_build
+from paper_2609_38095_gb300 import zo
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+@pytest.fixture(scope="module")
+def L():
+    zo_build.build()
+    return zo._lib()
+
+
+def header_functions():
+    src = open(os.path.join(ROOT, "include", "zo.h")).read()
+    src = re.sub(r"/\*.*?\*/", "", src, flags=re.S)
+    return sorted(set(re.findall(r"\b(zo_[a-z0-9_]+)\s*\(", src)))
+
+
+def test_exports_every_declared_symbol(L):
+    names = header_functions()
+    assert len(names) >= 12
+    for n in names:
+        assert hasattr(L, n), n
+    assert set(names) == set(zo.EXPORTS)
+
+
+def test_version_and_strings(L):
+    assert zo.version() == 10000
+    for s in (0, -1, -2, -3, -4, -5, -6, -7):
+        assert zo.status_string(s).startswith("ZO_")
+    assert "unknown" in zo.status_string(99)
+    assert L.zo_last_cuda_error() == b""
+
+
+def tensors(*specs):
+    arr = (zo.zo_tensor * len(specs))()
+    for i, (ptr, numel, dtype) in enumerate(specs):
+        arr[i].ptr, arr[i].numel, arr[i].dtype, arr[i].reserved = ptr, numel, dtype, 0
+    return arr
+
+
+FAKE = 0x7F0000000000  # never dereferenced: validation rejects first
+
+
+def test_perturb_validation(L):
+    ok = tensors((FAKE, 16, 1))
+    assert L.zo_perturb(ok, -1, 1, 0, 1e-3, None) == zo.ZO_ERR_ARG
+    assert L.zo_perturb(None, 1, 1, 0, 1e-3, None) == zo.ZO_ERR_ARG
+    assert L.zo_perturb(tensors((FAKE, 16, 3)), 1, 1, 0, 1e-3, None) == zo.ZO_ERR_DTYPE
+    assert L.zo_perturb(tensors((FAKE + 1, 16, 1)), 1, 1, 0, 1e-3, None) == zo.ZO_ERR_ALIGN
+    assert L.zo_perturb(tensors((FAKE + 2, 16, 0)), 1, 1, 0, 1e-3, None) == zo.ZO_ERR_ALIGN
+    assert L.zo_perturb(tensors((0, 16, 1)), 1, 1, 0, 1e-3, None) == zo.ZO_ERR_ARG
+    assert L.zo_perturb(tensors((FAKE, -1, 1)), 1, 1, 0, 1e-3, None) == zo.ZO_ERR_ARG
+    assert L.zo_perturb(ok, 1, 1, 0, float("nan"), None) == zo.ZO_ERR_ARG
+    assert L.zo_perturb(ok, 1, 1, 0, float("inf"), None) == zo.ZO_ERR_ARG
+    bad_res = tensors((FAKE, 16, 1))
+    bad_res[0].reserved = 1
+    assert L.zo_perturb(bad_res, 1, 1, 0, 1e-3, None) == zo.ZO_ERR_ARG
+    assert L.zo_perturb(None, 0, 1, 0, 1e-3, None) == zo.ZO_OK  # empty list: nothing to do
+
+
+def test_update_validation(L):
+    ok = tensors((FAKE, 16, 1))
+    c = ctypes.c_void_p(FAKE)
+    for fn in (L.zo_update, L.zo_update_sequential):
+        assert fn(ok, 1, 1, c, 0, 1e-3, None, None) == zo.ZO_ERR_ARG
+        assert fn(ok, 1, 1, c, zo.ZO_MAX_PROBES + 1, 1e-3, None, None) == zo.ZO_ERR_TOO_MANY_PROBES
+        assert fn(ok, 1, 1, None, 4, 1e-3, None, None) == zo.ZO_ERR_ARG
+        assert fn(ok, 1, 1, c, 4, float("nan"), None, None) == zo.ZO_ERR_ARG
+        assert fn(tensors((FAKE, 16, 9)), 1, 1, c, 4, 1e-3, None, None) == zo.ZO_ERR_DTYPE
+        assert fn(None, 0, 1, c, 4, 1e-3, None, None) == zo.ZO_OK
+
+
+def test_precondition_validation(L):
+    p = ctypes.c_void_p(FAKE)
+    f = L.zo_precondition_ex
+    assert f(p, 0, 1e-3, 0.1, 1.0, 0, p, None, None, p, None) == zo.ZO_ERR_ARG
+    assert f(p, zo.ZO_MAX_PROBES + 1, 1e-3, 0.1, 1.0, 0, p, None, None, p, None) == zo.ZO_ERR_TOO_MANY_PROBES
+    assert f(p, 4, 0.0, 0.1, 1.0, 0, p, None, None, p, None) == zo.ZO_ERR_ARG
+    assert f(p, 4, float("inf"), 0.1, 1.0, 0, p, None, None, p, None) == zo.ZO_ERR_ARG
+    assert f(p, 4, 1e-3, -0.1, 1.0, 0, p, None, None, p, None) == zo.ZO_ERR_ARG
+    assert f(p, 4, 1e-3, 1.5, 1.0, 0, p, None, None, p, None) == zo.ZO_ERR_ARG
+    assert f(p, 4, 1e-3, 0.1, 0.0, 0, p, None, None, p, None) == zo.ZO_ERR_ARG
+    assert f(None, 4, 1e-3, 0.1, 1.0, 0, p, None, None, p, None) == zo.ZO_ERR_ARG
+    assert f(p, 4, 1e-3, 0.1, 1.0, 0, None, None, None, p, None) == zo.ZO_ERR_ARG
+    assert f(p, 4, 1e-3, 0.1, 1.0, 0, p, None, None, None, None) == zo.ZO_ERR_ARG
+    assert L.zo_precondition(p, 0, 1e-3, p, p, None) == zo.ZO_ERR_ARG
+
+
+def test_probe_view_and_loss_validation(L):
+    p = ctypes.c_void_p(FAKE)
+    assert L.zo_probe_bytes(1, 0, -1, 4, p, None) == zo.ZO_ERR_ARG
+    assert L.zo_probe_bytes(1, 0, 0, -4, p, None) == zo.ZO_ERR_ARG
+    assert L.zo_probe_bytes(1, 0, 0, 4, None, None) == zo.ZO_ERR_ARG
+    assert L.zo_probe_bytes(1, 0, 0, 0, None, None) == zo.ZO_OK
+    assert L.zo_probe_signs(1, 0, 0, -1, p, None) == zo.ZO_ERR_ARG
+    assert L.zo_probe_signs(1, 0, 0, 0, None, None) == zo.ZO_OK
+    ws = L.zo_quadratic_loss_workspace_size(1 << 20)
+    assert ws > 0
+    assert L.zo_quadratic_loss(p, p, -1, p, p, ws, None) == zo.ZO_ERR_ARG
+    assert L.zo_quadratic_loss(p, p, 16, None, p, ws, None) == zo.ZO_ERR_ARG
+    assert L.zo_quadratic_loss(p, p, 16, p, None, ws, None) == zo.ZO_ERR_WORKSPACE
+    assert L.zo_quadratic_loss(p, p, 16, p, p, ws - 8, None) == zo.ZO_ERR_WORKSPACE
+
+
+def test_binding_rejects_cpu_tensors():
+    import torch
+    with pytest.raises(TypeError):
+        zo.ParamList([torch.zeros(4)])

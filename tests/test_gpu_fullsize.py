@@ -1,0 +1,104 @@
+"""Parity at the full parameter-set sizes (OPT-1.3B/13B/30B- and Qwen3-8B-
+shaped), through the same ParamList / zo_perturb / zo_precondition /
+zo_update calls the benchmark times. The oracle recomputes sampled elements
+one by one (the generator is counter-based): every tensor's first and last 16
+elements plus 2^16 elements drawn uniformly over the whole set."""
+import gc
+
+import numpy as np
+import pytest
+import torch
+
+import oracle
+from paper_2609_38095_gb300 import build as zo_build
+from paper_2609_38095_gb300 import workloads as W
+from paper_2609_38095_gb300 import zo
+
+from gpu_helpers import assert_update_close, storage_bits
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _built():
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    zo_build.build()
+    oracle.lib()
+
+
+def sample_positions(numels, n_random=1 << 16, seed=0):
+    """(tensor index, element index) pairs: ends of every tensor + uniform."""
+    numels = np.asarray(numels, dtype=np.int64)
+    cum = np.concatenate([[0], np.cumsum(numels)])
+    rng = np.random.default_rng(seed)
+    flat = rng.integers(0, cum[-1], n_random)
+    t_r = np.searchsorted(cum, flat, side="right") - 1
+    i_r = flat - cum[t_r]
+    ts, is_ = [t_r], [i_r]
+    for t, n in enumerate(numels):
+        if n == 0:
+            continue
+        e = np.unique(np.concatenate([np.arange(min(16, n)), np.arange(max(0, n - 16), n)]))
+        ts.append(np.full(e.size, t))
+        is_.append(e)
+    t_all = np.concatenate(ts)
+    i_all = np.concatenate(is_)
+    order = np.lexsort((i_all, t_all))
+    return t_all[order], i_all[order]
+
+
+def gather(params, t_idx, i_idx):
+    """Storage bits and fp32 values of the sampled elements."""
+    out_bits, out_f32 = [], []
+    bounds = np.flatnonzero(np.diff(np.concatenate([[-1], t_idx, [len(params)]])))
+    for a, b in zip(bounds[:-1], bounds[1:]):
+        t = int(t_idx[a])
+        idx = torch.from_numpy(i_idx[a:b]).to(params[t].device)
+        v = params[t][idx]
+        out_f32.append(v.float().cpu().numpy())
+        out_bits.append(storage_bits(v))
+    return np.concatenate(out_bits), np.concatenate(out_f32)
+
+
+@pytest.mark.parametrize("key", ["opt-1.3b", "qwen3-8b", "opt-13b", "opt-30b"])
+def test_fullsize_sampled_parity(key):
+    ps = W.BY_KEY[key]
+    free, _ = torch.cuda.mem_get_info()
+    if free < ps.d * ps.bytes_per_elem * 1.1:
+        pytest.skip(f"needs {ps.d * ps.bytes_per_elem / 1e9:.0f} GB of device memory")
+    params = W.allocate_params(ps)
+    try:
+        plist = zo.ParamList(params)
+        S = oracle.virtual_offsets(ps.numels)
+        t_idx, i_idx = sample_positions(ps.numels)
+        g = (S[t_idx] + i_idx).astype(np.uint64)
+        seed, K, eps = W.step_seed(0), ps.K, ps.eps
+        k = K - 1
+
+        # perturb +eps with the last probe (highest probe group): bit-exact
+        bits0, f0 = gather(params, t_idx, i_idx)
+        zo.perturb(plist, seed, k, eps)
+        bits1, f1 = gather(params, t_idx, i_idx)
+        want = oracle.perturb_elements(ps.dtype, g, f0, seed, k, eps)
+        np.testing.assert_array_equal(bits1, want)
+        assert np.mean(bits1 != bits0) > 0.5
+
+        # preconditioner on the seeded loss triples
+        L = W.synthetic_losses(K, step=0)
+        c, st = zo.precondition(torch.tensor(L, device="cuda"), eps)
+        rc, c_o, _, _ = oracle.precondition(L, eps)
+        assert rc == oracle.OK and int(st.item()) == zo.ZO_OK
+        c_h = c.cpu().numpy()
+        np.testing.assert_allclose(c_h, c_o, rtol=1e-6)
+
+        # fused K-probe update with lr = eps (tied, as in the paper)
+        zo.update(plist, seed, c, eps, status=st)
+        bits2, _ = gather(params, t_idx, i_idx)
+        want2 = oracle.update_elements(ps.dtype, g, f1, seed, c_h, eps)
+        assert_update_close(bits2, want2, ps.dtype, c_h, eps, context=key)
+        assert np.mean(bits2 == want2) > 0.95
+    finally:
+        del params
+        gc.collect()
+        torch.cuda.empty_cache()

@@ -1,0 +1,323 @@
+"""GPU parity: every entry point of libzo.so, called through the C ABI, against
+the CPU oracle on the same seeded inputs, element by element.
+
+Bars: probe bytes / signs and perturb bit-exact; the fused update within one
+ulp of the storage dtype for bf16/fp16 and within the derived fp32 bound for
+fp32 storage; the preconditioner within 1e-6 relative; the quadratic loss
+within 1e-12 relative.
+"""
+import numpy as np
+import pytest
+import torch
+
+import oracle
+from paper_2609_38095_gb300 import build as zo_build
+from paper_2609_38095_gb300 import workloads as W
+from paper_2609_38095_gb300 import zo
+
+from gpu_helpers import (TORCH_TO_DT, assert_update_close, storage_bits, storage_np, to_torch, ulp_distance16)
+
+pytestmark = pytest.mark.gpu
+
+DTS = [torch.float32, torch.bfloat16, torch.float16]
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _built():
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    zo_build.build()
+    oracle.lib()
+
+
+def make_list(numels, dtypes, seed=0):
+    rng = np.random.default_rng(seed)
+    host = [W.random_storage(rng, n, TORCH_TO_DT[dt]) for n, dt in zip(numels, dtypes)]
+    dev = [to_torch(h, dt) for h, dt in zip(host, dtypes)]
+    return host, dev
+
+
+MIXED_NUMELS = [1, 15, 16, 17, 31, 33, 0, 255, 4096, 4099, 100003, 7, 65536 + 5]
+MIXED_DTYPES = [DTS[i % 3] for i in range(len(MIXED_NUMELS))]
+
+
+def assert_storage_equal(dev, host, what=""):
+    for i, (d, h) in enumerate(zip(dev, host)):
+        got = storage_np(d)
+        assert got.dtype == h.dtype
+        np.testing.assert_array_equal(got.view(np.uint32 if h.dtype == np.float32 else np.uint16),
+                                      h.view(np.uint32 if h.dtype == np.float32 else np.uint16),
+                                      err_msg=f"{what} tensor {i} numel {h.size}")
+
+
+# -------------------------------------------------------------- probe views
+@pytest.mark.parametrize("seed", [W.step_seed(0), 0xFFFFFFFFFFFFFFFF, 0])
+@pytest.mark.parametrize("probe", [0, 7, 8, 255, 1023, 5000])
+@pytest.mark.parametrize("first,n", [(0, 4096), (3, 1001), (2**33 + 5, 777)])
+def test_probe_bytes_bit_exact(seed, probe, first, n):
+    got = zo.probe_bytes(seed, probe, first, n).cpu().numpy()
+    want = oracle.probe_bytes(seed, probe, first, n)
+    np.testing.assert_array_equal(got, want)
+
+
+@pytest.mark.parametrize("seed", [W.step_seed(3), 0xFFFFFFFFFFFFFFFF])
+@pytest.mark.parametrize("probe", [0, 5, 9, 1023])
+@pytest.mark.parametrize("first,n", [(0, 5000), (13, 333), (2**36 + 1, 1000)])
+def test_probe_signs_bit_exact(seed, probe, first, n):
+    got = zo.probe_signs(seed, probe, first, n).cpu().numpy()
+    want = oracle.probe_signs(seed, probe, first, n)
+    np.testing.assert_array_equal(got, want)
+
+
+# ------------------------------------------------------------------ perturb
+def test_perturb_bit_exact_mixed_sequence():
+    host, dev = make_list(MIXED_NUMELS, MIXED_DTYPES)
+    plist = zo.ParamList(dev)
+    dts = [TORCH_TO_DT[d] for d in MIXED_DTYPES]
+    seed, eps = W.step_seed(1), 1e-3
+    for k in (0, 5, 8, 13):
+        for s in (eps, -2 * eps, eps):
+            zo.perturb(plist, seed, k, s)
+            oracle.perturb(host, dts, seed, k, s)
+            assert_storage_equal(dev, host, f"probe {k} scale {s}")
+
+
+@pytest.mark.parametrize("scale", [0.5, -3e-8, 0.0, 1e4])
+def test_perturb_bit_exact_scales(scale):
+    host, dev = make_list(MIXED_NUMELS, MIXED_DTYPES, seed=4)
+    zo.perturb(dev, W.step_seed(9), 3, scale)
+    oracle.perturb(host, [TORCH_TO_DT[d] for d in MIXED_DTYPES], W.step_seed(9), 3, scale)
+    assert_storage_equal(dev, host, f"scale {scale}")
+
+
+@pytest.mark.parametrize("dtype", DTS)
+@pytest.mark.parametrize("offset", [1, 2, 4, 8, 16])
+def test_perturb_unaligned_views(dtype, offset):
+    """Views at element offsets that break 32-byte alignment take the
+    element-wise path; results are identical."""
+    rng = np.random.default_rng(offset)
+    n = 4096 + 37
+    base_host = W.random_storage(rng, n + offset + 64, TORCH_TO_DT[dtype])
+    base = to_torch(base_host, dtype)
+    view = base[offset:offset + n]
+    host = [base_host[offset:offset + n].copy()]
+    zo.perturb([view], W.step_seed(2), 11, 1e-3)
+    oracle.perturb(host, [TORCH_TO_DT[dtype]], W.step_seed(2), 11, 1e-3)
+    assert_storage_equal([view], host, f"offset {offset}")
+    # everything outside the view is untouched
+    after = storage_np(base)
+    np.testing.assert_array_equal(after[:offset], base_host[:offset])
+    np.testing.assert_array_equal(after[offset + n:], base_host[offset + n:])
+
+
+def test_perturb_many_tensors_split_launches():
+    """More tensors than one launch's table holds (1024)."""
+    rng = np.random.default_rng(12)
+    numels = [int(x) for x in rng.integers(0, 300, 2500)]
+    dtypes = [DTS[int(x)] for x in rng.integers(0, 3, 2500)]
+    host, dev = make_list(numels, dtypes, seed=12)
+    dts = [TORCH_TO_DT[d] for d in dtypes]
+    zo.perturb(dev, W.step_seed(5), 17, -2e-3)
+    oracle.perturb(host, dts, W.step_seed(5), 17, -2e-3)
+    assert_storage_equal(dev, host)
+    c = torch.tensor(rng.normal(0, 20, 9), dtype=torch.float64, device="cuda")
+    zo.update(dev, W.step_seed(5), c, 1e-3)
+    oracle.update(host, dts, W.step_seed(5), c.cpu().numpy(), 1e-3)
+    for d, h, dt in zip(dev, host, dts):
+        assert_update_close(storage_bits(d), storage_bits(h), dt, c.cpu().numpy(), 1e-3)
+
+
+def test_guard_bands_untouched():
+    """Tensors carved out of one buffer with canaries between them."""
+    numels = [17, 4096, 33, 1000]
+    gap = 64
+    total = sum(numels) + gap * (len(numels) + 1)
+    buf = torch.full((total,), 7.0, dtype=torch.bfloat16, device="cuda")
+    views, pos = [], gap
+    for n in numels:
+        views.append(buf[pos:pos + n])
+        pos += n + gap
+    for v in views:
+        v.normal_(0, 0.02)
+    canary_mask = torch.ones(total, dtype=torch.bool)
+    pos = gap
+    for n in numels:
+        canary_mask[pos:pos + n] = False
+        pos += n + gap
+    zo.perturb(views, W.step_seed(0), 1, 1e-3)
+    c = torch.linspace(-30, 30, 37, dtype=torch.float64, device="cuda")
+    zo.update(views, W.step_seed(0), c, 1e-3)
+    zo.update_sequential(views, W.step_seed(0), c[:5].contiguous(), 1e-3)
+    assert torch.all(buf.cpu()[canary_mask] == 7.0)
+
+
+def test_empty_and_zero_length():
+    zo.perturb([], 1, 0, 1e-3)
+    zo.update([], 1, torch.ones(3, dtype=torch.float64, device="cuda"), 1e-3)
+    z = torch.empty(0, dtype=torch.bfloat16, device="cuda")
+    host, dev = make_list([0, 5, 0], [torch.bfloat16] * 3)
+    zo.perturb([z] + dev, 1, 0, 1e-3)
+    oracle.perturb([np.zeros(0, np.uint16)] + host, [W.DT_BF16] * 4, 1, 0, 1e-3)
+    assert_storage_equal(dev, host)
+
+
+# ------------------------------------------------------------------- update
+@pytest.mark.parametrize("K", [1, 3, 8, 13, 64, 256])
+def test_update_within_tolerance(K):
+    host, dev = make_list(MIXED_NUMELS, MIXED_DTYPES, seed=K)
+    dts = [TORCH_TO_DT[d] for d in MIXED_DTYPES]
+    rng = np.random.default_rng(100 + K)
+    c_np = rng.normal(0, 25, K)
+    c = torch.tensor(c_np, dtype=torch.float64, device="cuda")
+    lr, seed = 1e-3, W.step_seed(K)
+    zo.update(dev, seed, c, lr)
+    oracle.update(host, dts, seed, c_np, lr)
+    equal = total = 0
+    for i, (d, h, dt) in enumerate(zip(dev, host, dts)):
+        gb, wb = storage_bits(d), storage_bits(h)
+        assert_update_close(gb, wb, dt, c_np, lr, context=f"K={K} tensor {i}")
+        if dt != W.DT_F32:   # 16-bit results are almost always the oracle's exactly
+            equal += int(np.sum(gb == wb))
+            total += gb.size
+    assert equal >= 0.95 * total
+
+
+def test_update_max_probes():
+    K = zo.ZO_MAX_PROBES
+    host, dev = make_list([5003, 16, 1], [torch.float32, torch.bfloat16, torch.float16], seed=77)
+    dts = [W.DT_F32, W.DT_BF16, W.DT_F16]
+    c_np = np.random.default_rng(77).normal(0, 5, K)
+    c = torch.tensor(c_np, device="cuda")
+    zo.update(dev, W.step_seed(77), c, 1e-2)
+    oracle.update(host, dts, W.step_seed(77), c_np, 1e-2)
+    for d, h, dt in zip(dev, host, dts):
+        assert_update_close(storage_bits(d), storage_bits(h), dt, c_np, 1e-2)
+    with pytest.raises(zo.ZoError) as e:
+        zo.update(dev, 1, torch.ones(K + 1, dtype=torch.float64, device="cuda"), 1e-3)
+    assert e.value.status == zo.ZO_ERR_TOO_MANY_PROBES
+
+
+@pytest.mark.parametrize("K", [1, 5, 16])
+def test_update_sequential_bit_exact(K):
+    host, dev = make_list(MIXED_NUMELS, MIXED_DTYPES, seed=50 + K)
+    dts = [TORCH_TO_DT[d] for d in MIXED_DTYPES]
+    c_np = np.random.default_rng(K).normal(0, 25, K)
+    c = torch.tensor(c_np, device="cuda")
+    zo.update_sequential(dev, W.step_seed(K), c, 2e-3)
+    oracle.update_sequential(host, dts, W.step_seed(K), c_np, 2e-3)
+    assert_storage_equal(dev, host)
+
+
+def test_update_K1_is_a_perturb_fp32():
+    host, dev = make_list([70001], [torch.float32], seed=8)
+    c = torch.tensor([3.25], dtype=torch.float64, device="cuda")
+    d2 = [dev[0].clone()]
+    zo.update(dev, W.step_seed(8), c, 1e-3)
+    a0 = float(np.float32(-(1e-3 / 1) * 3.25))
+    zo.perturb(d2, W.step_seed(8), 0, a0)
+    assert torch.equal(dev[0], d2[0])
+
+
+# ------------------------------------------------------------ precondition
+def crafted_losses():
+    rows = [[2.5, 2.5, 2.5], [2.5 + 1e-7, 2.5, 2.5], [3.04, 2.98, 3.0], [2.98, 2.96, 3.0],
+            [50.0, 50.0, 0.0], [1.0, -1.0, 0.0], [0.0, 0.0, 1e-3]]
+    return np.array(rows, dtype=np.float64)
+
+
+@pytest.mark.parametrize("K", [1, 7, 16, 256, 1024])
+@pytest.mark.parametrize("alpha,lam,one_sided", [(0.1, 1.0, False), (0.0, 1.0, False), (1.0, 1.0, False),
+                                                 (0.5, 3.0, False), (0.1, 1.0, True)])
+def test_precondition_vs_oracle(K, alpha, lam, one_sided):
+    L = W.synthetic_losses(K, step=K)
+    cr = crafted_losses()
+    L[: min(K, len(cr))] = cr[: min(K, len(cr))]
+    eps = 1e-3
+    Ld = torch.tensor(L, device="cuda")
+    c, st, w, cv = zo.precondition(Ld, eps, alpha=alpha, lambda_reg=lam, one_sided=one_sided, with_weights=True)
+    rc, c_o, w_o, cv_o = oracle.precondition(L, eps, alpha=alpha, lambda_reg=lam, one_sided=one_sided)
+    assert rc == oracle.OK and int(st.item()) == zo.ZO_OK
+    for got, want in ((c, c_o), (w, w_o), (cv, cv_o)):
+        g = got.cpu().numpy()
+        np.testing.assert_allclose(g, want, rtol=1e-6, atol=0)
+        np.testing.assert_allclose(g, want, rtol=1e-13, atol=1e-300)
+
+
+@pytest.mark.parametrize("bad", [np.nan, np.inf])
+def test_precondition_nonfinite_blocks_update(bad):
+    L = W.synthetic_losses(16, 0)
+    L[5, 1] = bad
+    Ld = torch.tensor(L, device="cuda")
+    sentinel = torch.full((16,), 123.0, dtype=torch.float64, device="cuda")
+    status = torch.zeros(1, dtype=torch.int32, device="cuda")
+    c, st = zo.precondition(Ld, 1e-3, out=(sentinel, status))
+    assert int(st.item()) == zo.ZO_ERR_NONFINITE
+    assert torch.all(sentinel == 123.0)
+    host, dev = make_list([1000], [torch.bfloat16])
+    before = storage_np(dev[0])
+    zo.update(dev, 1, c, 1e-3, status=st)
+    zo.update_sequential(dev, 1, c, 1e-3, status=st)
+    np.testing.assert_array_equal(storage_np(dev[0]), before)
+    # a clean call resets the status and the update proceeds
+    c2, st2 = zo.precondition(torch.tensor(W.synthetic_losses(16, 0), device="cuda"), 1e-3, out=(sentinel, status))
+    assert int(st2.item()) == zo.ZO_OK
+    zo.update(dev, 1, c2, 1e-3, status=st2)
+    assert not np.array_equal(storage_np(dev[0]), before)
+
+
+# --------------------------------------------------------------------- loss
+@pytest.mark.parametrize("n", [0, 1, 1000, 1 << 20, (1 << 20) + 7, 3_000_001])
+def test_quadratic_loss(n):
+    th = W.tiny_theta(n) if n else np.zeros(0, np.float32)
+    a = W.tiny_curvatures(n) if n else np.zeros(0, np.float32)
+    td, ad = torch.from_numpy(th).cuda(), torch.from_numpy(a).cuda()
+    got = zo.quadratic_loss(td, ad).item()
+    want = oracle.quadratic_loss(th, a)
+    assert got == pytest.approx(want, rel=1e-12, abs=0)
+    assert zo.quadratic_loss(td, ad).item() == got   # fixed order: reproducible
+
+
+# ------------------------------------------------------- small workload, e2e
+def test_tiny_workload_lockstep():
+    """Ten full steps of the small workload (d = 2^20 fp32, quadratic loss,
+    K = 8, eps = 1e-3, lr = 1e-2). Each step starts the oracle from the GPU's
+    weights and compares every loss, coefficient and the updated weights."""
+    ps = W.TINY
+    th0, a = W.tiny_theta(), W.tiny_curvatures()
+    theta = torch.from_numpy(th0).cuda()
+    ad = torch.from_numpy(a).cuda()
+    plist = zo.ParamList([theta])
+    K, eps, lr = ps.K, ps.eps, W.TINY_LR
+    losses = torch.empty(K, 3, dtype=torch.float64, device="cuda")
+    ws = torch.empty(zo.quadratic_loss_workspace_size(theta.numel()), dtype=torch.uint8, device="cuda")
+    for step in range(W.TINY_STEPS):
+        seed = W.step_seed(step)
+        host = [theta.cpu().numpy().copy()]
+        # GPU step: the center loss first, once (Algorithm 1), then the probes
+        l0 = zo.quadratic_loss(theta, ad, workspace=ws)
+        for k in range(K):
+            zo.perturb(plist, seed, k, eps)
+            zo.quadratic_loss(theta, ad, out=losses[k, 0:1], workspace=ws)
+            zo.perturb(plist, seed, k, -2 * eps)
+            zo.quadratic_loss(theta, ad, out=losses[k, 1:2], workspace=ws)
+            zo.perturb(plist, seed, k, eps)
+        losses[:, 2] = l0
+        c, st = zo.precondition(losses, eps)
+        zo.update(plist, seed, c, lr, status=st)
+        # oracle step from the same starting weights
+        rows = []
+        l0_o = oracle.quadratic_loss(host[0], a)
+        for k in range(K):
+            oracle.perturb(host, [W.DT_F32], seed, k, eps)
+            lp = oracle.quadratic_loss(host[0], a)
+            oracle.perturb(host, [W.DT_F32], seed, k, -2 * eps)
+            lm = oracle.quadratic_loss(host[0], a)
+            oracle.perturb(host, [W.DT_F32], seed, k, eps)
+            rows.append([lp, lm, l0_o])
+        rc, c_o, _, _ = oracle.precondition(rows, eps)
+        assert rc == oracle.OK and int(st.item()) == zo.ZO_OK
+        np.testing.assert_allclose(losses.cpu().numpy(), np.array(rows), rtol=1e-12)
+        np.testing.assert_allclose(c.cpu().numpy(), c_o, rtol=1e-6)
+        oracle.update(host, [W.DT_F32], seed, c.cpu().numpy(), lr)
+        assert_update_close(storage_bits(theta), storage_bits(host[0]), W.DT_F32, c.cpu().numpy(), lr,
+                            context=f"step {step}")
