@@ -185,6 +185,29 @@ int64_t zo_quadratic_loss_workspace_size(int64_t n);
 int zo_quadratic_loss(const float* theta, const float* a, int64_t n, double* out, void* workspace,
                       int64_t workspace_bytes, void* stream);
 
+/* ---------------------------------------------------------------------------
+ * zo_quadratic_loss_static -- zo_quadratic_loss for callers that cannot
+ * allocate device memory. The paper has no counterpart: it exists for code
+ * that runs inside a device-memory budget fixed in advance (for example a
+ * framework whose caching allocator already holds the device memory, where
+ * an extra cudaMalloc fails) or that must not let an allocation synchronise
+ * the device (cudaMalloc and cudaFree may). It computes the same value as
+ * zo_quadratic_loss without a workspace argument: its scratch is a fixed
+ * 32 KB array inside the library, held by every device that loads the
+ * library until the process exits. The call allocates nothing.
+ *   n     0 .. ZO_QUADRATIC_LOSS_STATIC_MAX_N elements; larger n returns
+ *         ZO_ERR_WORKSPACE (the fixed scratch holds one partial sum per 2048
+ *         elements) and enqueues nothing.
+ * The first call on a device looks up the array's device address (once per
+ * device, with that device current); make that first call before any stream
+ * capture. All calls share the array: calls that overlap on the GPU (other
+ * streams, other host threads on the same device) race and must be ordered
+ * by the caller. Nothing in it needs clearing between calls.
+ * Errors: ZO_ERR_ARG, ZO_ERR_WORKSPACE, ZO_ERR_CUDA.
+ * ------------------------------------------------------------------------- */
+#define ZO_QUADRATIC_LOSS_STATIC_MAX_N 8388608
+int zo_quadratic_loss_static(const float* theta, const float* a, int64_t n, double* out, void* stream);
+
 #ifdef __cplusplus
 }
 #endif

@@ -318,4 +318,13 @@ int zo_quadratic_loss(const float* theta, const float* a, int64_t n, double* out
   return e == cudaSuccess ? ZO_OK : cuda_fail(e, "quadratic_loss");
 }
 
+int zo_quadratic_loss_static(const float* theta, const float* a, int64_t n, double* out, void* stream) {
+  if (n < 0 || out == nullptr || (n > 0 && (theta == nullptr || a == nullptr))) return ZO_ERR_ARG;
+  if (n > ZO_QUADRATIC_LOSS_STATIC_MAX_N) return ZO_ERR_WORKSPACE;
+  static_assert(ZO_QUADRATIC_LOSS_STATIC_MAX_N == zo::kStaticLossPartials * zo::kStaticLossSlice,
+                "static scratch capacity and the documented limit must agree");
+  cudaError_t e = zo::launch_quadratic_loss_static(theta, a, n, out, static_cast<cudaStream_t>(stream));
+  return e == cudaSuccess ? ZO_OK : cuda_fail(e, "quadratic_loss_static");
+}
+
 }  // extern "C"

@@ -11,6 +11,8 @@ namespace zo {
 constexpr int kStatusNonFinite = -4;  // ZO_ERR_NONFINITE
 constexpr int kThreads = 256;         // threads per block of the streaming kernels
 constexpr int kMaxLossPartials = 2048;
+constexpr int kStaticLossPartials = 4096;   // fixed scratch of the allocation-free loss (32 KB)
+constexpr int64_t kStaticLossSlice = 2048;  // elements per partial in that variant
 
 cudaError_t launch_perturb(const PerturbParams& p, int grid, cudaStream_t stream);
 cudaError_t launch_update(const UpdateParams& p, int grid, cudaStream_t stream);
@@ -26,5 +28,7 @@ cudaError_t launch_precondition(const double* losses, int K, double eps, double 
                                 cudaStream_t stream);
 cudaError_t launch_quadratic_loss(const float* theta, const float* a, int64_t n, double* out, double* partial,
                                   int max_partials, int num_sms, cudaStream_t stream);
+cudaError_t launch_quadratic_loss_static(const float* theta, const float* a, int64_t n, double* out,
+                                         cudaStream_t stream);
 
 }  // namespace zo

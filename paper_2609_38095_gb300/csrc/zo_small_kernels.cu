@@ -1,5 +1,7 @@
 // zo_small_kernels.cu -- the probe-space preconditioner (Sec. 4.1, Eqs. 3-4)
 // and the fixed-order fp64 reduction behind the quadratic test loss.
+#include <mutex>
+
 #include <cuda_runtime.h>
 
 #include "zo_device.cuh"
@@ -98,6 +100,56 @@ cudaError_t launch_quadratic_loss(const float* theta, const float* a, int64_t n,
   int grid = static_cast<int>(want < 1 ? 1 : (want > cap ? cap : want));
   quad_loss_partial_kernel<<<grid, threads, 0, stream>>>(theta, a, n, partial);
   cudaError_t e = cudaGetLastError();
+  if (e != cudaSuccess) return e;
+  quad_loss_final_kernel<<<1, threads, 0, stream>>>(partial, grid, out);
+  return cudaGetLastError();
+}
+
+// ---------------------------------------------------------------------------
+// Allocation-free variant of the quadratic loss. The partial sums live in a
+// fixed array compiled into the library (every device that loads the library
+// holds it until the process exits) instead of a caller workspace. Host code
+// cannot use the array's name as a device address, so its address is looked
+// up once per device with cudaGetSymbolAddress, with that device current.
+// One partial per 2048-element slice: n <= kStaticLossPartials * 2048. Every
+// block overwrites its own partial before the final fold reads it, so nothing
+// needs clearing between calls; calls that overlap on the GPU share the array
+// and race.
+// ---------------------------------------------------------------------------
+static __device__ __align__(256) double g_static_loss_partials[kStaticLossPartials];
+
+namespace {
+constexpr int kStaticMaxDevices = 64;
+std::mutex g_static_mu;
+double* g_static_ptr[kStaticMaxDevices] = {};
+}  // namespace
+
+cudaError_t static_loss_scratch(double** out) {
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return e;
+  if (dev < 0 || dev >= kStaticMaxDevices) return cudaErrorInvalidDevice;
+  std::lock_guard<std::mutex> lock(g_static_mu);
+  if (g_static_ptr[dev] == nullptr) {
+    void* p = nullptr;
+    e = cudaGetSymbolAddress(&p, g_static_loss_partials);
+    if (e != cudaSuccess) return e;
+    g_static_ptr[dev] = static_cast<double*>(p);
+  }
+  *out = g_static_ptr[dev];
+  return cudaSuccess;
+}
+
+cudaError_t launch_quadratic_loss_static(const float* theta, const float* a, int64_t n, double* out,
+                                         cudaStream_t stream) {
+  double* partial = nullptr;
+  cudaError_t e = static_loss_scratch(&partial);
+  if (e != cudaSuccess) return e;
+  const int threads = 256;
+  const int64_t want = (n + kStaticLossSlice - 1) / kStaticLossSlice;
+  const int grid = static_cast<int>(want < 1 ? 1 : want);  // n is checked against the capacity by the caller
+  quad_loss_partial_kernel<<<grid, threads, 0, stream>>>(theta, a, n, partial);
+  e = cudaGetLastError();
   if (e != cudaSuccess) return e;
   quad_loss_final_kernel<<<1, threads, 0, stream>>>(partial, grid, out);
   return cudaGetLastError();

@@ -27,7 +27,8 @@ DTYPE_CODE = {torch.float32: 0, torch.bfloat16: 1, torch.float16: 2}
 
 EXPORTS = ["zo_status_string", "zo_last_cuda_error", "zo_version", "zo_perturb", "zo_precondition",
            "zo_precondition_ex", "zo_update", "zo_update_sequential", "zo_probe_bytes", "zo_probe_signs",
-           "zo_quadratic_loss_workspace_size", "zo_quadratic_loss"]
+           "zo_quadratic_loss_workspace_size", "zo_quadratic_loss", "zo_quadratic_loss_static"]
+ZO_QUADRATIC_LOSS_STATIC_MAX_N = 8388608
 
 
 class zo_tensor(ctypes.Structure):
@@ -69,6 +70,7 @@ def _lib():
             "zo_probe_signs": ([u64, u32, i64, i64, vp, vp], c.c_int),
             "zo_quadratic_loss_workspace_size": ([i64], i64),
             "zo_quadratic_loss": ([vp, vp, i64, vp, vp, i64, vp], c.c_int),
+            "zo_quadratic_loss_static": ([vp, vp, i64, vp, vp], c.c_int),
         }
         for name, (args, res) in sig.items():
             f = getattr(L, name)
@@ -240,4 +242,21 @@ def quadratic_loss(theta, a, out=None, workspace=None):
                                       ctypes.c_void_p(out.data_ptr()), ctypes.c_void_p(workspace.data_ptr()),
                                       workspace.numel(), _stream(dev))
     _check("zo_quadratic_loss", rc)
+    return out
+
+
+def quadratic_loss_static(theta, a, out=None):
+    """zo_quadratic_loss_static: the same loss with the library's fixed
+    scratch instead of a workspace (the call itself allocates nothing; pass
+    `out` to avoid the one allocation this wrapper would make)."""
+    n = theta.numel()
+    if a.numel() != n:
+        raise ValueError("theta and a differ in size")
+    dev = theta.device
+    if out is None:
+        out = torch.empty(1, dtype=torch.float64, device=dev)
+    with torch.cuda.device(dev):
+        rc = _lib().zo_quadratic_loss_static(_dev_ptr(theta, torch.float32, "theta"), _dev_ptr(a, torch.float32, "a"),
+                                             n, ctypes.c_void_p(out.data_ptr()), _stream(dev))
+    _check("zo_quadratic_loss_static", rc)
     return out

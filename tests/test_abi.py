@@ -116,3 +116,12 @@ def test_binding_rejects_cpu_tensors():
     import torch
     with pytest.raises(TypeError):
         zo.ParamList([torch.zeros(4)])
+
+
+def test_static_loss_validation(L):
+    p = ctypes.c_void_p(FAKE)
+    f = L.zo_quadratic_loss_static
+    assert f(p, p, -1, p, None) == zo.ZO_ERR_ARG
+    assert f(p, p, 16, None, None) == zo.ZO_ERR_ARG
+    assert f(None, p, 16, p, None) == zo.ZO_ERR_ARG
+    assert f(p, p, zo.ZO_QUADRATIC_LOSS_STATIC_MAX_N + 1, p, None) == zo.ZO_ERR_WORKSPACE
