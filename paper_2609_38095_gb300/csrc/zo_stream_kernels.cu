@@ -106,26 +106,60 @@ __global__ void __launch_bounds__(256) perturb_kernel(const __grid_constant__ Pe
 // element adds the two looked-up partials to its fp32 accumulator, quads in
 // increasing order: one shared-memory load and one add per four probes
 // instead of a select and an add per probe. Probes K..8*groups-1 have a = 0.
+//
+// Shared-memory layout: probe group q owns a 256-byte frame starting on a
+// 256-byte boundary of the shared window; bytes [0, 64) hold the table of
+// quad 2q, [64, 128) the table of quad 2q + 1. Masking a Philox word once
+// with 0x3C3C3C3C (after a shift by 2) leaves four nibble*4 offsets in its
+// four bytes; one byte-permute then splices an offset under the frame's
+// upper bytes, giving the lookup address in a single instruction.
 // ---------------------------------------------------------------------------
+constexpr uint32_t kFrameBytes = 256;
+
+__device__ __forceinline__ float lds_lo(uint32_t addr) {
+  float v;
+  asm volatile("ld.shared.f32 %0, [%1];" : "=f"(v) : "r"(addr));
+  return v;
+}
+
+__device__ __forceinline__ float lds_hi(uint32_t addr) {
+  float v;
+  asm volatile("ld.shared.f32 %0, [%1+64];" : "=f"(v) : "r"(addr));
+  return v;
+}
+
 __device__ __forceinline__ void accumulate_block(float (&acc)[16], int64_t b, const UpdateParams& P,
-                                                 const float* __restrict__ lut) {
+                                                 uint32_t lut_base) {
   const uint32_t blo = static_cast<uint32_t>(b), bhi = static_cast<uint32_t>(static_cast<uint64_t>(b) >> 32);
-  for (int q = 0; q < P.groups; ++q) {
+  uint32_t frame = lut_base;
+  for (int q = 0; q < P.groups; ++q, frame += kFrameBytes) {
     const uint4 x = philox10(blo, bhi, static_cast<uint32_t>(q), 0u, P.keys);
-    const float* tlo = lut + 32 * q;
-    const float* thi = tlo + 16;
 #pragma unroll
-    for (int m = 0; m < 16; ++m) {
-      const uint32_t byte = (word_of(x, m >> 2) >> (8 * (m & 3))) & 0xFFu;
-      acc[m] = __fadd_rn(acc[m], tlo[byte & 0xFu]);
-      acc[m] = __fadd_rn(acc[m], thi[byte >> 4]);
+    for (int m = 0; m < 4; ++m) {
+      const uint32_t w = word_of(x, m);
+      const uint32_t lo4 = (w << 2) & 0x3C3C3C3Cu;  // byte j: 4 * low nibble of byte j of w
+      const uint32_t hi4 = (w >> 2) & 0x3C3C3C3Cu;  // byte j: 4 * high nibble of byte j of w
+#pragma unroll
+      for (int j = 0; j < 4; ++j) {
+        const uint32_t sel = 0x7650u | static_cast<uint32_t>(j);  // byte j of the offsets, bytes 1-3 of the frame
+        const float tlo = lds_lo(__byte_perm(lo4, frame, sel));
+        const float thi = lds_hi(__byte_perm(hi4, frame, sel));
+        acc[4 * m + j] = __fadd_rn(__fadd_rn(acc[4 * m + j], tlo), thi);
+      }
     }
   }
 }
 
+// One full, 32-byte aligned block: theta is loaded before the probe loop so
+// the load overlaps the arithmetic.
 template <uint8_t DT>
-__device__ __forceinline__ void apply_block_vec(void* base, int64_t e0, const float (&acc)[16]) {
+__device__ __forceinline__ void update_block_vec(void* base, int64_t e0, int64_t b, const UpdateParams& P,
+                                                 uint32_t lut_base) {
+  float acc[16];
+#pragma unroll
+  for (int m = 0; m < 16; ++m) acc[m] = 0.0f;
   if constexpr (DT == kF32) {
+    accumulate_block(acc, b, P, lut_base);
     float* p = static_cast<float*>(base) + e0;
 #pragma unroll
     for (int half = 0; half < 2; ++half) {
@@ -139,6 +173,7 @@ __device__ __forceinline__ void apply_block_vec(void* base, int64_t e0, const fl
     uint16_t* p = static_cast<uint16_t*>(base) + e0;
     uint32_t v[8];
     ld256(p, v);
+    accumulate_block(acc, b, P, lut_base);
 #pragma unroll
     for (int r = 0; r < 8; ++r) {
       const float2 f = unpack2<DT>(v[r]);
@@ -149,9 +184,11 @@ __device__ __forceinline__ void apply_block_vec(void* base, int64_t e0, const fl
 }
 
 __global__ void __launch_bounds__(256) update_kernel(const __grid_constant__ UpdateParams P) {
-  extern __shared__ float smem[];
-  float* a_s = smem;                 // 8 * groups coefficients (zero padded)
-  float* lut = smem + 8 * P.groups;  // 2 * groups tables of 16 partial sums
+  extern __shared__ __align__(16) unsigned char smem[];
+  float* a_s = reinterpret_cast<float*>(smem);  // 8 * groups coefficients (zero padded)
+  const uint32_t smem_sh = static_cast<uint32_t>(__cvta_generic_to_shared(smem));
+  const uint32_t lut_base = (smem_sh + 32u * P.groups + kFrameBytes - 1) & ~(kFrameBytes - 1);
+  float* lut = reinterpret_cast<float*>(smem + (lut_base - smem_sh));  // generic view of the frames
   __shared__ int skip;
   if (threadIdx.x == 0) skip = (P.status != nullptr && *P.status != 0);
   const int npad = 8 * P.groups;
@@ -166,7 +203,7 @@ __global__ void __launch_bounds__(256) update_kernel(const __grid_constant__ Upd
     s = __fadd_rn(s, (n & 2) ? a[1] : -a[1]);
     s = __fadd_rn(s, (n & 4) ? a[2] : -a[2]);
     s = __fadd_rn(s, (n & 8) ? a[3] : -a[3]);
-    lut[e] = s;
+    lut[(h >> 1) * (kFrameBytes / 4) + (h & 1) * 16 + n] = s;
   }
   __syncthreads();
 
@@ -177,10 +214,6 @@ __global__ void __launch_bounds__(256) update_kernel(const __grid_constant__ Upd
   for (int64_t b = tab.blk_begin + static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; b < blk_total;
        b += stride) {
     t = advance_tensor(tab, t, b);
-    float acc[16];
-#pragma unroll
-    for (int m = 0; m < 16; ++m) acc[m] = 0.0f;
-    accumulate_block(acc, b, P, lut);
     const int64_t e0 = (b - tensor_blk_begin(tab, t)) * 16;
     const int64_t cnt = min(static_cast<int64_t>(16), tab.numel[t] - e0);
     const uint8_t fl = tab.flags[t];
@@ -188,12 +221,16 @@ __global__ void __launch_bounds__(256) update_kernel(const __grid_constant__ Upd
     void* base = reinterpret_cast<void*>(tab.ptr[t]);
     if (cnt == 16 && (fl & kVec32)) {
       if (dt == kBF16)
-        apply_block_vec<kBF16>(base, e0, acc);
+        update_block_vec<kBF16>(base, e0, b, P, lut_base);
       else if (dt == kF16)
-        apply_block_vec<kF16>(base, e0, acc);
+        update_block_vec<kF16>(base, e0, b, P, lut_base);
       else
-        apply_block_vec<kF32>(base, e0, acc);
+        update_block_vec<kF32>(base, e0, b, P, lut_base);
     } else {
+      float acc[16];
+#pragma unroll
+      for (int m = 0; m < 16; ++m) acc[m] = 0.0f;
+      accumulate_block(acc, b, P, lut_base);
 #pragma unroll
       for (int i = 0; i < 16; ++i) {
         if (i < cnt) store_elem(base, dt, e0 + i, __fadd_rn(load_elem(base, dt, e0 + i), acc[i]));
@@ -259,7 +296,8 @@ cudaError_t launch_perturb(const PerturbParams& p, int grid, cudaStream_t stream
   return cudaGetLastError();
 }
 
-size_t update_smem_bytes(int groups) { return static_cast<size_t>(groups) * 40 * sizeof(float); }
+// Coefficients (32 bytes per group), alignment slack, one 256-byte frame per group.
+size_t update_smem_bytes(int groups) { return static_cast<size_t>(groups) * (32 + kFrameBytes) + kFrameBytes; }
 
 cudaError_t launch_update(const UpdateParams& p, int grid, cudaStream_t stream) {
   update_kernel<<<grid, kThreads, update_smem_bytes(p.groups), stream>>>(p);

@@ -314,10 +314,26 @@ def test_tiny_workload_lockstep():
             lm = oracle.quadratic_loss(host[0], a)
             oracle.perturb(host, [W.DT_F32], seed, k, eps)
             rows.append([lp, lm, l0_o])
+        rows = np.array(rows)
+        Lg = losses.cpu().numpy()
+        cg = c.cpu().numpy()
+        assert int(st.item()) == zo.ZO_OK
+        # losses: the same perturbed weights bit for bit; only the fp64
+        # summation order differs
+        np.testing.assert_allclose(Lg, rows, rtol=1e-12)
+        # preconditioner on identical inputs
+        rc, c_same, _, _ = oracle.precondition(Lg, eps)
+        assert rc == oracle.OK
+        np.testing.assert_allclose(cg, c_same, rtol=1e-12)
+        # against the oracle's own losses: a relative loss error r becomes
+        # r (|L+| + |L-|) / |L+ - L-| in the difference and
+        # alpha r (|L+| + 2|L0| + |L-|) / |L+ - 2 L0 + L-| through w
         rc, c_o, _, _ = oracle.precondition(rows, eps)
-        assert rc == oracle.OK and int(st.item()) == zo.ZO_OK
-        np.testing.assert_allclose(losses.cpu().numpy(), np.array(rows), rtol=1e-12)
-        np.testing.assert_allclose(c.cpu().numpy(), c_o, rtol=1e-6)
-        oracle.update(host, [W.DT_F32], seed, c.cpu().numpy(), lr)
+        assert rc == oracle.OK
+        lp, lm, l0 = np.abs(rows[:, 0]), np.abs(rows[:, 1]), np.abs(rows[:, 2])
+        cond = ((lp + lm) / np.abs(rows[:, 0] - rows[:, 1])
+                + 0.1 * (lp + 2 * l0 + lm) / np.abs(rows[:, 0] - 2 * rows[:, 2] + rows[:, 1]))
+        assert np.all(np.abs(cg - c_o) <= 1e-11 * cond * np.abs(c_o) + 1e-300)
+        oracle.update(host, [W.DT_F32], seed, cg, lr)
         assert_update_close(storage_bits(theta), storage_bits(host[0]), W.DT_F32, c.cpu().numpy(), lr,
                             context=f"step {step}")
