@@ -15,6 +15,7 @@ replicas: every rank trains its own copy; nothing is exchanged.
 prefix sample of the same workload.
 """
 import argparse
+import dataclasses
 import hashlib
 import json
 import os
@@ -45,6 +46,7 @@ def parse_args():
     ap.add_argument("--warmup", type=int, default=3)
     ap.add_argument("--impl", choices=["zo", "reference"], default="zo")
     ap.add_argument("--config", default="opt-30b", choices=sorted(W.BY_KEY))
+    ap.add_argument("--K", type=int, default=None, help="override the probes per step of --config")
     ap.add_argument("--cpu-seconds", type=float, default=12.0, help="target CPU time of the oracle sample")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
@@ -176,11 +178,18 @@ def time_oracle(ps, target_s, steps=1, warmup=0):
     return value, dt, M, sample
 
 
+def param_set(args):
+    ps = W.BY_KEY[args.config]
+    if args.K is not None:
+        ps = dataclasses.replace(ps, K=args.K)
+    return ps
+
+
 def run_reference(args):
     rank = int(os.environ.get("RANK", "0"))
     if rank != 0:
         return
-    ps = W.BY_KEY[args.config]
+    ps = param_set(args)
     value, dt, M, sample = time_oracle(ps, args.cpu_seconds / 2, steps=args.steps, warmup=args.warmup)
     line = {
         "impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": args.gpus,
@@ -220,7 +229,7 @@ def run_zo(args):
         dist.all_reduce(t, op=dist.ReduceOp.MAX)
         return float(t.item())
 
-    ps = W.BY_KEY[args.config]
+    ps = param_set(args)
     K, eps, d = ps.K, ps.eps, ps.d
     params = W.allocate_params(ps, device=dev)
     plist = zo.ParamList(params)

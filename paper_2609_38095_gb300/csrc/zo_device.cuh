@@ -89,14 +89,21 @@ __device__ __forceinline__ uint32_t word_of(const uint4& x, int m) {
 
 // 256-bit global accesses (sm_100+): one per 16-element block of a 16-bit
 // tensor, two for fp32. The caller guarantees 32-byte alignment.
+#ifndef ZO_LDQ
+#define ZO_LDQ ""  // cache qualifier of the streaming loads
+#endif
+#ifndef ZO_STQ
+#define ZO_STQ ""  // cache qualifier of the streaming stores
+#endif
+
 __device__ __forceinline__ void ld256(const void* p, uint32_t (&r)[8]) {
-  asm volatile("ld.global.v8.u32 {%0,%1,%2,%3,%4,%5,%6,%7}, [%8];"
+  asm volatile("ld.global" ZO_LDQ ".v8.u32 {%0,%1,%2,%3,%4,%5,%6,%7}, [%8];"
                : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7])
                : "l"(p));
 }
 
 __device__ __forceinline__ void st256(void* p, const uint32_t (&r)[8]) {
-  asm volatile("st.global.v8.u32 [%0], {%1,%2,%3,%4,%5,%6,%7,%8};" ::"l"(p), "r"(r[0]), "r"(r[1]), "r"(r[2]),
+  asm volatile("st.global" ZO_STQ ".v8.u32 [%0], {%1,%2,%3,%4,%5,%6,%7,%8};" ::"l"(p), "r"(r[0]), "r"(r[1]), "r"(r[2]),
                "r"(r[3]), "r"(r[4]), "r"(r[5]), "r"(r[6]), "r"(r[7])
                : "memory");
 }

@@ -57,6 +57,54 @@ __device__ __forceinline__ void perturb_block_vec(void* base, int64_t e0, const 
   }
 }
 
+template <uint8_t DT>
+__device__ __forceinline__ void perturb_regs16(uint32_t (&v)[8], const uint4& x, uint32_t nscale_bits, uint32_t j) {
+#pragma unroll
+  for (int r = 0; r < 8; ++r) {
+    const float2 f = unpack2<DT>(v[r]);
+    const float r0 = __fadd_rn(f.x, __uint_as_float(nscale_bits ^ sign_bit(x, 2 * r, j)));
+    const float r1 = __fadd_rn(f.y, __uint_as_float(nscale_bits ^ sign_bit(x, 2 * r + 1, j)));
+    v[r] = pack2<DT>(r0, r1);
+  }
+}
+
+// Address of block b of tensor t when it takes the pipelined path (a full,
+// 32-byte aligned block of a 16-bit tensor), else nullptr.
+__device__ __forceinline__ uint16_t* fast16_block(const TensorTable& tab, int t, int64_t b) {
+  const int64_t e0 = (b - tensor_blk_begin(tab, t)) * 16;
+  const uint8_t fl = tab.flags[t];
+  if ((fl & kVec32) && (fl & kDtypeMask) != kF32 && tab.numel[t] - e0 >= 16)
+    return reinterpret_cast<uint16_t*>(tab.ptr[t]) + e0;
+  return nullptr;
+}
+
+// Any other block: fp32, a partial last block, or an unaligned tensor.
+__device__ __noinline__ void perturb_block_other(const TensorTable& tab, int t, int64_t b, uint4 x,
+                                                 uint32_t nscale_bits, uint32_t j) {
+  const int64_t e0 = (b - tensor_blk_begin(tab, t)) * 16;
+  const int64_t cnt = min(static_cast<int64_t>(16), tab.numel[t] - e0);
+  const uint8_t fl = tab.flags[t];
+  const uint8_t dt = fl & kDtypeMask;
+  void* base = reinterpret_cast<void*>(tab.ptr[t]);
+  if (cnt == 16 && (fl & kVec32)) {
+    if (dt == kBF16)
+      perturb_block_vec<kBF16>(base, e0, x, nscale_bits, j);
+    else if (dt == kF16)
+      perturb_block_vec<kF16>(base, e0, x, nscale_bits, j);
+    else
+      perturb_block_vec<kF32>(base, e0, x, nscale_bits, j);
+  } else {
+    for (int i = 0; i < cnt; ++i) {
+      const float th = load_elem(base, dt, e0 + i);
+      store_elem(base, dt, e0 + i, __fadd_rn(th, __uint_as_float(nscale_bits ^ sign_bit(x, i, j))));
+    }
+  }
+}
+
+// Software-pipelined over a thread's blocks: the 256-bit load of the next
+// 16-bit block is issued before the current block is computed and stored, so
+// each thread keeps two loads in flight (the pass is HBM-bound and needs the
+// bytes in flight to cover DRAM latency).
 __global__ void __launch_bounds__(256) perturb_kernel(const __grid_constant__ PerturbParams P) {
   if (P.status != nullptr && *P.status != 0) return;
   float scale = P.scale;
@@ -68,30 +116,39 @@ __global__ void __launch_bounds__(256) perturb_kernel(const __grid_constant__ Pe
   const TensorTable& tab = P.tab;
   const int64_t blk_total = tab.blk_end[tab.n - 1];
   const int64_t stride = static_cast<int64_t>(gridDim.x) * blockDim.x;
-  int t = 0;
-  for (int64_t b = tab.blk_begin + static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; b < blk_total;
-       b += stride) {
-    t = advance_tensor(tab, t, b);
-    const int64_t e0 = (b - tensor_blk_begin(tab, t)) * 16;
-    const int64_t cnt = min(static_cast<int64_t>(16), tab.numel[t] - e0);
-    const uint8_t fl = tab.flags[t];
-    const uint8_t dt = fl & kDtypeMask;
-    void* base = reinterpret_cast<void*>(tab.ptr[t]);
+  int64_t b = tab.blk_begin + static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x;
+  if (b >= blk_total) return;
+  int t = advance_tensor(tab, 0, b);
+  uint16_t* p = fast16_block(tab, t, b);
+  uint32_t v[8];
+  if (p != nullptr) ld256(p, v);
+  while (true) {
+    const int64_t bn = b + stride;
+    int tn = t;
+    uint16_t* pn = nullptr;
+    uint32_t vn[8];
+    if (bn < blk_total) {
+      tn = advance_tensor(tab, t, bn);
+      pn = fast16_block(tab, tn, bn);
+      if (pn != nullptr) ld256(pn, vn);
+    }
     const uint4 x = philox10(static_cast<uint32_t>(b), static_cast<uint32_t>(static_cast<uint64_t>(b) >> 32), q, 0u,
                              P.keys);
-    if (cnt == 16 && (fl & kVec32)) {
-      if (dt == kBF16)
-        perturb_block_vec<kBF16>(base, e0, x, nscale_bits, j);
-      else if (dt == kF16)
-        perturb_block_vec<kF16>(base, e0, x, nscale_bits, j);
+    if (p != nullptr) {
+      if ((tab.flags[t] & kDtypeMask) == kBF16)
+        perturb_regs16<kBF16>(v, x, nscale_bits, j);
       else
-        perturb_block_vec<kF32>(base, e0, x, nscale_bits, j);
+        perturb_regs16<kF16>(v, x, nscale_bits, j);
+      st256(p, v);
     } else {
-      for (int i = 0; i < cnt; ++i) {
-        const float th = load_elem(base, dt, e0 + i);
-        store_elem(base, dt, e0 + i, __fadd_rn(th, __uint_as_float(nscale_bits ^ sign_bit(x, i, j))));
-      }
+      perturb_block_other(tab, t, b, x, nscale_bits, j);
     }
+    if (bn >= blk_total) break;
+    b = bn;
+    t = tn;
+    p = pn;
+#pragma unroll
+    for (int r = 0; r < 8; ++r) v[r] = vn[r];
   }
 }
 
