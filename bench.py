@@ -50,6 +50,8 @@ def parse_args():
     ap.add_argument("--cpu-seconds", type=float, default=12.0, help="target CPU time of the oracle sample")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--sequential", action="store_true",
+                    help="also time Algorithm 1's K sequential passes against the fused update")
     return ap.parse_args()
 
 
@@ -132,6 +134,34 @@ class ClockSampler:
             return None
         return {"sm_mhz": statistics.median(sm), "sm_max_mhz": max(mx), "reasons": sorted(reasons),
                 "samples": len(sm)}
+
+
+# ------------------------------------------------------- ranks (replicas)
+def dist_barrier(world, device):
+    """Barrier over the ranks, then a device synchronise."""
+    import torch
+    import torch.distributed as dist
+    if world > 1:
+        dist.barrier()
+    if device.type == "cuda":
+        torch.cuda.synchronize(device)
+
+
+def max_over_ranks(x, world, device):
+    """Largest value of x over all ranks (the slowest replica sets the time)."""
+    if world == 1:
+        return x
+    import torch
+    import torch.distributed as dist
+    t = torch.tensor([x], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def whole_job_rate(world, d, K, seconds):
+    """Gparam*probe/s of the whole job: every replica processes d weights x K
+    probes per step."""
+    return world * d * K / seconds / 1e9
 
 
 # ------------------------------------------------------------- oracle arm
@@ -218,16 +248,10 @@ def run_zo(args):
         dist.init_process_group("nccl", device_id=dev)
 
     def barrier():
-        if world > 1:
-            dist.barrier()
-        torch.cuda.synchronize()
+        dist_barrier(world, dev)
 
-    def max_over_ranks(x):
-        if world == 1:
-            return x
-        t = torch.tensor([x], dtype=torch.float64, device=dev)
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        return float(t.item())
+    def ranks_max(x):
+        return max_over_ranks(x, world, dev)
 
     ps = param_set(args)
     K, eps, d = ps.K, ps.eps, ps.d
@@ -289,7 +313,7 @@ def run_zo(args):
     t_end.record(stream)
     barrier()
     clk = clocks.stop()
-    elapsed_ms = max_over_ranks(t_start.elapsed_time(t_end))
+    elapsed_ms = ranks_max(t_start.elapsed_time(t_end))
     ms_per_step = elapsed_ms / args.steps
     launches = args.steps * (3 * K * chunks + 1 + chunks)
 
@@ -297,9 +321,9 @@ def run_zo(args):
         v = [a.elapsed_time(b) for a, b in timing[key]]
         return sum(v) / len(v)
 
-    perturb_ms = max_over_ranks(avg_ms("perturb"))
-    update_ms = max_over_ranks(avg_ms("update"))
-    precond_ms = max_over_ranks(avg_ms("precondition"))
+    perturb_ms = ranks_max(avg_ms("perturb"))
+    update_ms = ranks_max(avg_ms("update"))
+    precond_ms = ranks_max(avg_ms("precondition"))
 
     # ---- end to end through the public API with host buffers
     e2e = None
@@ -320,9 +344,30 @@ def run_zo(args):
             if int(st_host[0]) != 0:
                 raise RuntimeError("preconditioner reported non-finite losses")
         barrier()
-        e2e_s = max_over_ranks((time.perf_counter() - t0) / args.steps)
-        e2e = {"value": world * d * K / e2e_s / 1e9, "unit": UNIT, "h2d_bytes_per_step": K * 3 * 8,
+        e2e_s = ranks_max((time.perf_counter() - t0) / args.steps)
+        e2e = {"value": whole_job_rate(world, d, K, e2e_s), "unit": UNIT, "h2d_bytes_per_step": K * 3 * 8,
                "d2h_bytes_per_step": K * 8 + 4, "ms_per_step": e2e_s * 1e3}
+
+    # ---- Algorithm 1's K-pass update against the fused one (same coefficients)
+    seq = None
+    if args.sequential:
+        reps = 2
+        ev = [torch.cuda.Event(enable_timing=True) for _ in range(3)]
+        zo.update_sequential(plist, W.step_seed(0), c, eps, status=status)  # warm
+        barrier()
+        ev[0].record(stream)
+        for _ in range(reps):
+            zo.update(plist, W.step_seed(0), c, eps, status=status)
+        ev[1].record(stream)
+        for _ in range(reps):
+            zo.update_sequential(plist, W.step_seed(0), c, eps, status=status)
+        ev[2].record(stream)
+        barrier()
+        fused_ms = ev[0].elapsed_time(ev[1]) / reps
+        seq_ms = ev[1].elapsed_time(ev[2]) / reps
+        seq = {"fused_ms": fused_ms, "sequential_ms": seq_ms, "speedup": seq_ms / fused_ms,
+               "sequential_launches": K * chunks,
+               "sequential_GB/s": K * 2.0 * d * ps.bytes_per_elem / (seq_ms * 1e-3) / 1e9}
 
     peaks, peak_kind = measured_peaks()
     hbm_peak = float(peaks.get("hbm_gbs", FALLBACK_HBM_GBS))
@@ -333,7 +378,7 @@ def run_zo(args):
     sm_mhz = (clk or {}).get("sm_mhz") or float(peaks.get("sm_max_mhz", 2070.0))
     alu_peak = sms * LANES_PER_SM * sm_mhz * 1e6 / 1e9    # Gparam*probe/s at one instruction per pair
     upd_rate = d * K / (update_ms * 1e-3) / 1e9
-    value = world * d * K / (ms_per_step * 1e-3) / 1e9
+    value = whole_job_rate(world, d, K, ms_per_step * 1e-3)
 
     if rank != 0:
         return
@@ -361,6 +406,7 @@ def run_zo(args):
             "precondition": {"ms": precond_ms},
         },
         "e2e": e2e,
+        "sequential": seq,
         "gpu_launches": launches,
         "clocks": clk,
         "cpu_baseline": cpu,
