@@ -50,6 +50,8 @@ def parse_args():
     ap.add_argument("--cpu-seconds", type=float, default=12.0, help="target CPU time of the oracle sample")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--packing", type=int, default=1, choices=[1, 8],
+                    help="generated bits per (weight, probe): 1 (the paper's bit packing) or 8")
     ap.add_argument("--sequential", action="store_true",
                     help="also time Algorithm 1's K sequential passes against the fused update")
     return ap.parse_args()
@@ -190,9 +192,10 @@ def oracle_sample_size(ps, target_s):
     return max(16, min(M, ps.numels[0]) // 16 * 16)
 
 
-def time_oracle(ps, target_s, steps=1, warmup=0):
+def time_oracle(ps, target_s, steps=1, warmup=0, packing=1):
     import oracle
     oracle.lib()
+    oracle.set_packing(packing)
     M = oracle_sample_size(ps, target_s)
     rng = np.random.default_rng(1)
     th = [W.random_storage(rng, M, ps.dtype)]
@@ -220,12 +223,13 @@ def run_reference(args):
     if rank != 0:
         return
     ps = param_set(args)
-    value, dt, M, sample = time_oracle(ps, args.cpu_seconds / 2, steps=args.steps, warmup=args.warmup)
+    value, dt, M, sample = time_oracle(ps, args.cpu_seconds / 2, steps=args.steps, warmup=args.warmup,
+                                       packing=args.packing)
     line = {
         "impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": args.gpus,
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": dt * 1e3, "higher_is_better": True,
         "scaling": "weak", "vs_baseline": None, "dtype": "f32", "data": "synthetic",
-        "config": {"workload": ps.name, "K": ps.K, "d": ps.d, "sample_weights": M},
+        "config": {"workload": ps.name, "K": ps.K, "d": ps.d, "packing": args.packing, "sample_weights": M},
         "cpu_baseline": {"value": value, "unit": UNIT, "cores": 1, "kind": "oracle", "sample": sample},
         "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
     }
@@ -244,6 +248,7 @@ def run_zo(args):
     local = int(os.environ.get("LOCAL_RANK", "0"))
     torch.cuda.set_device(local)
     dev = torch.device("cuda", local)
+    zo.set_packing(args.packing)
     if world > 1:
         dist.init_process_group("nccl", device_id=dev)
 
@@ -384,13 +389,14 @@ def run_zo(args):
         return
     cpu = None
     if world == 1 and not args.no_cpu_baseline:
-        v, dt, M, sample = time_oracle(ps, args.cpu_seconds)
+        v, dt, M, sample = time_oracle(ps, args.cpu_seconds, packing=args.packing)
         cpu = {"value": v, "unit": UNIT, "cores": 1, "kind": "oracle", "sample": sample}
     line = {
         "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
         "warmup": args.warmup, "ms_per_step": ms_per_step, "higher_is_better": True, "scaling": "weak",
         "vs_baseline": None, "dtype": "f32", "data": "synthetic",
-        "config": {"workload": ps.name, "K": K, "d": d, "tensors": len(params), "storage": "fp16" if
+        "config": {"workload": ps.name, "K": K, "d": d, "tensors": len(params), "packing": args.packing,
+                   "storage": "fp16" if
                    ps.dtype == W.DT_F16 else ("bf16" if ps.dtype == W.DT_BF16 else "fp32"),
                    "eps": eps, "lr": eps, "parallelism": f"replicas{world}",
                    "l2": "inputs larger than L2 (every pass streams the whole parameter set)"},

@@ -50,7 +50,11 @@
  *   byte    m = g mod 16 is bits 8*(m mod 4) .. +7 of word x[m / 4]
  *   bit     z_k[g] = +1 if bit (k mod 8) of that byte is 1, else -1
  * so each 32-bit Philox word unpacks to four per-element bytes, each holding
- * the signs of eight probes.
+ * the signs of eight probes ("packing 1": one generated bit per weight and
+ * probe, as the paper's 1-bit packed perturbations).
+ * With zo_set_packing(8) every (weight, probe) pair takes a whole generated
+ * byte instead: output = Philox4x32-10(counter = (b mod 2^32, b / 2^32, k, 0),
+ * key), byte m = g mod 16 as above, z_k[g] = +1 if bit 0 of that byte is 1.
  *
  * Arithmetic. Weights are read as fp32, the operation is done in fp32 and the
  * result is rounded once to the storage dtype (round to nearest even).
@@ -95,6 +99,14 @@ const char* zo_last_cuda_error(void);
 
 /* Library version, major * 10000 + minor * 100 + patch. */
 int zo_version(void);
+
+/* Probe packing used by every later call of the process: 1 (default) or 8
+ * generated bits per (weight, probe), see "Probes" above (Sec. 4.3 "Bit-Packed
+ * perturbations" packs one bit; 8 gives each weight a whole byte per probe).
+ * Set it before a step and keep it for the whole step: every call of a step
+ * must regenerate the same probes. Returns ZO_ERR_ARG for other values. */
+int zo_set_packing(int32_t bits_per_value);
+int zo_get_packing(void);
 
 /* ---------------------------------------------------------------------------
  * zo_perturb -- Algorithm 1, ApplyPackedPerturbation(theta, scale, z_k): adds

@@ -98,10 +98,27 @@ void oracle_philox4x32_10(const uint32_t ctr[4], const uint32_t key[2], uint32_t
 /*                                                                           */
 /* Element index g is the "virtual" flattened index: tensor t starts at      */
 /* S_t = sum over earlier tensors of numel rounded up to a multiple of 16.   */
-/* Philox block b = g / 16 with probe group q = k / 8 gives 128 bits; byte    */
-/* (g mod 16) of that output (little-endian within each 32-bit word) holds   */
-/* the signs of probes 8q..8q+7 of element g, probe k in bit (k mod 8).       */
+/*                                                                           */
+/* Packing 1 (default, one generated bit per (element, probe)): Philox block */
+/* b = g / 16 with probe group q = k / 8 gives 128 bits; byte (g mod 16) of  */
+/* that output (little-endian within each 32-bit word) holds the signs of    */
+/* probes 8q..8q+7 of element g, probe k in bit (k mod 8).                   */
+/*                                                                           */
+/* Packing 8 (one generated byte per (element, probe)): Philox block         */
+/* b = g / 16 with the probe id k itself in the counter; the sign of element */
+/* g is bit 0 of byte (g mod 16).                                            */
 /* ------------------------------------------------------------------------- */
+
+static int g_packing = 1; /* 1 or 8, see above */
+
+/* Select the probe packing (1 or 8); returns ORC_ERR_ARG otherwise. */
+int oracle_set_packing(int bits_per_value) {
+  if (bits_per_value != 1 && bits_per_value != 8) return -1;
+  g_packing = bits_per_value;
+  return 0;
+}
+
+int oracle_get_packing(void) { return g_packing; }
 
 /* The 16 output bytes of Philox(counter = (b_lo, b_hi, q, 0), key = seed). */
 static void philox_block_bytes(uint64_t seed, uint64_t b, uint32_t q, uint8_t bytes[16]) {
@@ -115,6 +132,10 @@ static void philox_block_bytes(uint64_t seed, uint64_t b, uint32_t q, uint8_t by
 /* Probe bit of element g for probe k: 1 means z = +1, 0 means z = -1. */
 int oracle_probe_bit(uint64_t seed, uint32_t k, uint64_t g) {
   uint8_t bytes[16];
+  if (g_packing == 8) {
+    philox_block_bytes(seed, g / 16u, k, bytes);
+    return bytes[g % 16u] & 1;
+  }
   philox_block_bytes(seed, g / 16u, k / 8u, bytes);
   return (bytes[g % 16u] >> (k % 8u)) & 1;
 }

@@ -1,6 +1,7 @@
 // zo_api.cu -- the extern "C" entry points declared in include/zo.h: argument
 // validation, Philox key expansion, tensor-table planning and launch sizing.
 // Everything here runs on the host and only enqueues kernels.
+#include <atomic>
 #include <cmath>
 #include <cstdio>
 #include <cstring>
@@ -41,6 +42,20 @@ RoundKeys expand_keys(uint64_t seed) {
 
 int elem_size(int32_t dtype) { return dtype == ZO_F32 ? 4 : 2; }
 
+// Probe packing of every later call (1 or 8 generated bits per weight and probe).
+std::atomic<int> g_packing{zo::kPacking1};
+
+// Third Philox counter word and sign bit of probe k under the current packing.
+void probe_counter(uint32_t k, int packing, uint32_t* ctr2, uint32_t* bit) {
+  if (packing == zo::kPacking8) {
+    *ctr2 = k;
+    *bit = 0;
+  } else {
+    *ctr2 = k >> 3;
+    *bit = k & 7u;
+  }
+}
+
 // Resident perturb blocks per SM. The pass is HBM-bound and each thread keeps
 // two 32-byte loads in flight; on GB300 four 256-thread blocks per SM stream
 // fastest (measured: 3 -> 90.6 %, 4 -> 97.7 %, 5 -> 93.0 % of the copy
@@ -55,7 +70,7 @@ constexpr int kUpdateWaves = 4;
 struct DeviceInfo {
   int sms = 0;
   int perturb_bps = 0;                    // resident perturb blocks per SM
-  int update_bps[zo::kMaxGroups + 1] = {};  // by probe-group count
+  int update_bps[2][zo::kMaxGroups + 1] = {};  // by packing (1, 8) and probe-group count
 };
 constexpr int kMaxDevices = 64;
 DeviceInfo g_dev[kMaxDevices];
@@ -82,15 +97,16 @@ int device_info(DeviceInfo** out) {
   return ZO_OK;
 }
 
-int update_blocks_per_sm(DeviceInfo* d, int groups, int* out) {
+int update_blocks_per_sm(DeviceInfo* d, int groups, int packing, int* out) {
   std::lock_guard<std::mutex> lock(g_dev_mu);
-  if (d->update_bps[groups] == 0) {
+  int& slot = d->update_bps[packing == zo::kPacking8 ? 1 : 0][groups];
+  if (slot == 0) {
     int bps = 0;
-    cudaError_t e = zo::update_blocks_per_sm(groups, &bps);
+    cudaError_t e = zo::update_blocks_per_sm(groups, packing, &bps);
     if (e != cudaSuccess) return cuda_fail(e, "occupancy(update)");
-    d->update_bps[groups] = bps > 0 ? bps : 1;
+    slot = bps > 0 ? bps : 1;
   }
-  *out = d->update_bps[groups];
+  *out = slot;
   return ZO_OK;
 }
 
@@ -177,7 +193,15 @@ const char* zo_status_string(int status) {
 
 const char* zo_last_cuda_error(void) { return g_last_cuda_error; }
 
-int zo_version(void) { return 10000; }
+int zo_version(void) { return 10100; }
+
+int zo_set_packing(int32_t bits_per_value) {
+  if (bits_per_value != zo::kPacking1 && bits_per_value != zo::kPacking8) return ZO_ERR_ARG;
+  g_packing.store(bits_per_value);
+  return ZO_OK;
+}
+
+int zo_get_packing(void) { return g_packing.load(); }
 
 int zo_perturb(const zo_tensor* params, int32_t n_tensors, uint64_t seed, uint32_t probe, float scale,
                void* stream) {
@@ -190,6 +214,7 @@ int zo_perturb(const zo_tensor* params, int32_t n_tensors, uint64_t seed, uint32
   PerturbParams& pp = tl_perturb;
   pp.keys = expand_keys(seed);
   pp.probe = probe;
+  probe_counter(probe, g_packing.load(), &pp.ctr2, &pp.bit);
   pp.scale = scale;
   pp.coef = nullptr;
   pp.coef_mul = 0.0;
@@ -218,9 +243,10 @@ int zo_update(const zo_tensor* params, int32_t n_tensors, uint64_t seed, const d
   up.coef_mul = -(lr / static_cast<double>(K));
   up.K = K;
   up.groups = (K + 7) / 8;
+  up.packing = g_packing.load();
   up.status = status;
   int bps = 1;
-  if ((rc = update_blocks_per_sm(d, up.groups, &bps)) != ZO_OK) return rc;
+  if ((rc = update_blocks_per_sm(d, up.groups, up.packing, &bps)) != ZO_OK) return rc;
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   int64_t blk = 0;
   for (int32_t t0 = 0; t0 < n_tensors; t0 += zo::kMaxTensorsPerLaunch) {
@@ -247,8 +273,10 @@ int zo_update_sequential(const zo_tensor* params, int32_t n_tensors, uint64_t se
   pp.coef = c;
   pp.coef_mul = -(lr / static_cast<double>(K));
   pp.status = status;
+  const int packing = g_packing.load();
   for (int32_t k = 0; k < K; ++k) {
     pp.probe = static_cast<uint32_t>(k);
+    probe_counter(pp.probe, packing, &pp.ctr2, &pp.bit);
     if ((rc = run_perturb(params, n_tensors, pp, d, static_cast<cudaStream_t>(stream))) != ZO_OK) return rc;
   }
   return ZO_OK;
@@ -293,7 +321,9 @@ int zo_probe_bytes(uint64_t seed, uint32_t probe, int64_t first, int64_t n, uint
   int grid = 1;
   int rc = probe_view_grid((n + 1) / 2 + 1, &grid);
   if (rc != ZO_OK) return rc;
-  cudaError_t e = zo::launch_probe_bytes(expand_keys(seed), probe, first, n, out, grid,
+  uint32_t ctr2 = 0, bit = 0;
+  probe_counter(probe, g_packing.load(), &ctr2, &bit);
+  cudaError_t e = zo::launch_probe_bytes(expand_keys(seed), ctr2, bit, first, n, out, grid,
                                          static_cast<cudaStream_t>(stream));
   return e == cudaSuccess ? ZO_OK : cuda_fail(e, "probe_bytes_kernel");
 }
@@ -305,7 +335,9 @@ int zo_probe_signs(uint64_t seed, uint32_t probe, int64_t first, int64_t n, int8
   int grid = 1;
   int rc = probe_view_grid(n / 16 + 2, &grid);
   if (rc != ZO_OK) return rc;
-  cudaError_t e = zo::launch_probe_signs(expand_keys(seed), probe, first, n, out, grid,
+  uint32_t ctr2 = 0, bit = 0;
+  probe_counter(probe, g_packing.load(), &ctr2, &bit);
+  cudaError_t e = zo::launch_probe_signs(expand_keys(seed), ctr2, bit, first, n, out, grid,
                                          static_cast<cudaStream_t>(stream));
   return e == cudaSuccess ? ZO_OK : cuda_fail(e, "probe_signs_kernel");
 }

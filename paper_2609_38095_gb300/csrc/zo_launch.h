@@ -18,11 +18,11 @@ cudaError_t launch_perturb(const PerturbParams& p, int grid, cudaStream_t stream
 cudaError_t launch_update(const UpdateParams& p, int grid, cudaStream_t stream);
 size_t update_smem_bytes(int groups);
 cudaError_t perturb_blocks_per_sm(int* out);
-cudaError_t update_blocks_per_sm(int groups, int* out);
-cudaError_t launch_probe_bytes(const RoundKeys& keys, uint32_t probe, int64_t first, int64_t n, uint8_t* out,
-                               int grid, cudaStream_t stream);
-cudaError_t launch_probe_signs(const RoundKeys& keys, uint32_t probe, int64_t first, int64_t n, int8_t* out,
-                               int grid, cudaStream_t stream);
+cudaError_t update_blocks_per_sm(int groups, int packing, int* out);
+cudaError_t launch_probe_bytes(const RoundKeys& keys, uint32_t ctr2, uint32_t bit, int64_t first, int64_t n,
+                               uint8_t* out, int grid, cudaStream_t stream);
+cudaError_t launch_probe_signs(const RoundKeys& keys, uint32_t ctr2, uint32_t bit, int64_t first, int64_t n,
+                               int8_t* out, int grid, cudaStream_t stream);
 cudaError_t launch_precondition(const double* losses, int K, double eps, double alpha, double lambda_reg,
                                 int one_sided, double* c, double* w, double* curv, int32_t* status,
                                 cudaStream_t stream);

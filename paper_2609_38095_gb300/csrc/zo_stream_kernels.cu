@@ -110,8 +110,8 @@ __global__ void __launch_bounds__(256) perturb_kernel(const __grid_constant__ Pe
   float scale = P.scale;
   if (P.coef != nullptr) scale = __double2float_rn(P.coef_mul * P.coef[P.probe]);
   const uint32_t nscale_bits = __float_as_uint(scale) ^ 0x80000000u;  // -scale
-  const uint32_t j = P.probe & 7u;
-  const uint32_t q = P.probe >> 3;
+  const uint32_t j = P.bit;
+  const uint32_t q = P.ctr2;
 
   const TensorTable& tab = P.tab;
   const int64_t blk_total = tab.blk_end[tab.n - 1];
@@ -207,16 +207,60 @@ __device__ __forceinline__ void accumulate_block(float (&acc)[16], int64_t b, co
   }
 }
 
+// Packing 8: the sign of probe k is bit 0 of the element's byte of
+// Philox(b, k). Eight outputs (probes 8f..8f+7) are folded into the same
+// nibble layout as packing 1 -- bit 0 of every byte moved to bit i + 2 of the
+// low (i < 4) or high (i >= 4) offset word -- and looked up in the same tables.
+__device__ __forceinline__ void accumulate_block_p8(float (&acc)[16], int64_t b, const UpdateParams& P,
+                                                    uint32_t lut_base) {
+  const uint32_t blo = static_cast<uint32_t>(b), bhi = static_cast<uint32_t>(static_cast<uint64_t>(b) >> 32);
+  uint32_t frame = lut_base;
+  for (int f = 0; f < P.groups; ++f, frame += kFrameBytes) {
+    uint32_t lo4[4] = {0u, 0u, 0u, 0u}, hi4[4] = {0u, 0u, 0u, 0u};
+#pragma unroll
+    for (int i = 0; i < 8; ++i) {
+      const uint4 x = philox10(blo, bhi, static_cast<uint32_t>(8 * f + i), 0u, P.keys);
+#pragma unroll
+      for (int m = 0; m < 4; ++m) {
+        const uint32_t bits = word_of(x, m) & 0x01010101u;
+        if (i < 4)
+          lo4[m] |= bits << (i + 2);
+        else
+          hi4[m] |= bits << (i - 2);
+      }
+    }
+#pragma unroll
+    for (int m = 0; m < 4; ++m) {
+#pragma unroll
+      for (int j = 0; j < 4; ++j) {
+        const uint32_t sel = 0x7650u | static_cast<uint32_t>(j);
+        const float tlo = lds_lo(__byte_perm(lo4[m], frame, sel));
+        const float thi = lds_hi(__byte_perm(hi4[m], frame, sel));
+        acc[4 * m + j] = __fadd_rn(__fadd_rn(acc[4 * m + j], tlo), thi);
+      }
+    }
+  }
+}
+
+template <int PACK>
+__device__ __forceinline__ void accumulate_any(float (&acc)[16], int64_t b, const UpdateParams& P,
+                                               uint32_t lut_base) {
+  if constexpr (PACK == kPacking8)
+    accumulate_block_p8(acc, b, P, lut_base);
+  else
+    accumulate_block(acc, b, P, lut_base);
+}
+
 // One full, 32-byte aligned block: theta is loaded before the probe loop so
 // the load overlaps the arithmetic.
-template <uint8_t DT>
+template <int PACK, uint8_t DT>
 __device__ __forceinline__ void update_block_vec(void* base, int64_t e0, int64_t b, const UpdateParams& P,
                                                  uint32_t lut_base) {
   float acc[16];
 #pragma unroll
   for (int m = 0; m < 16; ++m) acc[m] = 0.0f;
   if constexpr (DT == kF32) {
-    accumulate_block(acc, b, P, lut_base);
+    accumulate_any<PACK>(acc, b, P, lut_base);
     float* p = static_cast<float*>(base) + e0;
 #pragma unroll
     for (int half = 0; half < 2; ++half) {
@@ -230,7 +274,7 @@ __device__ __forceinline__ void update_block_vec(void* base, int64_t e0, int64_t
     uint16_t* p = static_cast<uint16_t*>(base) + e0;
     uint32_t v[8];
     ld256(p, v);
-    accumulate_block(acc, b, P, lut_base);
+    accumulate_any<PACK>(acc, b, P, lut_base);
 #pragma unroll
     for (int r = 0; r < 8; ++r) {
       const float2 f = unpack2<DT>(v[r]);
@@ -240,6 +284,7 @@ __device__ __forceinline__ void update_block_vec(void* base, int64_t e0, int64_t
   }
 }
 
+template <int PACK>
 __global__ void __launch_bounds__(256) update_kernel(const __grid_constant__ UpdateParams P) {
   extern __shared__ __align__(16) unsigned char smem[];
   float* a_s = reinterpret_cast<float*>(smem);  // 8 * groups coefficients (zero padded)
@@ -278,16 +323,16 @@ __global__ void __launch_bounds__(256) update_kernel(const __grid_constant__ Upd
     void* base = reinterpret_cast<void*>(tab.ptr[t]);
     if (cnt == 16 && (fl & kVec32)) {
       if (dt == kBF16)
-        update_block_vec<kBF16>(base, e0, b, P, lut_base);
+        update_block_vec<PACK, kBF16>(base, e0, b, P, lut_base);
       else if (dt == kF16)
-        update_block_vec<kF16>(base, e0, b, P, lut_base);
+        update_block_vec<PACK, kF16>(base, e0, b, P, lut_base);
       else
-        update_block_vec<kF32>(base, e0, b, P, lut_base);
+        update_block_vec<PACK, kF32>(base, e0, b, P, lut_base);
     } else {
       float acc[16];
 #pragma unroll
       for (int m = 0; m < 16; ++m) acc[m] = 0.0f;
-      accumulate_block(acc, b, P, lut_base);
+      accumulate_any<PACK>(acc, b, P, lut_base);
 #pragma unroll
       for (int i = 0; i < 16; ++i) {
         if (i < cnt) store_elem(base, dt, e0 + i, __fadd_rn(load_elem(base, dt, e0 + i), acc[i]));
@@ -300,8 +345,7 @@ __global__ void __launch_bounds__(256) update_kernel(const __grid_constant__ Upd
 // Debug views: probe k packed one bit per element (Appendix F layout) and the
 // unpacked int8 signs, over a range of the virtual index space.
 // ---------------------------------------------------------------------------
-__global__ void probe_bytes_kernel(RoundKeys keys, uint32_t probe, int64_t first, int64_t n, uint8_t* out) {
-  const uint32_t j = probe & 7u, q = probe >> 3;
+__global__ void probe_bytes_kernel(RoundKeys keys, uint32_t q, uint32_t j, int64_t first, int64_t n, uint8_t* out) {
   const int64_t b_first = first >> 1, b_last = (first + n - 1) >> 1;  // packed bytes 2b, 2b+1 <- block b
   const int64_t stride = static_cast<int64_t>(gridDim.x) * blockDim.x;
   for (int64_t b = b_first + static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; b <= b_last; b += stride) {
@@ -322,8 +366,7 @@ __global__ void probe_bytes_kernel(RoundKeys keys, uint32_t probe, int64_t first
   }
 }
 
-__global__ void probe_signs_kernel(RoundKeys keys, uint32_t probe, int64_t first, int64_t n, int8_t* out) {
-  const uint32_t j = probe & 7u, q = probe >> 3;
+__global__ void probe_signs_kernel(RoundKeys keys, uint32_t q, uint32_t j, int64_t first, int64_t n, int8_t* out) {
   const int64_t b_first = first >> 4, b_last = (first + n - 1) >> 4;
   const int64_t stride = static_cast<int64_t>(gridDim.x) * blockDim.x;
   for (int64_t b = b_first + static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; b <= b_last; b += stride) {
@@ -357,7 +400,10 @@ cudaError_t launch_perturb(const PerturbParams& p, int grid, cudaStream_t stream
 size_t update_smem_bytes(int groups) { return static_cast<size_t>(groups) * (32 + kFrameBytes) + kFrameBytes; }
 
 cudaError_t launch_update(const UpdateParams& p, int grid, cudaStream_t stream) {
-  update_kernel<<<grid, kThreads, update_smem_bytes(p.groups), stream>>>(p);
+  if (p.packing == kPacking8)
+    update_kernel<kPacking8><<<grid, kThreads, update_smem_bytes(p.groups), stream>>>(p);
+  else
+    update_kernel<kPacking1><<<grid, kThreads, update_smem_bytes(p.groups), stream>>>(p);
   return cudaGetLastError();
 }
 
@@ -365,19 +411,23 @@ cudaError_t perturb_blocks_per_sm(int* out) {
   return cudaOccupancyMaxActiveBlocksPerMultiprocessor(out, perturb_kernel, kThreads, 0);
 }
 
-cudaError_t update_blocks_per_sm(int groups, int* out) {
-  return cudaOccupancyMaxActiveBlocksPerMultiprocessor(out, update_kernel, kThreads, update_smem_bytes(groups));
+cudaError_t update_blocks_per_sm(int groups, int packing, int* out) {
+  if (packing == kPacking8)
+    return cudaOccupancyMaxActiveBlocksPerMultiprocessor(out, update_kernel<kPacking8>, kThreads,
+                                                         update_smem_bytes(groups));
+  return cudaOccupancyMaxActiveBlocksPerMultiprocessor(out, update_kernel<kPacking1>, kThreads,
+                                                       update_smem_bytes(groups));
 }
 
-cudaError_t launch_probe_bytes(const RoundKeys& keys, uint32_t probe, int64_t first, int64_t n, uint8_t* out,
-                               int grid, cudaStream_t stream) {
-  probe_bytes_kernel<<<grid, kThreads, 0, stream>>>(keys, probe, first, n, out);
+cudaError_t launch_probe_bytes(const RoundKeys& keys, uint32_t ctr2, uint32_t bit, int64_t first, int64_t n,
+                               uint8_t* out, int grid, cudaStream_t stream) {
+  probe_bytes_kernel<<<grid, kThreads, 0, stream>>>(keys, ctr2, bit, first, n, out);
   return cudaGetLastError();
 }
 
-cudaError_t launch_probe_signs(const RoundKeys& keys, uint32_t probe, int64_t first, int64_t n, int8_t* out,
-                               int grid, cudaStream_t stream) {
-  probe_signs_kernel<<<grid, kThreads, 0, stream>>>(keys, probe, first, n, out);
+cudaError_t launch_probe_signs(const RoundKeys& keys, uint32_t ctr2, uint32_t bit, int64_t first, int64_t n,
+                               int8_t* out, int grid, cudaStream_t stream) {
+  probe_signs_kernel<<<grid, kThreads, 0, stream>>>(keys, ctr2, bit, first, n, out);
   return cudaGetLastError();
 }
 

@@ -25,7 +25,8 @@ ZO_MAX_PROBES = 1024
 
 DTYPE_CODE = {torch.float32: 0, torch.bfloat16: 1, torch.float16: 2}
 
-EXPORTS = ["zo_status_string", "zo_last_cuda_error", "zo_version", "zo_perturb", "zo_precondition",
+EXPORTS = ["zo_status_string", "zo_last_cuda_error", "zo_version", "zo_set_packing", "zo_get_packing",
+           "zo_perturb", "zo_precondition",
            "zo_precondition_ex", "zo_update", "zo_update_sequential", "zo_probe_bytes", "zo_probe_signs",
            "zo_quadratic_loss_workspace_size", "zo_quadratic_loss", "zo_quadratic_loss_static"]
 ZO_QUADRATIC_LOSS_STATIC_MAX_N = 8388608
@@ -61,6 +62,8 @@ def _lib():
             "zo_status_string": ([c.c_int], c.c_char_p),
             "zo_last_cuda_error": ([], c.c_char_p),
             "zo_version": ([], c.c_int),
+            "zo_set_packing": ([i32], c.c_int),
+            "zo_get_packing": ([], c.c_int),
             "zo_perturb": ([vp, i32, u64, u32, f32, vp], c.c_int),
             "zo_precondition": ([vp, i32, f64, vp, vp, vp], c.c_int),
             "zo_precondition_ex": ([vp, i32, f64, f64, f64, i32, vp, vp, vp, vp, vp], c.c_int),
@@ -86,6 +89,32 @@ def status_string(status: int) -> str:
 
 def version() -> int:
     return _lib().zo_version()
+
+
+def set_packing(bits_per_value: int):
+    """Probe packing of every later call: 1 (default) or 8 generated bits per
+    weight and probe (zo_set_packing)."""
+    _check("zo_set_packing", _lib().zo_set_packing(int(bits_per_value)))
+
+
+def get_packing() -> int:
+    return _lib().zo_get_packing()
+
+
+class packing:
+    """Context manager: run a block of calls under one probe packing."""
+
+    def __init__(self, bits_per_value):
+        self.bits = bits_per_value
+
+    def __enter__(self):
+        self.prev = get_packing()
+        set_packing(self.bits)
+        return self
+
+    def __exit__(self, *exc):
+        set_packing(self.prev)
+        return False
 
 
 def _check(fn, rc):

@@ -33,3 +33,14 @@ def triton_philox(tmp_path_factory):
         return np.load(dst)
 
     return run
+
+
+@pytest.fixture(params=[1, 8], ids=["pack1", "pack8"])
+def packing_mode(request):
+    """Runs a test under both probe packings, on the oracle and the library."""
+    import oracle
+    from paper_2609_38095_gb300 import build as zo_build
+    from paper_2609_38095_gb300 import zo
+    zo_build.build()
+    with oracle.packing(request.param), zo.packing(request.param):
+        yield request.param

@@ -34,7 +34,7 @@ def test_exports_every_declared_symbol(L):
 
 
 def test_version_and_strings(L):
-    assert zo.version() == 10000
+    assert zo.version() == 10100
     for s in (0, -1, -2, -3, -4, -5, -6, -7):
         assert zo.status_string(s).startswith("ZO_")
     assert "unknown" in zo.status_string(99)
@@ -125,3 +125,13 @@ def test_static_loss_validation(L):
     assert f(p, p, 16, None, None) == zo.ZO_ERR_ARG
     assert f(None, p, 16, p, None) == zo.ZO_ERR_ARG
     assert f(p, p, zo.ZO_QUADRATIC_LOSS_STATIC_MAX_N + 1, p, None) == zo.ZO_ERR_WORKSPACE
+
+
+def test_packing_switch(L):
+    assert zo.get_packing() == 1
+    assert L.zo_set_packing(3) == zo.ZO_ERR_ARG
+    assert L.zo_set_packing(0) == zo.ZO_ERR_ARG
+    assert zo.get_packing() == 1
+    with zo.packing(8):
+        assert zo.get_packing() == 8
+    assert zo.get_packing() == 1

@@ -63,6 +63,16 @@ def gather(params, t_idx, i_idx):
 
 @pytest.mark.parametrize("key", ["opt-1.3b", "qwen3-8b", "opt-13b", "opt-30b"])
 def test_fullsize_sampled_parity(key):
+    run_fullsize(key)
+
+
+def test_fullsize_sampled_parity_packing8():
+    """The 8-bit packing on the largest set (60 GB fp16, K = 256)."""
+    with oracle.packing(8), zo.packing(8):
+        run_fullsize("opt-30b")
+
+
+def run_fullsize(key):
     ps = W.BY_KEY[key]
     free, _ = torch.cuda.mem_get_info()
     if free < ps.d * ps.bytes_per_elem * 1.1:

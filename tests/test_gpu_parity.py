@@ -54,7 +54,7 @@ def assert_storage_equal(dev, host, what=""):
 @pytest.mark.parametrize("seed", [W.step_seed(0), 0xFFFFFFFFFFFFFFFF, 0])
 @pytest.mark.parametrize("probe", [0, 7, 8, 255, 1023, 5000])
 @pytest.mark.parametrize("first,n", [(0, 4096), (3, 1001), (2**33 + 5, 777)])
-def test_probe_bytes_bit_exact(seed, probe, first, n):
+def test_probe_bytes_bit_exact(seed, probe, first, n, packing_mode):
     got = zo.probe_bytes(seed, probe, first, n).cpu().numpy()
     want = oracle.probe_bytes(seed, probe, first, n)
     np.testing.assert_array_equal(got, want)
@@ -63,14 +63,14 @@ def test_probe_bytes_bit_exact(seed, probe, first, n):
 @pytest.mark.parametrize("seed", [W.step_seed(3), 0xFFFFFFFFFFFFFFFF])
 @pytest.mark.parametrize("probe", [0, 5, 9, 1023])
 @pytest.mark.parametrize("first,n", [(0, 5000), (13, 333), (2**36 + 1, 1000)])
-def test_probe_signs_bit_exact(seed, probe, first, n):
+def test_probe_signs_bit_exact(seed, probe, first, n, packing_mode):
     got = zo.probe_signs(seed, probe, first, n).cpu().numpy()
     want = oracle.probe_signs(seed, probe, first, n)
     np.testing.assert_array_equal(got, want)
 
 
 # ------------------------------------------------------------------ perturb
-def test_perturb_bit_exact_mixed_sequence():
+def test_perturb_bit_exact_mixed_sequence(packing_mode):
     host, dev = make_list(MIXED_NUMELS, MIXED_DTYPES)
     plist = zo.ParamList(dev)
     dts = [TORCH_TO_DT[d] for d in MIXED_DTYPES]
@@ -110,7 +110,7 @@ def test_perturb_unaligned_views(dtype, offset):
     np.testing.assert_array_equal(after[offset + n:], base_host[offset + n:])
 
 
-def test_perturb_many_tensors_split_launches():
+def test_perturb_many_tensors_split_launches(packing_mode):
     """More tensors than one launch's table holds (1024)."""
     rng = np.random.default_rng(12)
     numels = [int(x) for x in rng.integers(0, 300, 2500)]
@@ -163,7 +163,7 @@ def test_empty_and_zero_length():
 
 # ------------------------------------------------------------------- update
 @pytest.mark.parametrize("K", [1, 3, 8, 13, 64, 256])
-def test_update_within_tolerance(K):
+def test_update_within_tolerance(K, packing_mode):
     host, dev = make_list(MIXED_NUMELS, MIXED_DTYPES, seed=K)
     dts = [TORCH_TO_DT[d] for d in MIXED_DTYPES]
     rng = np.random.default_rng(100 + K)
@@ -182,7 +182,7 @@ def test_update_within_tolerance(K):
     assert equal >= 0.95 * total
 
 
-def test_update_max_probes():
+def test_update_max_probes(packing_mode):
     K = zo.ZO_MAX_PROBES
     host, dev = make_list([5003, 16, 1], [torch.float32, torch.bfloat16, torch.float16], seed=77)
     dts = [W.DT_F32, W.DT_BF16, W.DT_F16]
@@ -198,7 +198,7 @@ def test_update_max_probes():
 
 
 @pytest.mark.parametrize("K", [1, 5, 16])
-def test_update_sequential_bit_exact(K):
+def test_update_sequential_bit_exact(K, packing_mode):
     host, dev = make_list(MIXED_NUMELS, MIXED_DTYPES, seed=50 + K)
     dts = [TORCH_TO_DT[d] for d in MIXED_DTYPES]
     c_np = np.random.default_rng(K).normal(0, 25, K)

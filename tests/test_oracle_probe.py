@@ -106,3 +106,52 @@ def test_virtual_offsets():
     numel = [0, 1, 16, 17, 31, 32, 5]
     want = [0, 0, 16, 32, 64, 96, 128]
     np.testing.assert_array_equal(oracle.virtual_offsets(numel), want)
+
+
+def independent_signs_p8(triton_philox, seed, k, g):
+    """Packing 8: z_k[g] = bit 0 of byte g mod 16 of Philox(g/16, k, 0)."""
+    g = np.asarray(g, dtype=np.uint64)
+    blocks = g // np.uint64(16)
+    N = 1
+    while N < len(blocks):
+        N *= 2
+    ctr = np.zeros((1, N, 4), dtype=np.uint32)
+    ctr[0, : len(blocks), 0] = (blocks & np.uint64(U32)).astype(np.uint32)
+    ctr[0, : len(blocks), 1] = (blocks >> np.uint64(32)).astype(np.uint32)
+    ctr[0, :, 2] = k
+    words = triton_philox([seed], ctr)[0, : len(blocks)]
+    by = np.ascontiguousarray(words.astype("<u4")).view(np.uint8).reshape(-1, 16)
+    b = by[np.arange(len(g)), (g % np.uint64(16)).astype(np.int64)] & 1
+    return b.astype(np.int8) * 2 - 1
+
+
+@pytest.mark.parametrize("k", [0, 3, 8, 1023])
+def test_probe_signs_packing8_independent_route(triton_philox, k):
+    import oracle as O
+    seed = 0x15E5A0003
+    rng = np.random.default_rng(k + 50)
+    g = np.concatenate([np.arange(0, 64), rng.integers(0, 2**40, 200)]).astype(np.uint64)
+    want = independent_signs_p8(triton_philox, seed, k, g)
+    with O.packing(8):
+        got = np.array([O.probe_sign(seed, k, int(x)) for x in g], dtype=np.int8)
+    np.testing.assert_array_equal(got, want)
+
+
+def test_packing8_balance_and_independence():
+    import oracle as O
+    n = 1 << 18
+    seed = 0x15E5A0000
+    with O.packing(8):
+        zs = [O.probe_signs(seed, k, 0, n).astype(np.float64) for k in (0, 1, 7, 8)]
+        packed = O.probe_bytes(seed, 5, 0, 1000)
+        signs = O.probe_signs(seed, 5, 0, 8000)
+    np.testing.assert_array_equal(np.unpackbits(packed, bitorder="little").astype(np.int8) * 2 - 1, signs)
+    sigma = 1.0 / np.sqrt(n)
+    for z in zs:
+        assert abs(z.mean()) < 5 * sigma
+    for a in range(4):
+        for b in range(a + 1, 4):
+            assert abs(np.mean(zs[a] * zs[b])) < 5 * sigma
+    # the two packings define different probes
+    z1 = oracle.probe_signs(seed, 1, 0, n).astype(np.float64)
+    assert abs(np.mean(z1 * zs[1])) < 5 * sigma
