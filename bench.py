@@ -52,6 +52,9 @@ def parse_args():
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--packing", type=int, default=1, choices=[1, 8],
                     help="generated bits per (weight, probe): 1 (the paper's bit packing) or 8")
+    ap.add_argument("--schedule", default="fused", choices=["fused", "alg1"],
+                    help="fused: each restore is folded into the next probe's +eps pass and the last one into "
+                         "the update (2K+1 passes); alg1: Algorithm 1's +eps, -2eps, +eps per probe (3K+1)")
     ap.add_argument("--sequential", action="store_true",
                     help="also time Algorithm 1's K sequential passes against the fused update")
     return ap.parse_args()
@@ -270,32 +273,37 @@ def run_zo(args):
     stream = torch.cuda.current_stream(dev)
     chunks = (len(params) + 1023) // 1024
 
-    timing = {"perturb": [], "update": [], "precondition": []}
+    timing = {"perturb": [], "perturb2": [], "update": [], "precondition": []}
+    fused = args.schedule == "fused"
+
+    def timed(key, record, fn, *a, **kw):
+        if not record:
+            return fn(*a, **kw)
+        e0 = torch.cuda.Event(enable_timing=True)
+        e1 = torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        fn(*a, **kw)
+        e1.record(stream)
+        timing[key].append((e0, e1))
 
     def step(s, losses_d, record):
+        """One step; the forward passes (out of scope) would sit after each
+        +eps and each -2eps pass. The fused schedule leaves the weights at
+        those points, and at the end, bit for bit as Algorithm 1's does."""
         seed = W.step_seed(s)
-        for k in range(K):
-            for sc in (eps, -2 * eps, eps):
-                if record:
-                    e0 = torch.cuda.Event(enable_timing=True)
-                    e1 = torch.cuda.Event(enable_timing=True)
-                    e0.record(stream)
-                    zo.perturb(plist, seed, k, sc)
-                    e1.record(stream)
-                    timing["perturb"].append((e0, e1))
-                else:
-                    zo.perturb(plist, seed, k, sc)
-        if record:
-            e0, e1, e2 = (torch.cuda.Event(enable_timing=True) for _ in range(3))
-            e0.record(stream)
-        zo.precondition(losses_d, eps, out=(c, status))
-        if record:
-            e1.record(stream)
-        zo.update(plist, seed, c, eps, status=status)
-        if record:
-            e2.record(stream)
-            timing["precondition"].append((e0, e1))
-            timing["update"].append((e1, e2))
+        if fused:
+            timed("perturb", record, zo.perturb, plist, seed, 0, eps)
+            for k in range(K):
+                timed("perturb", record, zo.perturb, plist, seed, k, -2 * eps)
+                if k + 1 < K:
+                    timed("perturb2", record, zo.perturb2, plist, seed, k, eps, k + 1, eps)
+        else:
+            for k in range(K):
+                for sc in (eps, -2 * eps, eps):
+                    timed("perturb", record, zo.perturb, plist, seed, k, sc)
+        timed("precondition", record, zo.precondition, losses_d, eps, out=(c, status))
+        timed("update", record, zo.update, plist, seed, c, eps, status=status,
+              pre=(K - 1, eps) if fused else None)
 
     for s in range(args.warmup):
         step(s, losses_dev[s], record=False)
@@ -320,13 +328,15 @@ def run_zo(args):
     clk = clocks.stop()
     elapsed_ms = ranks_max(t_start.elapsed_time(t_end))
     ms_per_step = elapsed_ms / args.steps
-    launches = args.steps * (3 * K * chunks + 1 + chunks)
+    passes = 2 * K + 1 if fused else 3 * K + 1   # sweeps over the weights per step (update included)
+    launches = args.steps * ((passes - 1) * chunks + 1 + chunks)
 
     def avg_ms(key):
         v = [a.elapsed_time(b) for a, b in timing[key]]
-        return sum(v) / len(v)
+        return sum(v) / len(v) if v else 0.0
 
     perturb_ms = ranks_max(avg_ms("perturb"))
+    perturb2_ms = ranks_max(avg_ms("perturb2"))
     update_ms = ranks_max(avg_ms("update"))
     precond_ms = ranks_max(avg_ms("precondition"))
 
@@ -396,6 +406,7 @@ def run_zo(args):
         "warmup": args.warmup, "ms_per_step": ms_per_step, "higher_is_better": True, "scaling": "weak",
         "vs_baseline": None, "dtype": "f32", "data": "synthetic",
         "config": {"workload": ps.name, "K": K, "d": d, "tensors": len(params), "packing": args.packing,
+                   "schedule": f"{args.schedule} ({passes} passes over the weights per step)",
                    "storage": "fp16" if
                    ps.dtype == W.DT_F16 else ("bf16" if ps.dtype == W.DT_BF16 else "fp32"),
                    "eps": eps, "lr": eps, "parallelism": f"replicas{world}",
@@ -405,7 +416,13 @@ def run_zo(args):
                      "peak_source": f"{peak_kind} hbm_gbs", "bytes_per_launch": perturb_bytes},
         "kernels": {
             "perturb": {"ms": perturb_ms, "GB/s": achieved, "frac_of_measured_hbm": achieved / hbm_peak,
-                        "frac_of_nominal_hbm": achieved / NOMINAL_HBM_GBS, "launches_per_step": 3 * K * chunks},
+                        "frac_of_nominal_hbm": achieved / NOMINAL_HBM_GBS,
+                        "launches_per_step": (K + 1 if fused else 3 * K) * chunks},
+            "perturb2": ({"ms": perturb2_ms, "GB/s": perturb_bytes / (perturb2_ms * 1e-3) / 1e9,
+                          "frac_of_measured_hbm": perturb_bytes / (perturb2_ms * 1e-3) / 1e9 / hbm_peak,
+                          "launches_per_step": (K - 1) * chunks} if fused and K > 1 else None),
+            "step_hbm": {"passes": passes, "ideal_ms": passes * perturb_bytes / (hbm_peak * 1e9) * 1e3,
+                         "frac": passes * perturb_bytes / (hbm_peak * 1e9) / (ms_per_step * 1e-3)},
             "update": {"ms": update_ms, "gparam_probe_per_s": upd_rate, "bound": "alu",
                        "peak_gparam_probe_per_s_1instr": alu_peak, "frac_alu_1instr": upd_rate / alu_peak,
                        "GB/s": perturb_bytes / (update_ms * 1e-3) / 1e9},

@@ -123,6 +123,18 @@ int zo_perturb(const zo_tensor* params, int32_t n_tensors, uint64_t seed, uint32
                void* stream);
 
 /* ---------------------------------------------------------------------------
+ * zo_perturb2 -- two consecutive perturbations in one pass over theta:
+ * exactly zo_perturb(probe_a, scale_a) followed by zo_perturb(probe_b,
+ * scale_b) (each result rounded to storage, bit for bit the same), with one
+ * read and one write of every weight instead of two. In Algorithm 1 no
+ * forward pass runs between probe k's restore (+eps) and probe k+1's first
+ * perturbation (+eps), so a step can apply them together:
+ * zo_perturb2(k, +eps, k + 1, +eps). Errors as zo_perturb.
+ * ------------------------------------------------------------------------- */
+int zo_perturb2(const zo_tensor* params, int32_t n_tensors, uint64_t seed, uint32_t probe_a, float scale_a,
+                uint32_t probe_b, float scale_b, void* stream);
+
+/* ---------------------------------------------------------------------------
  * zo_precondition -- the probe-space diagonal preconditioner of Sec. 4.1 with
  * the paper's settings (alpha = 0.1, lambda_reg = 1, two-sided difference).
  * For each probe k, from losses row k = {L+_k, L-_k, L0_k} (device, K x 3 fp64,
@@ -165,6 +177,16 @@ int zo_precondition_ex(const double* losses, int32_t K, double eps, double alpha
  * ------------------------------------------------------------------------- */
 int zo_update(const zo_tensor* params, int32_t n_tensors, uint64_t seed, const double* c, int32_t K, double lr,
               const int32_t* status, void* stream);
+
+/* zo_update preceded, in the same pass, by one perturbation: exactly
+ * zo_perturb(pre_probe, pre_scale) then zo_update(...) (the perturbed value
+ * is rounded to storage before the probe sum is added), with one read and
+ * one write of theta. Used to fold the last probe's restore (+eps) into the
+ * update. has_pre = 0 makes it zo_update. When `status` holds anything but
+ * ZO_OK only the leading perturbation is applied (a restore must always
+ * happen). Errors as zo_update (ZO_ERR_ARG also for a non-finite pre_scale). */
+int zo_update_ex(const zo_tensor* params, int32_t n_tensors, uint64_t seed, const double* c, int32_t K, double lr,
+                 const int32_t* status, int32_t has_pre, uint32_t pre_probe, float pre_scale, void* stream);
 
 /* Comparator with Algorithm 1's own schedule: K in-place passes, pass k adds
  * a_k z_k (same a_k as zo_update) and rounds to storage, exactly as

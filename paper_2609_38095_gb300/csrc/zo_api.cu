@@ -56,6 +56,16 @@ void probe_counter(uint32_t k, int packing, uint32_t* ctr2, uint32_t* bit) {
   }
 }
 
+// theta <- rn(theta + scale z_k) as a kernel operand.
+zo::PerturbOp make_op(uint32_t k, float scale, int packing) {
+  zo::PerturbOp op;
+  probe_counter(k, packing, &op.ctr2, &op.bit);
+  uint32_t u;
+  std::memcpy(&u, &scale, sizeof(u));
+  op.nscale_bits = u ^ 0x80000000u;  // -scale: the probe bit flips it to +scale
+  return op;
+}
+
 // Resident perturb blocks per SM. The pass is HBM-bound and each thread keeps
 // two 32-byte loads in flight; on GB300 four 256-thread blocks per SM stream
 // fastest (measured: 3 -> 90.6 %, 4 -> 97.7 %, 5 -> 93.0 % of the copy
@@ -214,8 +224,30 @@ int zo_perturb(const zo_tensor* params, int32_t n_tensors, uint64_t seed, uint32
   PerturbParams& pp = tl_perturb;
   pp.keys = expand_keys(seed);
   pp.probe = probe;
-  probe_counter(probe, g_packing.load(), &pp.ctr2, &pp.bit);
-  pp.scale = scale;
+  pp.op[0] = make_op(probe, scale, g_packing.load());
+  pp.op[1] = pp.op[0];
+  pp.nops = 1;
+  pp.coef = nullptr;
+  pp.coef_mul = 0.0;
+  pp.status = nullptr;
+  return run_perturb(params, n_tensors, pp, d, static_cast<cudaStream_t>(stream));
+}
+
+int zo_perturb2(const zo_tensor* params, int32_t n_tensors, uint64_t seed, uint32_t probe_a, float scale_a,
+                uint32_t probe_b, float scale_b, void* stream) {
+  int rc = validate_params(params, n_tensors);
+  if (rc != ZO_OK) return rc;
+  if (!std::isfinite(scale_a) || !std::isfinite(scale_b)) return ZO_ERR_ARG;
+  if (n_tensors == 0) return ZO_OK;
+  DeviceInfo* d = nullptr;
+  if ((rc = device_info(&d)) != ZO_OK) return rc;
+  const int packing = g_packing.load();
+  PerturbParams& pp = tl_perturb;
+  pp.keys = expand_keys(seed);
+  pp.probe = probe_a;
+  pp.op[0] = make_op(probe_a, scale_a, packing);
+  pp.op[1] = make_op(probe_b, scale_b, packing);
+  pp.nops = 2;
   pp.coef = nullptr;
   pp.coef_mul = 0.0;
   pp.status = nullptr;
@@ -233,8 +265,15 @@ static int check_update_args(const zo_tensor* params, int32_t n, const double* c
 
 int zo_update(const zo_tensor* params, int32_t n_tensors, uint64_t seed, const double* c, int32_t K, double lr,
               const int32_t* status, void* stream) {
+  return zo_update_ex(params, n_tensors, seed, c, K, lr, status, 0, 0u, 0.0f, stream);
+}
+
+int zo_update_ex(const zo_tensor* params, int32_t n_tensors, uint64_t seed, const double* c, int32_t K, double lr,
+                 const int32_t* status, int32_t has_pre, uint32_t pre_probe, float pre_scale, void* stream) {
   int rc = check_update_args(params, n_tensors, c, K, lr);
-  if (rc != ZO_OK || n_tensors == 0) return rc;
+  if (rc != ZO_OK) return rc;
+  if (has_pre != 0 && !std::isfinite(pre_scale)) return ZO_ERR_ARG;
+  if (n_tensors == 0) return rc;
   DeviceInfo* d = nullptr;
   if ((rc = device_info(&d)) != ZO_OK) return rc;
   UpdateParams& up = tl_update;
@@ -244,6 +283,8 @@ int zo_update(const zo_tensor* params, int32_t n_tensors, uint64_t seed, const d
   up.K = K;
   up.groups = (K + 7) / 8;
   up.packing = g_packing.load();
+  up.has_pre = has_pre != 0;
+  up.pre = make_op(pre_probe, has_pre != 0 ? pre_scale : 0.0f, up.packing);
   up.status = status;
   int bps = 1;
   if ((rc = update_blocks_per_sm(d, up.groups, up.packing, &bps)) != ZO_OK) return rc;
@@ -269,14 +310,15 @@ int zo_update_sequential(const zo_tensor* params, int32_t n_tensors, uint64_t se
   if ((rc = device_info(&d)) != ZO_OK) return rc;
   PerturbParams& pp = tl_perturb;
   pp.keys = expand_keys(seed);
-  pp.scale = 0.0f;
   pp.coef = c;
   pp.coef_mul = -(lr / static_cast<double>(K));
   pp.status = status;
+  pp.nops = 1;
   const int packing = g_packing.load();
   for (int32_t k = 0; k < K; ++k) {
     pp.probe = static_cast<uint32_t>(k);
-    probe_counter(pp.probe, packing, &pp.ctr2, &pp.bit);
+    pp.op[0] = make_op(pp.probe, 0.0f, packing);  // scale read from c on the device
+    pp.op[1] = pp.op[0];
     if ((rc = run_perturb(params, n_tensors, pp, d, static_cast<cudaStream_t>(stream))) != ZO_OK) return rc;
   }
   return ZO_OK;

@@ -14,21 +14,81 @@ namespace zo {
 // ---------------------------------------------------------------------------
 // Perturb: theta <- rn(fp32(theta) + scale * z_k) in place.
 //
-// z_k[g] is bit (k mod 8) of byte (g mod 16) of Philox(b = g/16, q = k/8).
-// Byte m sits at bits 8(m mod 4).. of word m/4; shifting the word left by
-// 31 - 8(m mod 4) - (k mod 8) puts the probe bit in the sign position, which
-// then flips -scale into +scale (bit 1 -> z = +1). The product scale * z is
-// exact, so the element result is one fp32 add and one rounding to storage.
+// z_k[g] is bit `bit` of byte (g mod 16) of Philox(b = g/16, ctr2) (packing 1:
+// ctr2 = k/8, bit = k mod 8; packing 8: ctr2 = k, bit = 0). Byte m sits at
+// bits 8(m mod 4).. of word m/4; shifting the word left by
+// 31 - 8(m mod 4) - bit puts the probe bit in the sign position, which then
+// flips -scale into +scale (bit 1 -> z = +1). The product scale * z is exact,
+// so the element result is one fp32 add and one rounding to storage.
+//
+// A launch may apply two perturbations in sequence (zo_perturb2): the value
+// is rounded to storage after each, exactly as two separate passes would,
+// but theta crosses HBM once.
 // ---------------------------------------------------------------------------
 // Probe bit of element i (0..15) of a block, moved to bit 31.
 __device__ __forceinline__ uint32_t sign_bit(const uint4& x, int i, uint32_t j) {
   return (word_of(x, i >> 2) << (31u - 8u * static_cast<uint32_t>(i & 3) - j)) & 0x80000000u;
 }
 
-template <uint8_t DT>
-__device__ __forceinline__ void perturb_block_vec(void* base, int64_t e0, const uint4& x, uint32_t nscale_bits,
-                                                  uint32_t j) {
-  if constexpr (DT == kF32) {
+__device__ __forceinline__ float add_signed(float th, const uint4& x, int i, const PerturbOp& op) {
+  return __fadd_rn(th, __uint_as_float(op.nscale_bits ^ sign_bit(x, i, op.bit)));
+}
+
+__device__ __forceinline__ uint4 block_bits(int64_t b, uint32_t ctr2, const RoundKeys& keys) {
+  return philox10(static_cast<uint32_t>(b), static_cast<uint32_t>(static_cast<uint64_t>(b) >> 32), ctr2, 0u, keys);
+}
+
+// Sixteen 16-bit weights in registers (element 2r in the low half of v[r]).
+template <uint8_t DT, int NOPS>
+__device__ __forceinline__ void perturb_regs16(uint32_t (&v)[8], const uint4 (&x)[2], const PerturbOp (&op)[2]) {
+#pragma unroll
+  for (int r = 0; r < 8; ++r) {
+#pragma unroll
+    for (int o = 0; o < NOPS; ++o) {
+      const float2 f = unpack2<DT>(v[r]);
+      v[r] = pack2<DT>(add_signed(f.x, x[o], 2 * r, op[o]), add_signed(f.y, x[o], 2 * r + 1, op[o]));
+    }
+  }
+}
+
+// A thread's position in the tensor table. Its blocks only move forward and
+// usually stay inside one tensor, so the table is re-read only when a block
+// leaves the current tensor.
+struct Cursor {
+  int t;           // tensor index
+  int64_t tb;      // first virtual block of tensor t
+  int64_t te;      // one past its last block
+  int64_t tfe;     // one past its last full block when it takes the pipelined path, else tb
+  uint16_t* tp;    // base pointer
+  uint8_t dt;      // storage dtype
+};
+
+__device__ __forceinline__ void cursor_seek(const TensorTable& tab, Cursor& c, int64_t b) {
+  c.t = advance_tensor(tab, c.t, b);
+  c.tb = tensor_blk_begin(tab, c.t);
+  c.te = tab.blk_end[c.t];
+  const uint8_t fl = tab.flags[c.t];
+  c.dt = fl & kDtypeMask;
+  // pipelined path: full, 32-byte aligned blocks of a 16-bit tensor
+  c.tfe = ((fl & kVec32) && c.dt != kF32) ? c.tb + tab.numel[c.t] / 16 : c.tb;
+  c.tp = reinterpret_cast<uint16_t*>(tab.ptr[c.t]);
+}
+
+// Address of block b (inside the cursor's tensor) on the pipelined path, else nullptr.
+__device__ __forceinline__ uint16_t* fast16_block(const Cursor& c, int64_t b) {
+  return b < c.tfe ? c.tp + (b - c.tb) * 16 : nullptr;
+}
+
+// Any other block: fp32, a partial last block, or an unaligned tensor.
+template <int NOPS>
+__device__ __noinline__ void perturb_block_other(const TensorTable& tab, int t, int64_t b, uint4 x0, uint4 x1,
+                                                 PerturbOp op0, PerturbOp op1) {
+  const int64_t e0 = (b - tensor_blk_begin(tab, t)) * 16;
+  const int64_t cnt = min(static_cast<int64_t>(16), tab.numel[t] - e0);
+  const uint8_t fl = tab.flags[t];
+  const uint8_t dt = fl & kDtypeMask;
+  void* base = reinterpret_cast<void*>(tab.ptr[t]);
+  if (cnt == 16 && (fl & kVec32) && dt == kF32) {
     float* p = static_cast<float*>(base) + e0;
 #pragma unroll
     for (int half = 0; half < 2; ++half) {
@@ -36,67 +96,17 @@ __device__ __forceinline__ void perturb_block_vec(void* base, int64_t e0, const 
       ld256(p + 8 * half, v);
 #pragma unroll
       for (int r = 0; r < 8; ++r) {
-        const int i = 8 * half + r;  // element within the block
-        const float d = __uint_as_float(nscale_bits ^ sign_bit(x, i, j));
-        v[r] = __float_as_uint(__fadd_rn(__uint_as_float(v[r]), d));
+        float th = add_signed(__uint_as_float(v[r]), x0, 8 * half + r, op0);
+        if (NOPS == 2) th = add_signed(th, x1, 8 * half + r, op1);
+        v[r] = __float_as_uint(th);
       }
       st256(p + 8 * half, v);
     }
   } else {
-    uint16_t* p = static_cast<uint16_t*>(base) + e0;
-    uint32_t v[8];
-    ld256(p, v);
-#pragma unroll
-    for (int r = 0; r < 8; ++r) {
-      const float2 f = unpack2<DT>(v[r]);
-      const float r0 = __fadd_rn(f.x, __uint_as_float(nscale_bits ^ sign_bit(x, 2 * r, j)));
-      const float r1 = __fadd_rn(f.y, __uint_as_float(nscale_bits ^ sign_bit(x, 2 * r + 1, j)));
-      v[r] = pack2<DT>(r0, r1);
-    }
-    st256(p, v);
-  }
-}
-
-template <uint8_t DT>
-__device__ __forceinline__ void perturb_regs16(uint32_t (&v)[8], const uint4& x, uint32_t nscale_bits, uint32_t j) {
-#pragma unroll
-  for (int r = 0; r < 8; ++r) {
-    const float2 f = unpack2<DT>(v[r]);
-    const float r0 = __fadd_rn(f.x, __uint_as_float(nscale_bits ^ sign_bit(x, 2 * r, j)));
-    const float r1 = __fadd_rn(f.y, __uint_as_float(nscale_bits ^ sign_bit(x, 2 * r + 1, j)));
-    v[r] = pack2<DT>(r0, r1);
-  }
-}
-
-// Address of block b of tensor t when it takes the pipelined path (a full,
-// 32-byte aligned block of a 16-bit tensor), else nullptr.
-__device__ __forceinline__ uint16_t* fast16_block(const TensorTable& tab, int t, int64_t b) {
-  const int64_t e0 = (b - tensor_blk_begin(tab, t)) * 16;
-  const uint8_t fl = tab.flags[t];
-  if ((fl & kVec32) && (fl & kDtypeMask) != kF32 && tab.numel[t] - e0 >= 16)
-    return reinterpret_cast<uint16_t*>(tab.ptr[t]) + e0;
-  return nullptr;
-}
-
-// Any other block: fp32, a partial last block, or an unaligned tensor.
-__device__ __noinline__ void perturb_block_other(const TensorTable& tab, int t, int64_t b, uint4 x,
-                                                 uint32_t nscale_bits, uint32_t j) {
-  const int64_t e0 = (b - tensor_blk_begin(tab, t)) * 16;
-  const int64_t cnt = min(static_cast<int64_t>(16), tab.numel[t] - e0);
-  const uint8_t fl = tab.flags[t];
-  const uint8_t dt = fl & kDtypeMask;
-  void* base = reinterpret_cast<void*>(tab.ptr[t]);
-  if (cnt == 16 && (fl & kVec32)) {
-    if (dt == kBF16)
-      perturb_block_vec<kBF16>(base, e0, x, nscale_bits, j);
-    else if (dt == kF16)
-      perturb_block_vec<kF16>(base, e0, x, nscale_bits, j);
-    else
-      perturb_block_vec<kF32>(base, e0, x, nscale_bits, j);
-  } else {
     for (int i = 0; i < cnt; ++i) {
-      const float th = load_elem(base, dt, e0 + i);
-      store_elem(base, dt, e0 + i, __fadd_rn(th, __uint_as_float(nscale_bits ^ sign_bit(x, i, j))));
+      float th = add_signed(load_elem(base, dt, e0 + i), x0, i, op0);
+      if (NOPS == 2) th = add_signed(round_to_storage(dt, th), x1, i, op1);
+      store_elem(base, dt, e0 + i, th);
     }
   }
 }
@@ -105,47 +115,53 @@ __device__ __noinline__ void perturb_block_other(const TensorTable& tab, int t, 
 // 16-bit block is issued before the current block is computed and stored, so
 // each thread keeps two loads in flight (the pass is HBM-bound and needs the
 // bytes in flight to cover DRAM latency).
+template <int NOPS>
 __global__ void __launch_bounds__(256) perturb_kernel(const __grid_constant__ PerturbParams P) {
   if (P.status != nullptr && *P.status != 0) return;
-  float scale = P.scale;
-  if (P.coef != nullptr) scale = __double2float_rn(P.coef_mul * P.coef[P.probe]);
-  const uint32_t nscale_bits = __float_as_uint(scale) ^ 0x80000000u;  // -scale
-  const uint32_t j = P.bit;
-  const uint32_t q = P.ctr2;
+  PerturbOp op[2] = {P.op[0], P.op[1]};
+  if (P.coef != nullptr)
+    op[0].nscale_bits = __float_as_uint(__double2float_rn(P.coef_mul * P.coef[P.probe])) ^ 0x80000000u;
+  const bool same_ctr = op[1].ctr2 == op[0].ctr2;
 
   const TensorTable& tab = P.tab;
   const int64_t blk_total = tab.blk_end[tab.n - 1];
   const int64_t stride = static_cast<int64_t>(gridDim.x) * blockDim.x;
   int64_t b = tab.blk_begin + static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x;
   if (b >= blk_total) return;
-  int t = advance_tensor(tab, 0, b);
-  uint16_t* p = fast16_block(tab, t, b);
+  Cursor c;
+  c.t = 0;
+  cursor_seek(tab, c, b);
+  int t = c.t;          // tensor and dtype of the current block
+  uint8_t dt = c.dt;
+  uint16_t* p = fast16_block(c, b);
   uint32_t v[8];
   if (p != nullptr) ld256(p, v);
   while (true) {
     const int64_t bn = b + stride;
-    int tn = t;
     uint16_t* pn = nullptr;
     uint32_t vn[8];
     if (bn < blk_total) {
-      tn = advance_tensor(tab, t, bn);
-      pn = fast16_block(tab, tn, bn);
+      if (bn >= c.te) cursor_seek(tab, c, bn);
+      pn = fast16_block(c, bn);
       if (pn != nullptr) ld256(pn, vn);
     }
-    const uint4 x = philox10(static_cast<uint32_t>(b), static_cast<uint32_t>(static_cast<uint64_t>(b) >> 32), q, 0u,
-                             P.keys);
+    uint4 x[2];
+    x[0] = block_bits(b, op[0].ctr2, P.keys);
+    x[1] = x[0];
+    if (NOPS == 2 && !same_ctr) x[1] = block_bits(b, op[1].ctr2, P.keys);
     if (p != nullptr) {
-      if ((tab.flags[t] & kDtypeMask) == kBF16)
-        perturb_regs16<kBF16>(v, x, nscale_bits, j);
+      if (dt == kBF16)
+        perturb_regs16<kBF16, NOPS>(v, x, op);
       else
-        perturb_regs16<kF16>(v, x, nscale_bits, j);
+        perturb_regs16<kF16, NOPS>(v, x, op);
       st256(p, v);
     } else {
-      perturb_block_other(tab, t, b, x, nscale_bits, j);
+      perturb_block_other<NOPS>(tab, t, b, x[0], x[1], op[0], op[1]);
     }
     if (bn >= blk_total) break;
     b = bn;
-    t = tn;
+    t = c.t;
+    dt = c.dt;
     p = pn;
 #pragma unroll
     for (int r = 0; r < 8; ++r) v[r] = vn[r];
@@ -253,32 +269,51 @@ __device__ __forceinline__ void accumulate_any(float (&acc)[16], int64_t b, cons
 
 // One full, 32-byte aligned block: theta is loaded before the probe loop so
 // the load overlaps the arithmetic.
+// Leading perturbation of zo_update_ex, rounded to storage (16-bit pairs).
+template <uint8_t DT>
+__device__ __forceinline__ uint32_t pre_regs16(uint32_t v, const uint4& xp, int r, const PerturbOp& op) {
+  const float2 f = unpack2<DT>(v);
+  return pack2<DT>(add_signed(f.x, xp, 2 * r, op), add_signed(f.y, xp, 2 * r + 1, op));
+}
+
 template <int PACK, uint8_t DT>
 __device__ __forceinline__ void update_block_vec(void* base, int64_t e0, int64_t b, const UpdateParams& P,
-                                                 uint32_t lut_base) {
+                                                 uint32_t lut_base, bool do_sum) {
   float acc[16];
 #pragma unroll
   for (int m = 0; m < 16; ++m) acc[m] = 0.0f;
   if constexpr (DT == kF32) {
-    accumulate_any<PACK>(acc, b, P, lut_base);
+    if (do_sum) accumulate_any<PACK>(acc, b, P, lut_base);
+    uint4 xp = make_uint4(0u, 0u, 0u, 0u);
+    if (P.has_pre) xp = block_bits(b, P.pre.ctr2, P.keys);
     float* p = static_cast<float*>(base) + e0;
 #pragma unroll
     for (int half = 0; half < 2; ++half) {
       uint32_t v[8];
       ld256(p + 8 * half, v);
 #pragma unroll
-      for (int r = 0; r < 8; ++r) v[r] = __float_as_uint(__fadd_rn(__uint_as_float(v[r]), acc[8 * half + r]));
+      for (int r = 0; r < 8; ++r) {
+        float th = __uint_as_float(v[r]);
+        if (P.has_pre) th = add_signed(th, xp, 8 * half + r, P.pre);
+        if (do_sum) th = __fadd_rn(th, acc[8 * half + r]);
+        v[r] = __float_as_uint(th);
+      }
       st256(p + 8 * half, v);
     }
   } else {
     uint16_t* p = static_cast<uint16_t*>(base) + e0;
     uint32_t v[8];
     ld256(p, v);
-    accumulate_any<PACK>(acc, b, P, lut_base);
+    if (do_sum) accumulate_any<PACK>(acc, b, P, lut_base);
+    uint4 xp = make_uint4(0u, 0u, 0u, 0u);
+    if (P.has_pre) xp = block_bits(b, P.pre.ctr2, P.keys);
 #pragma unroll
     for (int r = 0; r < 8; ++r) {
-      const float2 f = unpack2<DT>(v[r]);
-      v[r] = pack2<DT>(__fadd_rn(f.x, acc[2 * r]), __fadd_rn(f.y, acc[2 * r + 1]));
+      if (P.has_pre) v[r] = pre_regs16<DT>(v[r], xp, r, P.pre);
+      if (do_sum) {
+        const float2 f = unpack2<DT>(v[r]);
+        v[r] = pack2<DT>(__fadd_rn(f.x, acc[2 * r]), __fadd_rn(f.y, acc[2 * r + 1]));
+      }
     }
     st256(p, v);
   }
@@ -297,7 +332,8 @@ __global__ void __launch_bounds__(256) update_kernel(const __grid_constant__ Upd
   for (int k = threadIdx.x; k < npad; k += blockDim.x)
     a_s[k] = k < P.K ? __double2float_rn(P.coef_mul * P.coef[k]) : 0.0f;
   __syncthreads();
-  if (skip) return;
+  if (skip && !P.has_pre) return;
+  const bool do_sum = !skip;  // a failed preconditioner still gets the leading perturbation
   for (int e = threadIdx.x; e < 32 * P.groups; e += blockDim.x) {
     const int h = e >> 4, n = e & 15;
     const float* a = a_s + 4 * h;
@@ -323,19 +359,26 @@ __global__ void __launch_bounds__(256) update_kernel(const __grid_constant__ Upd
     void* base = reinterpret_cast<void*>(tab.ptr[t]);
     if (cnt == 16 && (fl & kVec32)) {
       if (dt == kBF16)
-        update_block_vec<PACK, kBF16>(base, e0, b, P, lut_base);
+        update_block_vec<PACK, kBF16>(base, e0, b, P, lut_base, do_sum);
       else if (dt == kF16)
-        update_block_vec<PACK, kF16>(base, e0, b, P, lut_base);
+        update_block_vec<PACK, kF16>(base, e0, b, P, lut_base, do_sum);
       else
-        update_block_vec<PACK, kF32>(base, e0, b, P, lut_base);
+        update_block_vec<PACK, kF32>(base, e0, b, P, lut_base, do_sum);
     } else {
       float acc[16];
 #pragma unroll
       for (int m = 0; m < 16; ++m) acc[m] = 0.0f;
-      accumulate_any<PACK>(acc, b, P, lut_base);
+      if (do_sum) accumulate_any<PACK>(acc, b, P, lut_base);
+      uint4 xp = make_uint4(0u, 0u, 0u, 0u);
+      if (P.has_pre) xp = block_bits(b, P.pre.ctr2, P.keys);
 #pragma unroll
       for (int i = 0; i < 16; ++i) {
-        if (i < cnt) store_elem(base, dt, e0 + i, __fadd_rn(load_elem(base, dt, e0 + i), acc[i]));
+        if (i < cnt) {
+          float th = load_elem(base, dt, e0 + i);
+          if (P.has_pre) th = round_to_storage(dt, add_signed(th, xp, i, P.pre));
+          if (do_sum) th = __fadd_rn(th, acc[i]);
+          store_elem(base, dt, e0 + i, th);
+        }
       }
     }
   }
@@ -392,7 +435,10 @@ __global__ void probe_signs_kernel(RoundKeys keys, uint32_t q, uint32_t j, int64
 namespace zo {
 
 cudaError_t launch_perturb(const PerturbParams& p, int grid, cudaStream_t stream) {
-  perturb_kernel<<<grid, kThreads, 0, stream>>>(p);
+  if (p.nops == 2)
+    perturb_kernel<2><<<grid, kThreads, 0, stream>>>(p);
+  else
+    perturb_kernel<1><<<grid, kThreads, 0, stream>>>(p);
   return cudaGetLastError();
 }
 
@@ -408,7 +454,12 @@ cudaError_t launch_update(const UpdateParams& p, int grid, cudaStream_t stream) 
 }
 
 cudaError_t perturb_blocks_per_sm(int* out) {
-  return cudaOccupancyMaxActiveBlocksPerMultiprocessor(out, perturb_kernel, kThreads, 0);
+  int a = 0, b = 0;
+  cudaError_t e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&a, perturb_kernel<1>, kThreads, 0);
+  if (e != cudaSuccess) return e;
+  e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&b, perturb_kernel<2>, kThreads, 0);
+  *out = a < b ? a : b;
+  return e;
 }
 
 cudaError_t update_blocks_per_sm(int groups, int packing, int* out) {

@@ -26,8 +26,8 @@ ZO_MAX_PROBES = 1024
 DTYPE_CODE = {torch.float32: 0, torch.bfloat16: 1, torch.float16: 2}
 
 EXPORTS = ["zo_status_string", "zo_last_cuda_error", "zo_version", "zo_set_packing", "zo_get_packing",
-           "zo_perturb", "zo_precondition",
-           "zo_precondition_ex", "zo_update", "zo_update_sequential", "zo_probe_bytes", "zo_probe_signs",
+           "zo_perturb", "zo_perturb2", "zo_precondition",
+           "zo_precondition_ex", "zo_update", "zo_update_ex", "zo_update_sequential", "zo_probe_bytes", "zo_probe_signs",
            "zo_quadratic_loss_workspace_size", "zo_quadratic_loss", "zo_quadratic_loss_static"]
 ZO_QUADRATIC_LOSS_STATIC_MAX_N = 8388608
 
@@ -65,6 +65,8 @@ def _lib():
             "zo_set_packing": ([i32], c.c_int),
             "zo_get_packing": ([], c.c_int),
             "zo_perturb": ([vp, i32, u64, u32, f32, vp], c.c_int),
+            "zo_perturb2": ([vp, i32, u64, u32, f32, u32, f32, vp], c.c_int),
+            "zo_update_ex": ([vp, i32, u64, vp, i32, f64, vp, i32, u32, f32, vp], c.c_int),
             "zo_precondition": ([vp, i32, f64, vp, vp, vp], c.c_int),
             "zo_precondition_ex": ([vp, i32, f64, f64, f64, i32, vp, vp, vp, vp, vp], c.c_int),
             "zo_update": ([vp, i32, u64, vp, i32, f64, vp, vp], c.c_int),
@@ -184,6 +186,15 @@ def perturb(params, seed: int, probe: int, scale: float):
         _check("zo_perturb", _lib().zo_perturb(p._arr, p.n, seed, probe, scale, _stream(p.device)))
 
 
+def perturb2(params, seed: int, probe_a: int, scale_a: float, probe_b: int, scale_b: float):
+    """perturb(probe_a, scale_a) then perturb(probe_b, scale_b), bit for bit, in
+    one pass over theta (zo_perturb2)."""
+    p = _plist(params)
+    with torch.cuda.device(p.device):
+        _check("zo_perturb2", _lib().zo_perturb2(p._arr, p.n, seed, probe_a, scale_a, probe_b, scale_b,
+                                                 _stream(p.device)))
+
+
 def precondition(losses, eps: float, alpha: float = 0.1, lambda_reg: float = 1.0, one_sided: bool = False,
                  out=None, with_weights: bool = False):
     """losses: CUDA float64 tensor (K, 3) of rows (L+, L-, L0).
@@ -213,13 +224,16 @@ def precondition(losses, eps: float, alpha: float = 0.1, lambda_reg: float = 1.0
     return (c, status, w, curv) if with_weights else (c, status)
 
 
-def update(params, seed: int, c, lr: float, status=None):
-    """theta <- theta - (lr / K) * sum_k c_k z_k in one pass (zo_update)."""
+def update(params, seed: int, c, lr: float, status=None, pre=None):
+    """theta <- theta - (lr / K) * sum_k c_k z_k in one pass (zo_update).
+    pre=(probe, scale) first applies perturb(probe, scale) in the same pass
+    (zo_update_ex), e.g. the last probe's restore."""
     p = _plist(params)
     st = _dev_ptr(status, torch.int32, "status") if status is not None else None
+    has_pre, pre_probe, pre_scale = (0, 0, 0.0) if pre is None else (1, int(pre[0]), float(pre[1]))
     with torch.cuda.device(p.device):
-        rc = _lib().zo_update(p._arr, p.n, seed, _dev_ptr(c, torch.float64, "c"), c.numel(), lr, st,
-                              _stream(p.device))
+        rc = _lib().zo_update_ex(p._arr, p.n, seed, _dev_ptr(c, torch.float64, "c"), c.numel(), lr, st,
+                                 has_pre, pre_probe, pre_scale, _stream(p.device))
     _check("zo_update", rc)
 
 

@@ -135,3 +135,15 @@ def test_packing_switch(L):
     with zo.packing(8):
         assert zo.get_packing() == 8
     assert zo.get_packing() == 1
+
+
+def test_perturb2_and_update_ex_validation(L):
+    ok = tensors((FAKE, 16, 1))
+    c = ctypes.c_void_p(FAKE)
+    assert L.zo_perturb2(ok, 1, 1, 0, 1e-3, 1, float("nan"), None) == zo.ZO_ERR_ARG
+    assert L.zo_perturb2(ok, 1, 1, 0, float("inf"), 1, 1e-3, None) == zo.ZO_ERR_ARG
+    assert L.zo_perturb2(tensors((FAKE + 1, 16, 1)), 1, 1, 0, 1e-3, 1, 1e-3, None) == zo.ZO_ERR_ALIGN
+    assert L.zo_perturb2(None, 0, 1, 0, 1e-3, 1, 1e-3, None) == zo.ZO_OK
+    assert L.zo_update_ex(ok, 1, 1, c, 4, 1e-3, None, 1, 3, float("nan"), None) == zo.ZO_ERR_ARG
+    assert L.zo_update_ex(ok, 1, 1, c, 0, 1e-3, None, 1, 3, 1e-3, None) == zo.ZO_ERR_ARG
+    assert L.zo_update_ex(None, 0, 1, c, 4, 1e-3, None, 1, 3, 1e-3, None) == zo.ZO_OK

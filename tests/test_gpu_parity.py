@@ -337,3 +337,88 @@ def test_tiny_workload_lockstep():
         oracle.update(host, [W.DT_F32], seed, cg, lr)
         assert_update_close(storage_bits(theta), storage_bits(host[0]), W.DT_F32, c.cpu().numpy(), lr,
                             context=f"step {step}")
+
+
+# ------------------------------------------- fused passes of a step schedule
+@pytest.mark.parametrize("a,b", [(3, 4), (7, 8), (5, 5), (0, 1023)])
+def test_perturb2_is_two_perturbs(a, b, packing_mode):
+    host, dev = make_list(MIXED_NUMELS, MIXED_DTYPES, seed=a + 31 * b)
+    dts = [TORCH_TO_DT[d] for d in MIXED_DTYPES]
+    dev2 = [t.clone() for t in dev]
+    seed, sa, sb = W.step_seed(a), 1e-3, -2.5e-3
+    zo.perturb2(dev, seed, a, sa, b, sb)
+    zo.perturb(dev2, seed, a, sa)
+    zo.perturb(dev2, seed, b, sb)
+    for x, y in zip(dev, dev2):
+        assert torch.equal(x.view(torch.uint8), y.view(torch.uint8)) if x.numel() else True
+    oracle.perturb(host, dts, seed, a, sa)
+    oracle.perturb(host, dts, seed, b, sb)
+    assert_storage_equal(dev, host)
+
+
+@pytest.mark.parametrize("K", [1, 9, 64])
+def test_update_with_leading_perturb(K, packing_mode):
+    host, dev = make_list(MIXED_NUMELS, MIXED_DTYPES, seed=K + 5)
+    dts = [TORCH_TO_DT[d] for d in MIXED_DTYPES]
+    dev2 = [t.clone() for t in dev]
+    c_np = np.random.default_rng(K).normal(0, 25, K)
+    c = torch.tensor(c_np, device="cuda")
+    seed, lr, eps = W.step_seed(K), 1e-3, 1e-3
+    zo.update(dev, seed, c, lr, pre=(K - 1, eps))
+    zo.perturb(dev2, seed, K - 1, eps)
+    zo.update(dev2, seed, c, lr)
+    for x, y in zip(dev, dev2):
+        assert torch.equal(x.view(torch.uint8), y.view(torch.uint8)) if x.numel() else True
+    oracle.perturb(host, dts, seed, K - 1, eps)
+    oracle.update(host, dts, seed, c_np, lr)
+    for d, h, dt in zip(dev, host, dts):
+        assert_update_close(storage_bits(d), storage_bits(h), dt, c_np, lr)
+
+
+def test_update_with_leading_perturb_after_failed_preconditioner():
+    """A non-finite loss skips the probe sum but never the restore."""
+    host, dev = make_list(MIXED_NUMELS, MIXED_DTYPES, seed=99)
+    dev2 = [t.clone() for t in dev]
+    L = W.synthetic_losses(8, 0)
+    L[2, 0] = np.nan
+    c, st = zo.precondition(torch.tensor(L, device="cuda"), 1e-3)
+    assert int(st.item()) == zo.ZO_ERR_NONFINITE
+    zo.update(dev, 3, c, 1e-3, status=st, pre=(7, 1e-3))
+    zo.perturb(dev2, 3, 7, 1e-3)
+    for x, y in zip(dev, dev2):
+        assert torch.equal(x.view(torch.uint8), y.view(torch.uint8)) if x.numel() else True
+
+
+def test_fused_schedule_matches_algorithm1(packing_mode):
+    """A whole step with restores folded into the next probe's +eps and into
+    the update gives, bit for bit, the weights Algorithm 1's schedule gives at
+    every point a forward pass would see them, and at the end."""
+    K, eps, lr = 6, 1e-3, 1e-3
+    _, dev_a = make_list(MIXED_NUMELS, MIXED_DTYPES, seed=123)
+    dev_b = [t.clone() for t in dev_a]
+    seed = W.step_seed(42)
+    L = torch.tensor(W.synthetic_losses(K, 42), device="cuda")
+    c, st = zo.precondition(L, eps)
+
+    def snap(ts):
+        return [t.clone() for t in ts]
+
+    seen_a, seen_b = [], []
+    for k in range(K):                         # Algorithm 1
+        zo.perturb(dev_a, seed, k, eps)
+        seen_a.append(snap(dev_a))
+        zo.perturb(dev_a, seed, k, -2 * eps)
+        seen_a.append(snap(dev_a))
+        zo.perturb(dev_a, seed, k, eps)
+    zo.update(dev_a, seed, c, lr, status=st)
+    zo.perturb(dev_b, seed, 0, eps)            # fused schedule: 2K + 1 passes
+    for k in range(K):
+        seen_b.append(snap(dev_b))
+        zo.perturb(dev_b, seed, k, -2 * eps)
+        seen_b.append(snap(dev_b))
+        if k + 1 < K:
+            zo.perturb2(dev_b, seed, k, eps, k + 1, eps)
+    zo.update(dev_b, seed, c, lr, status=st, pre=(K - 1, eps))
+    for sa, sb in zip(seen_a + [dev_a], seen_b + [dev_b]):
+        for x, y in zip(sa, sb):
+            assert torch.equal(x.view(torch.uint8), y.view(torch.uint8)) if x.numel() else True
