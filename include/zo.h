@@ -34,9 +34,10 @@
  * dtype}: the trained weights, each updated in place. The same list, in the
  * same order and with the same sizes, must be given to every call of a step:
  * the probe is a function of the position of each element in that list.
- * Tensors may mix dtypes. numel may be 0. ptr must be aligned to its element
- * size; 32-byte alignment selects the vectorised path, anything else the
- * element-wise path (same results).
+ * Tensors may mix dtypes. numel may be 0 and at most 16 * (2^31 - 1) - 1
+ * (ZO_ERR_ARG beyond). ptr must be aligned to its element size; 32-byte
+ * alignment selects the vectorised path, anything else the element-wise path
+ * (same results).
  *
  * Probes. z_k is Rademacher, one bit per parameter per probe (Sec. 2, Sec. 4.3
  * "Bit-Packed perturbations"; unpack rule of Appendix F: bit 1 -> +1, bit 0 ->

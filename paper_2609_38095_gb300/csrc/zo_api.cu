@@ -131,31 +131,39 @@ int validate_params(const zo_tensor* params, int32_t n) {
     if (p.numel > 0 && p.ptr == nullptr) return ZO_ERR_ARG;
     if (reinterpret_cast<uintptr_t>(p.ptr) % static_cast<uintptr_t>(elem_size(p.dtype)) != 0) return ZO_ERR_ALIGN;
     const int64_t nb = (p.numel + 15) / 16;
-    if (nb > (INT64_C(1) << 58) - blocks) return ZO_ERR_ARG;  // virtual index space
+    if (nb >= zo::kMaxLaunchBlocks) return ZO_ERR_ARG;          // one tensor must fit one launch
+    if (nb > (INT64_C(1) << 58) - blocks) return ZO_ERR_ARG;   // virtual index space
     blocks += nb;
   }
   return ZO_OK;
 }
 
-// Fill `tab` with tensors [t0, t1) whose first virtual block is blk_begin.
-// Returns the number of blocks the launch covers.
-int64_t fill_table(TensorTable& tab, const zo_tensor* params, int32_t t0, int32_t t1, int64_t blk_begin) {
-  tab.n = t1 - t0;
-  tab.pad_ = 0;
-  tab.blk_begin = blk_begin;
-  int64_t b = blk_begin;
-  for (int32_t t = t0; t < t1; ++t) {
+// Fill `tab` with tensors t0, t0+1, ... while the launch holds fewer than
+// kMaxTensorsPerLaunch tensors and fewer than kMaxLaunchBlocks blocks; the
+// launch's first block has virtual index blk_base. Returns the first tensor
+// not taken; *nblocks receives the blocks the launch covers.
+int32_t fill_table(TensorTable& tab, const zo_tensor* params, int32_t t0, int32_t n, int64_t blk_base,
+                   int64_t* nblocks) {
+  tab.n = 0;
+  tab.blk_base = blk_base;
+  int64_t b = 0;
+  int32_t t = t0;
+  for (; t < n && tab.n < zo::kMaxTensorsPerLaunch; ++t) {
     const zo_tensor& p = params[t];
-    const int i = t - t0;
-    b += (p.numel + 15) / 16;
-    tab.blk_end[i] = b;
+    const int64_t nb = (p.numel + 15) / 16;
+    if (tab.n > 0 && b + nb >= zo::kMaxLaunchBlocks) break;
+    const int i = tab.n++;
+    b += nb;
+    tab.blk_end[i] = static_cast<uint32_t>(b);
     tab.ptr[i] = reinterpret_cast<uint64_t>(p.ptr);
     tab.numel[i] = p.numel;
     uint8_t fl = static_cast<uint8_t>(p.dtype);
     if (reinterpret_cast<uintptr_t>(p.ptr) % 32 == 0) fl |= zo::kVec32;
     tab.flags[i] = fl;
   }
-  return b - blk_begin;
+  tab.blk_total = static_cast<uint32_t>(b);
+  *nblocks = b;
+  return t;
 }
 
 int grid_for(int64_t blocks, int sms, int bps) {
@@ -168,9 +176,9 @@ int grid_for(int64_t blocks, int sms, int bps) {
 // Enqueue perturb launches over the whole parameter list.
 int run_perturb(const zo_tensor* params, int32_t n, PerturbParams& pp, DeviceInfo* d, cudaStream_t s) {
   int64_t blk = 0;
-  for (int32_t t0 = 0; t0 < n; t0 += zo::kMaxTensorsPerLaunch) {
-    const int32_t t1 = (n - t0 > zo::kMaxTensorsPerLaunch) ? t0 + zo::kMaxTensorsPerLaunch : n;
-    const int64_t nb = fill_table(pp.tab, params, t0, t1, blk);
+  for (int32_t t0 = 0; t0 < n;) {
+    int64_t nb = 0;
+    t0 = fill_table(pp.tab, params, t0, n, blk, &nb);
     if (nb > 0) {
       cudaError_t e = zo::launch_perturb(pp, grid_for(nb, d->sms, d->perturb_bps), s);
       if (e != cudaSuccess) return cuda_fail(e, "perturb_kernel");
@@ -290,9 +298,9 @@ int zo_update_ex(const zo_tensor* params, int32_t n_tensors, uint64_t seed, cons
   if ((rc = update_blocks_per_sm(d, up.groups, up.packing, &bps)) != ZO_OK) return rc;
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   int64_t blk = 0;
-  for (int32_t t0 = 0; t0 < n_tensors; t0 += zo::kMaxTensorsPerLaunch) {
-    const int32_t t1 = (n_tensors - t0 > zo::kMaxTensorsPerLaunch) ? t0 + zo::kMaxTensorsPerLaunch : n_tensors;
-    const int64_t nb = fill_table(up.tab, params, t0, t1, blk);
+  for (int32_t t0 = 0; t0 < n_tensors;) {
+    int64_t nb = 0;
+    t0 = fill_table(up.tab, params, t0, n_tensors, blk, &nb);
     if (nb > 0) {
       cudaError_t e = zo::launch_update(up, grid_for(nb, d->sms, bps * kUpdateWaves), s);
       if (e != cudaSuccess) return cuda_fail(e, "update_kernel");

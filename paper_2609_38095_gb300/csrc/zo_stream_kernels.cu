@@ -56,34 +56,34 @@ __device__ __forceinline__ void perturb_regs16(uint32_t (&v)[8], const uint4 (&x
 // leaves the current tensor.
 struct Cursor {
   int t;           // tensor index
-  int64_t tb;      // first virtual block of tensor t
-  int64_t te;      // one past its last block
-  int64_t tfe;     // one past its last full block when it takes the pipelined path, else tb
+  uint32_t tb;     // first launch block of tensor t
+  uint32_t te;     // one past its last block
+  uint32_t tfe;    // one past its last full block when it takes the pipelined path, else tb
   uint16_t* tp;    // base pointer
   uint8_t dt;      // storage dtype
 };
 
-__device__ __forceinline__ void cursor_seek(const TensorTable& tab, Cursor& c, int64_t b) {
+__device__ __forceinline__ void cursor_seek(const TensorTable& tab, Cursor& c, uint32_t b) {
   c.t = advance_tensor(tab, c.t, b);
   c.tb = tensor_blk_begin(tab, c.t);
   c.te = tab.blk_end[c.t];
   const uint8_t fl = tab.flags[c.t];
   c.dt = fl & kDtypeMask;
   // pipelined path: full, 32-byte aligned blocks of a 16-bit tensor
-  c.tfe = ((fl & kVec32) && c.dt != kF32) ? c.tb + tab.numel[c.t] / 16 : c.tb;
+  c.tfe = ((fl & kVec32) && c.dt != kF32) ? c.tb + static_cast<uint32_t>(tab.numel[c.t] / 16) : c.tb;
   c.tp = reinterpret_cast<uint16_t*>(tab.ptr[c.t]);
 }
 
-// Address of block b (inside the cursor's tensor) on the pipelined path, else nullptr.
-__device__ __forceinline__ uint16_t* fast16_block(const Cursor& c, int64_t b) {
-  return b < c.tfe ? c.tp + (b - c.tb) * 16 : nullptr;
+// Address of launch block b (inside the cursor's tensor) on the pipelined path, else nullptr.
+__device__ __forceinline__ uint16_t* fast16_block(const Cursor& c, uint32_t b) {
+  return b < c.tfe ? c.tp + static_cast<size_t>(b - c.tb) * 16 : nullptr;
 }
 
 // Any other block: fp32, a partial last block, or an unaligned tensor.
 template <int NOPS>
-__device__ __noinline__ void perturb_block_other(const TensorTable& tab, int t, int64_t b, uint4 x0, uint4 x1,
+__device__ __noinline__ void perturb_block_other(const TensorTable& tab, int t, uint32_t b, uint4 x0, uint4 x1,
                                                  PerturbOp op0, PerturbOp op1) {
-  const int64_t e0 = (b - tensor_blk_begin(tab, t)) * 16;
+  const int64_t e0 = static_cast<int64_t>(b - tensor_blk_begin(tab, t)) * 16;
   const int64_t cnt = min(static_cast<int64_t>(16), tab.numel[t] - e0);
   const uint8_t fl = tab.flags[t];
   const uint8_t dt = fl & kDtypeMask;
@@ -124,9 +124,9 @@ __global__ void __launch_bounds__(256) perturb_kernel(const __grid_constant__ Pe
   const bool same_ctr = op[1].ctr2 == op[0].ctr2;
 
   const TensorTable& tab = P.tab;
-  const int64_t blk_total = tab.blk_end[tab.n - 1];
-  const int64_t stride = static_cast<int64_t>(gridDim.x) * blockDim.x;
-  int64_t b = tab.blk_begin + static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x;
+  const uint32_t blk_total = tab.blk_total;
+  const uint32_t stride = gridDim.x * blockDim.x;
+  uint32_t b = blockIdx.x * blockDim.x + threadIdx.x;  // launch-relative; < 2^31 + stride never wraps
   if (b >= blk_total) return;
   Cursor c;
   c.t = 0;
@@ -137,7 +137,7 @@ __global__ void __launch_bounds__(256) perturb_kernel(const __grid_constant__ Pe
   uint32_t v[8];
   if (p != nullptr) ld256(p, v);
   while (true) {
-    const int64_t bn = b + stride;
+    const uint32_t bn = b + stride;
     uint16_t* pn = nullptr;
     uint32_t vn[8];
     if (bn < blk_total) {
@@ -145,10 +145,11 @@ __global__ void __launch_bounds__(256) perturb_kernel(const __grid_constant__ Pe
       pn = fast16_block(c, bn);
       if (pn != nullptr) ld256(pn, vn);
     }
+    const int64_t vb = tab.blk_base + b;  // virtual block: the Philox counter
     uint4 x[2];
-    x[0] = block_bits(b, op[0].ctr2, P.keys);
+    x[0] = block_bits(vb, op[0].ctr2, P.keys);
     x[1] = x[0];
-    if (NOPS == 2 && !same_ctr) x[1] = block_bits(b, op[1].ctr2, P.keys);
+    if (NOPS == 2 && !same_ctr) x[1] = block_bits(vb, op[1].ctr2, P.keys);
     if (p != nullptr) {
       if (dt == kBF16)
         perturb_regs16<kBF16, NOPS>(v, x, op);
@@ -346,13 +347,12 @@ __global__ void __launch_bounds__(256) update_kernel(const __grid_constant__ Upd
   __syncthreads();
 
   const TensorTable& tab = P.tab;
-  const int64_t blk_total = tab.blk_end[tab.n - 1];
-  const int64_t stride = static_cast<int64_t>(gridDim.x) * blockDim.x;
+  const uint32_t stride = gridDim.x * blockDim.x;
   int t = 0;
-  for (int64_t b = tab.blk_begin + static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; b < blk_total;
-       b += stride) {
-    t = advance_tensor(tab, t, b);
-    const int64_t e0 = (b - tensor_blk_begin(tab, t)) * 16;
+  for (uint32_t bl = blockIdx.x * blockDim.x + threadIdx.x; bl < tab.blk_total; bl += stride) {
+    t = advance_tensor(tab, t, bl);
+    const int64_t e0 = static_cast<int64_t>(bl - tensor_blk_begin(tab, t)) * 16;
+    const int64_t b = tab.blk_base + bl;  // virtual block: the Philox counter
     const int64_t cnt = min(static_cast<int64_t>(16), tab.numel[t] - e0);
     const uint8_t fl = tab.flags[t];
     const uint8_t dt = fl & kDtypeMask;
@@ -454,12 +454,17 @@ cudaError_t launch_update(const UpdateParams& p, int grid, cudaStream_t stream) 
 }
 
 cudaError_t perturb_blocks_per_sm(int* out) {
-  int a = 0, b = 0;
-  cudaError_t e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&a, perturb_kernel<1>, kThreads, 0);
-  if (e != cudaSuccess) return e;
-  e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&b, perturb_kernel<2>, kThreads, 0);
-  *out = a < b ? a : b;
-  return e;
+  int m = 1 << 30;
+  const void* kernels[2] = {reinterpret_cast<const void*>(perturb_kernel<1>),
+                            reinterpret_cast<const void*>(perturb_kernel<2>)};
+  for (const void* k : kernels) {
+    int a = 0;
+    cudaError_t e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&a, k, kThreads, 0);
+    if (e != cudaSuccess) return e;
+    m = a < m ? a : m;
+  }
+  *out = m;
+  return cudaSuccess;
 }
 
 cudaError_t update_blocks_per_sm(int groups, int packing, int* out) {

@@ -147,3 +147,11 @@ def test_perturb2_and_update_ex_validation(L):
     assert L.zo_update_ex(ok, 1, 1, c, 4, 1e-3, None, 1, 3, float("nan"), None) == zo.ZO_ERR_ARG
     assert L.zo_update_ex(ok, 1, 1, c, 0, 1e-3, None, 1, 3, 1e-3, None) == zo.ZO_ERR_ARG
     assert L.zo_update_ex(None, 0, 1, c, 4, 1e-3, None, 1, 3, 1e-3, None) == zo.ZO_OK
+
+
+def test_tensor_block_limit(L):
+    """One tensor may span fewer than 2^31 16-element blocks (a launch's
+    32-bit block offsets); larger tensors are rejected on the host."""
+    big = (1 << 31) * 16
+    assert L.zo_perturb(tensors((FAKE, big, 1)), 1, 1, 0, 1e-3, None) == zo.ZO_ERR_ARG
+    assert L.zo_perturb(tensors((FAKE, big - 16 + 1, 1)), 1, 1, 0, 1e-3, None) == zo.ZO_ERR_ARG
