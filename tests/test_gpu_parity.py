@@ -422,3 +422,26 @@ def test_fused_schedule_matches_algorithm1(packing_mode):
     for sa, sb in zip(seen_a + [dev_a], seen_b + [dev_b]):
         for x, y in zip(sa, sb):
             assert torch.equal(x.view(torch.uint8), y.view(torch.uint8)) if x.numel() else True
+
+
+def test_fused_calls_on_split_launches_and_unaligned_views(packing_mode):
+    """zo_perturb2 and zo_update_ex on 2500 tensors of odd sizes and mixed
+    dtypes (several launches) plus unaligned views (element-wise path): bit
+    for bit the unfused calls."""
+    rng = np.random.default_rng(77)
+    numels = [int(x) for x in rng.integers(0, 200, 2500)]
+    dtypes = [DTS[int(x)] for x in rng.integers(0, 3, 2500)]
+    _, dev = make_list(numels, dtypes, seed=77)
+    base = torch.randn(5000, device="cuda").to(torch.bfloat16)
+    dev += [base[1:1 + 777], base[1000 + 3:1000 + 3 + 2049]]      # 2-byte aligned views
+    dev2 = [t.clone() for t in dev]
+    seed, eps = W.step_seed(77), 1e-3
+    c = torch.tensor(rng.normal(0, 20, 11), dtype=torch.float64, device="cuda")
+    zo.perturb2(dev, seed, 7, eps, 8, -eps)
+    zo.update(dev, seed, c, 1e-3, pre=(10, eps))
+    zo.perturb(dev2, seed, 7, eps)
+    zo.perturb(dev2, seed, 8, -eps)
+    zo.perturb(dev2, seed, 10, eps)
+    zo.update(dev2, seed, c, 1e-3)
+    for x, y in zip(dev, dev2):
+        assert torch.equal(x.view(torch.uint8), y.view(torch.uint8)) if x.numel() else True
