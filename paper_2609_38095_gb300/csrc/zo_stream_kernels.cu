@@ -74,11 +74,6 @@ __device__ __forceinline__ void cursor_seek(const TensorTable& tab, Cursor& c, u
   c.tp = reinterpret_cast<uint16_t*>(tab.ptr[c.t]);
 }
 
-// Address of launch block b (inside the cursor's tensor) on the pipelined path, else nullptr.
-__device__ __forceinline__ uint16_t* fast16_block(const Cursor& c, uint32_t b) {
-  return b < c.tfe ? c.tp + static_cast<size_t>(b - c.tb) * 16 : nullptr;
-}
-
 // Any other block: fp32, a partial last block, or an unaligned tensor.
 template <int NOPS>
 __device__ __noinline__ void perturb_block_other(const TensorTable& tab, int t, uint32_t b, uint4 x0, uint4 x1,
@@ -111,10 +106,38 @@ __device__ __noinline__ void perturb_block_other(const TensorTable& tab, int t, 
   }
 }
 
-// Software-pipelined over a thread's blocks: the 256-bit load of the next
-// 16-bit block is issued before the current block is computed and stored, so
-// each thread keeps two loads in flight (the pass is HBM-bound and needs the
-// bytes in flight to cover DRAM latency).
+// A run of n blocks of one 16-bit tensor, all full and 32-byte aligned, at
+// p, p + pstride, ... with virtual blocks vb, vb + stride, ...: a tight,
+// software-pipelined loop (the next block's 256-bit load is issued before the
+// current block is computed and stored, so two loads per thread stay in
+// flight; the pass is HBM-bound and needs the bytes in flight).
+template <int NOPS, uint8_t DT>
+__device__ __forceinline__ void perturb_run16(uint16_t* p, uint32_t n, size_t pstride, int64_t vb,
+                                              uint32_t stride, const PerturbOp (&op)[2], bool same_ctr,
+                                              const RoundKeys& keys) {
+  uint32_t v[8];
+  ld256(p, v);
+  for (uint32_t i = 0; i < n; ++i) {
+    uint16_t* pn = p + pstride;
+    uint32_t vn[8];
+    if (i + 1 < n) ld256(pn, vn);
+    uint4 x[2];
+    x[0] = block_bits(vb, op[0].ctr2, keys);
+    x[1] = x[0];
+    if (NOPS == 2 && !same_ctr) x[1] = block_bits(vb, op[1].ctr2, keys);
+    perturb_regs16<DT, NOPS>(v, x, op);
+    st256(p, v);
+    p = pn;
+    vb += stride;
+#pragma unroll
+    for (int r = 0; r < 8; ++r) v[r] = vn[r];
+  }
+}
+
+// Grid-stride over the launch's blocks. While a thread's next blocks lie in
+// the full, aligned 16-bit region of its current tensor they go through
+// perturb_run16; any other block (fp32, a partial last block, an unaligned
+// tensor) is handled on its own.
 template <int NOPS>
 __global__ void __launch_bounds__(256) perturb_kernel(const __grid_constant__ PerturbParams P) {
   if (P.status != nullptr && *P.status != 0) return;
@@ -127,45 +150,32 @@ __global__ void __launch_bounds__(256) perturb_kernel(const __grid_constant__ Pe
   const uint32_t blk_total = tab.blk_total;
   const uint32_t stride = gridDim.x * blockDim.x;
   uint32_t b = blockIdx.x * blockDim.x + threadIdx.x;  // launch-relative; < 2^31 + stride never wraps
-  if (b >= blk_total) return;
   Cursor c;
   c.t = 0;
-  cursor_seek(tab, c, b);
-  int t = c.t;          // tensor and dtype of the current block
-  uint8_t dt = c.dt;
-  uint16_t* p = fast16_block(c, b);
-  uint32_t v[8];
-  if (p != nullptr) ld256(p, v);
-  while (true) {
-    const uint32_t bn = b + stride;
-    uint16_t* pn = nullptr;
-    uint32_t vn[8];
-    if (bn < blk_total) {
-      if (bn >= c.te) cursor_seek(tab, c, bn);
-      pn = fast16_block(c, bn);
-      if (pn != nullptr) ld256(pn, vn);
+  bool seeked = false;
+  while (b < blk_total) {
+    if (!seeked || b >= c.te) {
+      cursor_seek(tab, c, b);
+      seeked = true;
     }
     const int64_t vb = tab.blk_base + b;  // virtual block: the Philox counter
-    uint4 x[2];
-    x[0] = block_bits(vb, op[0].ctr2, P.keys);
-    x[1] = x[0];
-    if (NOPS == 2 && !same_ctr) x[1] = block_bits(vb, op[1].ctr2, P.keys);
-    if (p != nullptr) {
-      if (dt == kBF16)
-        perturb_regs16<kBF16, NOPS>(v, x, op);
+    if (b < c.tfe) {
+      const uint32_t n = (c.tfe - b + stride - 1) / stride;  // this thread's blocks in the region
+      uint16_t* p = c.tp + static_cast<size_t>(b - c.tb) * 16;
+      const size_t pstride = static_cast<size_t>(stride) * 16;
+      if (c.dt == kBF16)
+        perturb_run16<NOPS, kBF16>(p, n, pstride, vb, stride, op, same_ctr, P.keys);
       else
-        perturb_regs16<kF16, NOPS>(v, x, op);
-      st256(p, v);
+        perturb_run16<NOPS, kF16>(p, n, pstride, vb, stride, op, same_ctr, P.keys);
+      b += n * stride;
     } else {
-      perturb_block_other<NOPS>(tab, t, b, x[0], x[1], op[0], op[1]);
+      uint4 x[2];
+      x[0] = block_bits(vb, op[0].ctr2, P.keys);
+      x[1] = x[0];
+      if (NOPS == 2 && !same_ctr) x[1] = block_bits(vb, op[1].ctr2, P.keys);
+      perturb_block_other<NOPS>(tab, c.t, b, x[0], x[1], op[0], op[1]);
+      b += stride;
     }
-    if (bn >= blk_total) break;
-    b = bn;
-    t = c.t;
-    dt = c.dt;
-    p = pn;
-#pragma unroll
-    for (int r = 0; r < 8; ++r) v[r] = vn[r];
   }
 }
 
@@ -268,8 +278,6 @@ __device__ __forceinline__ void accumulate_any(float (&acc)[16], int64_t b, cons
     accumulate_block(acc, b, P, lut_base);
 }
 
-// One full, 32-byte aligned block: theta is loaded before the probe loop so
-// the load overlaps the arithmetic.
 // Leading perturbation of zo_update_ex, rounded to storage (16-bit pairs).
 template <uint8_t DT>
 __device__ __forceinline__ uint32_t pre_regs16(uint32_t v, const uint4& xp, int r, const PerturbOp& op) {
@@ -277,6 +285,9 @@ __device__ __forceinline__ uint32_t pre_regs16(uint32_t v, const uint4& xp, int 
   return pack2<DT>(add_signed(f.x, xp, 2 * r, op), add_signed(f.y, xp, 2 * r + 1, op));
 }
 
+// One full, 32-byte aligned block: theta (16-bit) is loaded before the probe
+// loop so the load overlaps the arithmetic; the leading perturbation, when
+// present, is applied and rounded to storage before the probe sum is added.
 template <int PACK, uint8_t DT>
 __device__ __forceinline__ void update_block_vec(void* base, int64_t e0, int64_t b, const UpdateParams& P,
                                                  uint32_t lut_base, bool do_sum) {
