@@ -22,6 +22,7 @@ import os
 import platform
 import statistics
 import subprocess
+import tempfile
 import sys
 import time
 
@@ -50,6 +51,8 @@ def parse_args():
     ap.add_argument("--cpu-seconds", type=float, default=12.0, help="target CPU time of the oracle sample")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--clocks-csv", default=None,
+                    help="keep the nvidia-smi clock samples of the timed region in this file")
     ap.add_argument("--packing", type=int, default=1, choices=[1, 8],
                     help="generated bits per (weight, probe): 1 (the paper's bit packing) or 8")
     ap.add_argument("--schedule", default="fused", choices=["fused", "alg1"],
@@ -96,14 +99,15 @@ class ClockSampler:
               "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
               "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
 
-    def __init__(self, device_id):
+    def __init__(self, device_id, path=None):
         self.proc = None
-        self.path = os.path.join(ROOT, "gpurun_out", f"clocks_{os.getpid()}.csv")
+        self.keep = path is not None
+        self.path = path or os.path.join(tempfile.gettempdir(), f"zo_bench_clocks_{os.getpid()}.csv")
         self.device_id = device_id
 
     def start(self):
         try:
-            os.makedirs(os.path.dirname(self.path), exist_ok=True)
+            os.makedirs(os.path.dirname(os.path.abspath(self.path)), exist_ok=True)
             self.fh = open(self.path, "w")
             cmd = ["nvidia-smi", f"--query-gpu={self.FIELDS}", "--format=csv,noheader,nounits", "-lms", "200"]
             if self.device_id:
@@ -135,6 +139,11 @@ class ClockSampler:
             for n, v in zip(names, f[5:9]):
                 if v.lower().startswith("active"):
                     reasons.add(n)
+        if not self.keep:
+            try:
+                os.remove(self.path)
+            except OSError:
+                pass
         if not sm:
             return None
         return {"sm_mhz": statistics.median(sm), "sm_max_mhz": max(mx), "reasons": sorted(reasons),
@@ -314,7 +323,7 @@ def run_zo(args):
         dev_uuid = "GPU-" + str(torch.cuda.get_device_properties(dev).uuid)
     except Exception:
         pass
-    clocks = ClockSampler(dev_uuid)
+    clocks = ClockSampler(dev_uuid, args.clocks_csv)
     clocks.start()
     barrier()
     t_start = torch.cuda.Event(enable_timing=True)
