@@ -151,13 +151,27 @@ int zo_perturb2(const zo_tensor* params, int32_t n_tensors, uint64_t seed, uint3
  * ------------------------------------------------------------------------- */
 int zo_precondition(const double* losses, int32_t K, double eps, double* c, int32_t* status, void* stream);
 
+/* Bits of zo_precondition_ex's `flags` (0 = the paper's preconditioner). */
+#define ZO_PRECOND_ONE_SIDED 1          /* c_k = w_k (L+ - L0) / eps, a non-paper forward difference */
+#define ZO_PRECOND_RELATIVE_CURVATURE 2 /* Eq. 4 on curv_k / m, m = (1/K) sum_j |curv_j| */
+
 /* zo_precondition with every knob of Sec. 4.1 exposed: alpha in [0, 1]
  * (alpha = 0 recovers 1SPSA, alpha = 1 is a diagonal Newton step in probe
- * space), lambda_reg > 0, and one_sided != 0 for the non-paper forward
- * difference c_k = w_k (L+ - L0) / eps. w and curv (device, K fp64) are
- * optional outputs (NULL to skip), written under the same rule as c. */
+ * space), lambda_reg > 0, and `flags`, a bitwise OR of:
+ *   ZO_PRECOND_ONE_SIDED           the forward difference above instead of
+ *                                  the paper's central one;
+ *   ZO_PRECOND_RELATIVE_CURVATURE  Eq. 4 applied to the relative curvature
+ *       r_k = curv_k / m with m = (1/K) sum_j |curv_j| over this call's K
+ *       probes (r_k = 0 for all k when m = 0; a non-finite m is
+ *       ZO_ERR_NONFINITE). Sec. 6 names per-step curvature normalisation as
+ *       future work without a formula; this is one reading of it: the weight
+ *       then depends only on how a probe's curvature compares with the
+ *       step's average, not on the loss scale.
+ * Any other bit is ZO_ERR_ARG. w and curv (device, K fp64) are optional
+ * outputs (NULL to skip), written under the same rule as c; curv is always
+ * Eq. 3's curvature. */
 int zo_precondition_ex(const double* losses, int32_t K, double eps, double alpha, double lambda_reg,
-                       int32_t one_sided, double* c, double* w, double* curv, int32_t* status, void* stream);
+                       int32_t flags, double* c, double* w, double* curv, int32_t* status, void* stream);
 
 /* ---------------------------------------------------------------------------
  * zo_update -- the fused K-probe update of Sec. 4.2 (Eq. 5 and its compact form

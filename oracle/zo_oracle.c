@@ -341,27 +341,56 @@ int oracle_perturb_elements(int32_t dtype, int64_t n, const uint64_t* g, const f
 /*                c_k = w * (L+ - L0) / eps       one-sided variant            */
 /* losses is K rows of {L+, L-, L0}. Non-finite inputs or results return      */
 /* ORC_ERR_NONFINITE and leave the outputs untouched.                         */
+/*                                                                           */
+/* flags: ORC_PRECOND_ONE_SIDED selects the one-sided coefficient;            */
+/* ORC_PRECOND_RELATIVE applies Eq. 4 to the relative curvature               */
+/*   r_k = c_hat_k / m,   m = (1/K) sum_j |c_hat_j|  (j in probe order),      */
+/* one reading of the per-step curvature normalisation that Sec. 6 leaves to  */
+/* future work; m = 0 (every curvature zero) gives r_k = 0, a non-finite m is */
+/* ORC_ERR_NONFINITE. curv_out always receives Eq. 3's c_hat.                 */
 /* ------------------------------------------------------------------------- */
+#define ORC_PRECOND_ONE_SIDED 1
+#define ORC_PRECOND_RELATIVE 2
+
+static double curvature(const double* l, double eps) { return (l[0] - 2.0 * l[2] + l[1]) / (eps * eps); }
+
+static double difference(const double* l, double eps, int one_sided) {
+  return one_sided ? (l[0] - l[2]) / eps : (l[0] - l[1]) / (2.0 * eps);
+}
+
 int oracle_precondition(const double* losses, int32_t K, double eps, double alpha, double lambda_reg,
-                        int32_t one_sided, double* c, double* w_out, double* curv_out) {
+                        int32_t flags, double* c, double* w_out, double* curv_out) {
   if (K < 1 || !(eps > 0.0) || !isfinite(eps) || !(alpha >= 0.0) || !(alpha <= 1.0) ||
-      !(lambda_reg > 0.0) || !isfinite(lambda_reg))
+      !(lambda_reg > 0.0) || !isfinite(lambda_reg) || (flags & ~(ORC_PRECOND_ONE_SIDED | ORC_PRECOND_RELATIVE)) != 0)
     return ORC_ERR_ARG;
-  /* first pass: everything must be finite before anything is written */
+  const int one_sided = (flags & ORC_PRECOND_ONE_SIDED) != 0;
+  const int relative = (flags & ORC_PRECOND_RELATIVE) != 0;
+  /* first pass: every loss and curvature finite, and the normaliser m */
+  double m = 1.0;
+  if (relative) m = 0.0;
   for (int32_t k = 0; k < K; ++k) {
-    double lp = losses[3 * k + 0], lm = losses[3 * k + 1], l0 = losses[3 * k + 2];
-    if (!isfinite(lp) || !isfinite(lm) || !isfinite(l0)) return ORC_ERR_NONFINITE;
-    double curv = (lp - 2.0 * l0 + lm) / (eps * eps);
-    double w = 1.0 / fmax(lambda_reg, pow(fabs(curv), alpha));
-    double g = one_sided ? (lp - l0) / eps : (lp - lm) / (2.0 * eps);
-    if (!isfinite(curv) || !isfinite(w * g)) return ORC_ERR_NONFINITE;
+    const double* l = losses + 3 * k;
+    if (!isfinite(l[0]) || !isfinite(l[1]) || !isfinite(l[2])) return ORC_ERR_NONFINITE;
+    double curv = curvature(l, eps);
+    if (!isfinite(curv)) return ORC_ERR_NONFINITE;
+    if (relative) m += fabs(curv);
+  }
+  if (relative) {
+    m = m / (double)K;
+    if (!isfinite(m)) return ORC_ERR_NONFINITE;
+  }
+  /* second pass: weights and coefficients, all checked before any write */
+  for (int32_t k = 0; k < K; ++k) {
+    double curv = curvature(losses + 3 * k, eps);
+    double r = relative ? (m > 0.0 ? curv / m : 0.0) : curv;
+    double w = 1.0 / fmax(lambda_reg, pow(fabs(r), alpha));
+    if (!isfinite(w * difference(losses + 3 * k, eps, one_sided))) return ORC_ERR_NONFINITE;
   }
   for (int32_t k = 0; k < K; ++k) {
-    double lp = losses[3 * k + 0], lm = losses[3 * k + 1], l0 = losses[3 * k + 2];
-    double curv = (lp - 2.0 * l0 + lm) / (eps * eps);
-    double w = 1.0 / fmax(lambda_reg, pow(fabs(curv), alpha));
-    double g = one_sided ? (lp - l0) / eps : (lp - lm) / (2.0 * eps);
-    c[k] = w * g;
+    double curv = curvature(losses + 3 * k, eps);
+    double r = relative ? (m > 0.0 ? curv / m : 0.0) : curv;
+    double w = 1.0 / fmax(lambda_reg, pow(fabs(r), alpha));
+    c[k] = w * difference(losses + 3 * k, eps, one_sided);
     if (w_out) w_out[k] = w;
     if (curv_out) curv_out[k] = curv;
   }

@@ -211,7 +211,7 @@ const char* zo_status_string(int status) {
 
 const char* zo_last_cuda_error(void) { return g_last_cuda_error; }
 
-int zo_version(void) { return 10100; }
+int zo_version(void) { return 10200; }
 
 int zo_set_packing(int32_t bits_per_value) {
   if (bits_per_value != zo::kPacking1 && bits_per_value != zo::kPacking8) return ZO_ERR_ARG;
@@ -344,10 +344,13 @@ static int check_precondition_args(const double* losses, int32_t K, double eps, 
 }
 
 int zo_precondition_ex(const double* losses, int32_t K, double eps, double alpha, double lambda_reg,
-                       int32_t one_sided, double* c, double* w, double* curv, int32_t* status, void* stream) {
+                       int32_t flags, double* c, double* w, double* curv, int32_t* status, void* stream) {
   int rc = check_precondition_args(losses, K, eps, alpha, lambda_reg, c, status);
   if (rc != ZO_OK) return rc;
-  cudaError_t e = zo::launch_precondition(losses, K, eps, alpha, lambda_reg, one_sided != 0, c, w, curv, status,
+  if ((flags & ~(ZO_PRECOND_ONE_SIDED | ZO_PRECOND_RELATIVE_CURVATURE)) != 0) return ZO_ERR_ARG;
+  static_assert(ZO_PRECOND_ONE_SIDED == zo::kPrecondOneSided && ZO_PRECOND_RELATIVE_CURVATURE == zo::kPrecondRelative,
+                "flag values");
+  cudaError_t e = zo::launch_precondition(losses, K, eps, alpha, lambda_reg, flags, c, w, curv, status,
                                           static_cast<cudaStream_t>(stream));
   return e == cudaSuccess ? ZO_OK : cuda_fail(e, "precondition_kernel");
 }

@@ -9,6 +9,8 @@
 namespace zo {
 
 constexpr int kStatusNonFinite = -4;  // ZO_ERR_NONFINITE
+constexpr int kPrecondOneSided = 1;   // ZO_PRECOND_ONE_SIDED
+constexpr int kPrecondRelative = 2;   // ZO_PRECOND_RELATIVE_CURVATURE
 constexpr int kThreads = 256;         // threads per block of the streaming kernels
 constexpr int kMaxLossPartials = 2048;
 constexpr int kStaticLossPartials = 4096;   // fixed scratch of the allocation-free loss (32 KB)
@@ -24,7 +26,7 @@ cudaError_t launch_probe_bytes(const RoundKeys& keys, uint32_t ctr2, uint32_t bi
 cudaError_t launch_probe_signs(const RoundKeys& keys, uint32_t ctr2, uint32_t bit, int64_t first, int64_t n,
                                int8_t* out, int grid, cudaStream_t stream);
 cudaError_t launch_precondition(const double* losses, int K, double eps, double alpha, double lambda_reg,
-                                int one_sided, double* c, double* w, double* curv, int32_t* status,
+                                int flags, double* c, double* w, double* curv, int32_t* status,
                                 cudaStream_t stream);
 cudaError_t launch_quadratic_loss(const float* theta, const float* a, int64_t n, double* out, double* partial,
                                   int max_partials, int num_sms, cudaStream_t stream);

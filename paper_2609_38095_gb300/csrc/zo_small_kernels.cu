@@ -14,23 +14,54 @@ namespace zo {
 //   curv_k = (L+ - 2 L0 + L-) / eps^2                        (Eq. 3)
 //   w_k    = 1 / max(lambda_reg, |curv_k|^alpha)             (Eq. 4)
 //   c_k    = w_k (L+ - L-) / (2 eps)   or   w_k (L+ - L0) / eps
+// With kPrecondRelative, Eq. 4 takes the relative curvature curv_k / m,
+// m = (1/K) sum_j |curv_j| (a fixed-order block sum; m = 0 gives ratio 0):
+// one reading of the per-step curvature normalisation of Sec. 6.
 // Every value is checked before any is written: one non-finite loss,
-// curvature or coefficient makes the block write ZO_ERR_NONFINITE and nothing
-// else. One block of up to kMaxProbes threads.
+// curvature, normaliser or coefficient makes the block write
+// ZO_ERR_NONFINITE and nothing else. One block of up to kMaxProbes threads.
 // ---------------------------------------------------------------------------
 __global__ void precondition_kernel(const double* __restrict__ losses, int K, double eps, double alpha,
-                                    double lambda_reg, int one_sided, double* __restrict__ c, double* __restrict__ w,
+                                    double lambda_reg, int flags, double* __restrict__ c, double* __restrict__ w,
                                     double* __restrict__ curv, int32_t* __restrict__ status) {
+  __shared__ double warp_sums[kMaxProbes / 32];
+  __shared__ double s_norm;
   const int k = threadIdx.x;
-  double cv = 0.0, wk = 0.0, ck = 0.0;
+  const bool one_sided = (flags & kPrecondOneSided) != 0;
+  const bool relative = (flags & kPrecondRelative) != 0;
+  double lp = 0.0, lm = 0.0, l0 = 0.0, cv = 0.0;
   bool bad = false;
   if (k < K) {
-    const double lp = losses[3 * k + 0], lm = losses[3 * k + 1], l0 = losses[3 * k + 2];
+    lp = losses[3 * k + 0];
+    lm = losses[3 * k + 1];
+    l0 = losses[3 * k + 2];
     cv = __ddiv_rn(__dadd_rn(__dsub_rn(lp, __dmul_rn(2.0, l0)), lm), __dmul_rn(eps, eps));
-    wk = __ddiv_rn(1.0, fmax(lambda_reg, pow(fabs(cv), alpha)));
+    bad = !isfinite(lp) || !isfinite(lm) || !isfinite(l0) || !isfinite(cv);
+  }
+  double r = cv;
+  if (relative) {
+    // m: |curv| summed by a fixed shuffle tree per warp, warps in index order
+    double v = (k < K && !bad) ? fabs(cv) : 0.0;
+#pragma unroll
+    for (int off = 16; off > 0; off >>= 1) v = __dadd_rn(v, __shfl_down_sync(0xFFFFFFFFu, v, off));
+    if ((k & 31) == 0) warp_sums[k >> 5] = v;
+    __syncthreads();
+    if (k == 0) {
+      double sum = 0.0;
+      for (int i = 0; i < static_cast<int>(blockDim.x >> 5); ++i) sum = __dadd_rn(sum, warp_sums[i]);
+      s_norm = __ddiv_rn(sum, static_cast<double>(K));
+    }
+    __syncthreads();
+    const double m = s_norm;
+    bad = bad || !isfinite(m);
+    r = m > 0.0 ? __ddiv_rn(cv, m) : 0.0;
+  }
+  double wk = 0.0, ck = 0.0;
+  if (k < K) {
+    wk = __ddiv_rn(1.0, fmax(lambda_reg, pow(fabs(r), alpha)));
     const double g = one_sided ? __ddiv_rn(__dsub_rn(lp, l0), eps) : __ddiv_rn(__dsub_rn(lp, lm), __dmul_rn(2.0, eps));
     ck = __dmul_rn(wk, g);
-    bad = !isfinite(lp) || !isfinite(lm) || !isfinite(l0) || !isfinite(cv) || !isfinite(ck);
+    bad = bad || !isfinite(ck);
   }
   bad = __syncthreads_or(bad);
   if (k == 0) *status = bad ? static_cast<int32_t>(kStatusNonFinite) : 0;
@@ -84,10 +115,10 @@ __global__ void __launch_bounds__(256) quad_loss_final_kernel(const double* __re
 }
 
 cudaError_t launch_precondition(const double* losses, int K, double eps, double alpha, double lambda_reg,
-                                int one_sided, double* c, double* w, double* curv, int32_t* status,
+                                int flags, double* c, double* w, double* curv, int32_t* status,
                                 cudaStream_t stream) {
   const int threads = ((K + 31) / 32) * 32;
-  precondition_kernel<<<1, threads, 0, stream>>>(losses, K, eps, alpha, lambda_reg, one_sided, c, w, curv, status);
+  precondition_kernel<<<1, threads, 0, stream>>>(losses, K, eps, alpha, lambda_reg, flags, c, w, curv, status);
   return cudaGetLastError();
 }
 

@@ -22,6 +22,8 @@ ZO_ERR_CUDA = -5
 ZO_ERR_TOO_MANY_PROBES = -6
 ZO_ERR_WORKSPACE = -7
 ZO_MAX_PROBES = 1024
+ZO_PRECOND_ONE_SIDED = 1
+ZO_PRECOND_RELATIVE_CURVATURE = 2
 
 DTYPE_CODE = {torch.float32: 0, torch.bfloat16: 1, torch.float16: 2}
 
@@ -196,10 +198,14 @@ def perturb2(params, seed: int, probe_a: int, scale_a: float, probe_b: int, scal
 
 
 def precondition(losses, eps: float, alpha: float = 0.1, lambda_reg: float = 1.0, one_sided: bool = False,
-                 out=None, with_weights: bool = False):
+                 out=None, with_weights: bool = False, relative: bool = False, flags=None):
     """losses: CUDA float64 tensor (K, 3) of rows (L+, L-, L0).
+    one_sided / relative set ZO_PRECOND_ONE_SIDED / ZO_PRECOND_RELATIVE_CURVATURE
+    (`flags`, the raw bit word, overrides both when given).
     Returns (c, status) -- or (c, status, w, curv) with with_weights -- as CUDA
     tensors; status[0] is ZO_OK or ZO_ERR_NONFINITE once the kernel has run."""
+    if flags is None:
+        flags = (ZO_PRECOND_ONE_SIDED if one_sided else 0) | (ZO_PRECOND_RELATIVE_CURVATURE if relative else 0)
     if losses.dim() != 2 or losses.shape[1] != 3:
         raise ValueError("losses must have shape (K, 3)")
     lp = _dev_ptr(losses, torch.float64, "losses")
@@ -215,7 +221,7 @@ def precondition(losses, eps: float, alpha: float = 0.1, lambda_reg: float = 1.0
         w = torch.empty(K, dtype=torch.float64, device=dev)
         curv = torch.empty(K, dtype=torch.float64, device=dev)
     with torch.cuda.device(dev):
-        rc = _lib().zo_precondition_ex(lp, K, eps, alpha, lambda_reg, int(one_sided),
+        rc = _lib().zo_precondition_ex(lp, K, eps, alpha, lambda_reg, int(flags),
                                        _dev_ptr(c, torch.float64, "c"),
                                        _dev_ptr(w, torch.float64) if w is not None else None,
                                        _dev_ptr(curv, torch.float64) if curv is not None else None,

@@ -34,7 +34,7 @@ def test_exports_every_declared_symbol(L):
 
 
 def test_version_and_strings(L):
-    assert zo.version() == 10100
+    assert zo.version() == 10200
     for s in (0, -1, -2, -3, -4, -5, -6, -7):
         assert zo.status_string(s).startswith("ZO_")
     assert "unknown" in zo.status_string(99)
@@ -94,6 +94,8 @@ def test_precondition_validation(L):
     assert f(p, 4, 1e-3, 0.1, 1.0, 0, None, None, None, p, None) == zo.ZO_ERR_ARG
     assert f(p, 4, 1e-3, 0.1, 1.0, 0, p, None, None, None, None) == zo.ZO_ERR_ARG
     assert L.zo_precondition(p, 0, 1e-3, p, p, None) == zo.ZO_ERR_ARG
+    for bad_flags in (4, 8, -1, 1 << 30):
+        assert f(p, 4, 1e-3, 0.1, 1.0, bad_flags, p, None, None, p, None) == zo.ZO_ERR_ARG
 
 
 def test_probe_view_and_loss_validation(L):

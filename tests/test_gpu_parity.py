@@ -226,21 +226,44 @@ def crafted_losses():
 
 
 @pytest.mark.parametrize("K", [1, 7, 16, 256, 1024])
-@pytest.mark.parametrize("alpha,lam,one_sided", [(0.1, 1.0, False), (0.0, 1.0, False), (1.0, 1.0, False),
-                                                 (0.5, 3.0, False), (0.1, 1.0, True)])
-def test_precondition_vs_oracle(K, alpha, lam, one_sided):
+@pytest.mark.parametrize("alpha,lam,one_sided,relative", [(0.1, 1.0, False, False), (0.0, 1.0, False, False),
+                                                          (1.0, 1.0, False, False), (0.5, 3.0, False, False),
+                                                          (0.1, 1.0, True, False), (0.1, 1.0, False, True),
+                                                          (1.0, 1e-3, True, True)])
+def test_precondition_vs_oracle(K, alpha, lam, one_sided, relative):
     L = W.synthetic_losses(K, step=K)
     cr = crafted_losses()
     L[: min(K, len(cr))] = cr[: min(K, len(cr))]
     eps = 1e-3
     Ld = torch.tensor(L, device="cuda")
-    c, st, w, cv = zo.precondition(Ld, eps, alpha=alpha, lambda_reg=lam, one_sided=one_sided, with_weights=True)
-    rc, c_o, w_o, cv_o = oracle.precondition(L, eps, alpha=alpha, lambda_reg=lam, one_sided=one_sided)
+    c, st, w, cv = zo.precondition(Ld, eps, alpha=alpha, lambda_reg=lam, one_sided=one_sided, relative=relative,
+                                   with_weights=True)
+    rc, c_o, w_o, cv_o = oracle.precondition(L, eps, alpha=alpha, lambda_reg=lam, one_sided=one_sided,
+                                             relative=relative)
     assert rc == oracle.OK and int(st.item()) == zo.ZO_OK
     for got, want in ((c, c_o), (w, w_o), (cv, cv_o)):
         g = got.cpu().numpy()
         np.testing.assert_allclose(g, want, rtol=1e-6, atol=0)
         np.testing.assert_allclose(g, want, rtol=1e-13, atol=1e-300)
+
+
+def test_precondition_relative_degenerate():
+    """All-zero curvature (m = 0 -> w = 1/lambda_reg) and an overflowing mean."""
+    eps = 1e-3
+    L = np.array([[2.0, 2.0, 2.0], [2.5, 1.5, 2.0], [3.0, 1.0, 2.0]])
+    c, st, w, _ = zo.precondition(torch.tensor(L, device="cuda"), eps, lambda_reg=0.5, relative=True,
+                                  with_weights=True)
+    rc, c_o, w_o, _ = oracle.precondition(L, eps, lambda_reg=0.5, relative=True)
+    assert rc == oracle.OK and int(st.item()) == zo.ZO_OK
+    np.testing.assert_array_equal(w.cpu().numpy(), w_o)
+    np.testing.assert_allclose(c.cpu().numpy(), c_o, rtol=1e-15)
+    big = 1.5e308 * 1e-6 / 2
+    Lb = np.array([[big, big, 0.0], [big, big, 0.0]])
+    sentinel = torch.full((2,), 7.0, dtype=torch.float64, device="cuda")
+    status = torch.zeros(1, dtype=torch.int32, device="cuda")
+    zo.precondition(torch.tensor(Lb, device="cuda"), eps, relative=True, out=(sentinel, status))
+    assert int(status.item()) == zo.ZO_ERR_NONFINITE == oracle.precondition(Lb, eps, relative=True)[0]
+    assert torch.all(sentinel == 7.0)
 
 
 @pytest.mark.parametrize("bad", [np.nan, np.inf])

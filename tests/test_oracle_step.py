@@ -183,6 +183,84 @@ def test_precondition_bad_args():
     assert oracle.precondition([[1, 1, 1]], 0.0)[0] == oracle.ERR_ARG
     assert oracle.precondition([[1, 1, 1]], 1e-3, alpha=1.5)[0] == oracle.ERR_ARG
     assert oracle.precondition([[1, 1, 1]], 1e-3, lambda_reg=0.0)[0] == oracle.ERR_ARG
+    for bad_flags in (4, 8, -1):
+        assert oracle.precondition([[1, 1, 1]], 1e-3, flags=bad_flags)[0] == oracle.ERR_ARG
+
+
+# ------------------------------------------- relative curvature (Sec. 6 reading)
+def triples_with_curvature(g, curv, eps):
+    """(L+, L-, L0) rows with first difference g and curvature curv:
+    L0 = 0, L+- = +-g eps + curv eps^2 / 2."""
+    g, curv = np.asarray(g, float), np.asarray(curv, float)
+    return np.column_stack([g * eps + curv * eps * eps / 2, -g * eps + curv * eps * eps / 2, np.zeros_like(g)])
+
+
+def test_relative_curvature_alpha1_closed_form():
+    """alpha = 1 and a negligible floor: w_k = m / |curv_k|, so sum_k 1/w_k = K
+    and w_k |curv_k| is the same for every probe (= m, the mean |curvature|)."""
+    eps = 1e-2
+    curv = np.array([1.0, 1.0, 1.0, 5.0, -3.0, 0.5, 20.0, -7.5])
+    g = np.linspace(-1, 1, len(curv))
+    rc, c, w, cv = oracle.precondition(triples_with_curvature(g, curv, eps), eps, alpha=1.0, lambda_reg=1e-12,
+                                       relative=True)
+    assert rc == oracle.OK
+    m = np.mean(np.abs(curv))
+    np.testing.assert_allclose(cv, curv, rtol=1e-9)             # curv is still Eq. 3's curvature
+    np.testing.assert_allclose(w * np.abs(cv), m, rtol=1e-9)
+    assert np.sum(1.0 / w) == pytest.approx(len(curv), rel=1e-12)
+    np.testing.assert_allclose(c, w * g, rtol=1e-9)              # central difference unchanged
+
+
+def test_relative_curvature_equal_magnitudes():
+    """Equal |curvature| in every probe: every ratio is +-1, so w = 1/max(lambda, 1)
+    whatever alpha and the common magnitude (a plain sum instead of the mean would
+    give ratios 1/K and w = K^alpha here)."""
+    eps = 1e-3
+    for mag in (1e-3, 1.0, 3e4):
+        curv = mag * np.array([1, -1, 1, 1, -1, -1, 1, 1, 1, -1, 1, 1])
+        for alpha in (0.1, 0.5, 1.0):
+            rc, c, w, _ = oracle.precondition(triples_with_curvature(np.ones(12), curv, eps), eps, alpha=alpha,
+                                              lambda_reg=1e-3, relative=True)
+            assert rc == oracle.OK
+            np.testing.assert_allclose(w, 1.0, rtol=1e-12)
+
+
+def test_relative_curvature_scale_invariance():
+    """Scaling every curvature by s leaves the relative weights unchanged, while
+    the paper's absolute weights move by s^-alpha where the floor is inactive."""
+    rng = np.random.default_rng(9)
+    eps = 1e-3
+    curv = rng.uniform(-2e4, 2e4, 64)
+    g = rng.uniform(-50, 50, 64)
+    _, _, w1, _ = oracle.precondition(triples_with_curvature(g, curv, eps), eps, relative=True)
+    for s in (1e-3, 10.0, 1e3):
+        _, _, ws, _ = oracle.precondition(triples_with_curvature(g, s * curv, eps), eps, relative=True)
+        np.testing.assert_allclose(ws, w1, rtol=1e-6)
+    _, _, a1, _ = oracle.precondition(triples_with_curvature(g, curv, eps), eps)
+    _, _, a2, _ = oracle.precondition(triples_with_curvature(g, 1e3 * curv, eps), eps)
+    big = np.abs(curv) > 10
+    np.testing.assert_allclose(a2[big], a1[big] * 1e3 ** -0.1, rtol=1e-6)
+
+
+def test_relative_curvature_degenerate_cases():
+    eps = 1e-3
+    # K = 1: the ratio is +-1
+    rc, _, w, _ = oracle.precondition(triples_with_curvature([2.0], [-123.0], eps), eps, alpha=0.7,
+                                      lambda_reg=1e-3, relative=True)
+    assert rc == oracle.OK and w[0] == pytest.approx(1.0, rel=1e-12)
+    # every curvature zero: m = 0, ratios 0, w = 1 / lambda_reg
+    rc, c, w, _ = oracle.precondition([[2.0, 2.0, 2.0], [2.5, 1.5, 2.0]], eps, lambda_reg=0.5, relative=True)
+    assert rc == oracle.OK
+    np.testing.assert_array_equal(w, 2.0)
+    assert c[1] == pytest.approx(2.0 * 1.0 / (2 * eps), rel=1e-12)
+    # combined with the one-sided difference
+    rc, c, w, _ = oracle.precondition([[3.04, 2.98, 3.0]], 0.01, alpha=1.0, lambda_reg=1e-9, relative=True,
+                                      one_sided=True)
+    assert w[0] == pytest.approx(1.0, rel=1e-12) and c[0] == pytest.approx(4.0, rel=1e-9)
+    # a sum of |curvature| overflowing to infinity is non-finite
+    big = 1.5e308 * 1e-6 / 2
+    rc, c, _, _ = oracle.precondition([[big, big, 0.0], [big, big, 0.0]], 1e-3, relative=True)
+    assert rc == oracle.ERR_NONFINITE and np.all(np.isnan(c))
 
 
 def quad_setup(d=4096, seed=11):
