@@ -50,6 +50,8 @@ def parse_args():
     ap.add_argument("--K", type=int, default=None, help="override the probes per step of --config")
     ap.add_argument("--cpu-seconds", type=float, default=12.0, help="target CPU time of the oracle sample")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--cpu-workers", type=int, default=None,
+                    help="oracle worker processes for the CPU baseline (default: one per host core)")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--clocks-csv", default=None,
                     help="keep the nvidia-smi clock samples of the timed region in this file")
@@ -179,48 +181,79 @@ def whole_job_rate(world, d, K, seconds):
 
 
 # ------------------------------------------------------------- oracle arm
-def oracle_step(ps, M, step, host_theta):
-    """One step of the workload restricted to its first M weights (a prefix of
-    the first tensor), computed by the CPU oracle."""
+def _widen(bits, dtype):
+    """Storage bits -> float32 values (exact)."""
+    if dtype == W.DT_F32:
+        return bits
+    if dtype == W.DT_F16:
+        return bits.view(np.float16).astype(np.float32)
+    return (bits.astype(np.uint32) << 16).view(np.float32)
+
+
+def _narrow(out_bits, dtype):
+    return out_bits.view(np.float32) if dtype == W.DT_F32 else out_bits.astype(np.uint16)
+
+
+def oracle_block_step(task):
+    """One step of the workload on the weights with virtual indices
+    [first, first + n) of the first tensor, computed by the CPU oracle's
+    element-list routines: K x (+eps, -2 eps, +eps), the preconditioner on the
+    step's loss triples and the fused update. Returns the seconds it took
+    (input generation excluded). Runs in a worker process."""
+    dtype, first, n, K, eps, step, packing = task
     import oracle
-    K, eps = ps.K, ps.eps
+    oracle.set_packing(packing)
+    bits = W.random_storage(np.random.default_rng([1, first]), n, dtype)
+    g = np.arange(first, first + n, dtype=np.uint64)
     seed = W.step_seed(step)
+    t0 = time.perf_counter()
     for k in range(K):
         for s in (eps, -2 * eps, eps):
-            oracle.perturb(host_theta, [ps.dtype], seed, k, s)
+            bits = _narrow(oracle.perturb_elements(dtype, g, _widen(bits, dtype), seed, k, s), dtype)
     rc, c, _, _ = oracle.precondition(W.synthetic_losses(K, step), eps)
     assert rc == 0
-    oracle.update(host_theta, [ps.dtype], seed, c, eps)
+    bits = _narrow(oracle.update_elements(dtype, g, _widen(bits, dtype), seed, c, eps), dtype)
+    return time.perf_counter() - t0
 
 
-def oracle_sample_size(ps, target_s):
-    rng = np.random.default_rng(0)
-    M0 = 2048
-    th = [W.random_storage(rng, M0, ps.dtype)]
-    t0 = time.perf_counter()
-    oracle_step(ps, M0, 0, th)
-    dt = time.perf_counter() - t0
-    M = int(M0 * target_s / max(dt, 1e-6))
-    return max(16, min(M, ps.numels[0]) // 16 * 16)
+def host_cores():
+    try:
+        return len(os.sched_getaffinity(0))
+    except AttributeError:
+        return os.cpu_count() or 1
 
 
-def time_oracle(ps, target_s, steps=1, warmup=0, packing=1):
+def time_oracle(ps, target_s, steps=1, warmup=0, packing=1, workers=None):
+    """The oracle on a bounded sample of the workload, one process per host
+    core (spawned, so no CUDA state is inherited), each on its own range of
+    the first tensor's weights. Returns (value, seconds per step, weights,
+    cores, sample description)."""
+    import multiprocessing
+
     import oracle
-    oracle.lib()
-    oracle.set_packing(packing)
-    M = oracle_sample_size(ps, target_s)
-    rng = np.random.default_rng(1)
-    th = [W.random_storage(rng, M, ps.dtype)]
-    for s in range(warmup):
-        oracle_step(ps, M, s, th)
-    t0 = time.perf_counter()
-    for s in range(steps):
-        oracle_step(ps, M, warmup + s, th)
-    dt = (time.perf_counter() - t0) / steps
+    oracle.lib()                                    # build once before the workers load it
+    P = max(1, workers or host_cores())
+    t_cal = oracle_block_step((ps.dtype, 0, 2048, ps.K, ps.eps, 0, packing))
+    per = int(2048 * target_s / max(t_cal, 1e-6)) // 16 * 16
+    per = max(16, min(per, ps.numels[0] // P // 16 * 16))
+    M = per * P
+    ctx = multiprocessing.get_context("spawn")
+    with ctx.Pool(P) as pool:
+        pool.map(oracle_block_step, [(ps.dtype, j * per, 16, 8, ps.eps, 0, packing) for j in range(P)])
+        walls = []
+        for s in range(warmup + steps):
+            tasks = [(ps.dtype, j * per, per, ps.K, ps.eps, s, packing) for j in range(P)]
+            t0 = time.perf_counter()
+            pool.map(oracle_block_step, tasks, chunksize=1)
+            if s >= warmup:
+                walls.append(time.perf_counter() - t0)
+    dt = sum(walls) / len(walls)
     value = M * ps.K / dt / 1e9
-    sample = (f"first {M} weights of the first tensor ({ps.shapes[0][0]}) of the {ps.name} set, K={ps.K}: "
-              f"{3 * ps.K} perturb passes + preconditioner + fused update per step, single-threaded oracle")
-    return value, dt, M, sample
+    sample = (f"first {M} weights of the first tensor ({ps.shapes[0][0]}) of the {ps.name} set, K={ps.K}, "
+              f"split over {P} worker processes ({per} weights each, one per host core): "
+              f"{3 * ps.K} perturb passes + preconditioner + fused update per step, by the oracle's "
+              f"element-list routines; wall time of the slowest worker")
+    return value, dt, M, P, sample
 
 
 def param_set(args):
@@ -235,14 +268,14 @@ def run_reference(args):
     if rank != 0:
         return
     ps = param_set(args)
-    value, dt, M, sample = time_oracle(ps, args.cpu_seconds / 2, steps=args.steps, warmup=args.warmup,
-                                       packing=args.packing)
+    value, dt, M, cores, sample = time_oracle(ps, args.cpu_seconds / 2, steps=args.steps, warmup=args.warmup,
+                                              packing=args.packing, workers=args.cpu_workers)
     line = {
         "impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": args.gpus,
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": dt * 1e3, "higher_is_better": True,
         "scaling": "weak", "vs_baseline": None, "dtype": "f32", "data": "synthetic",
         "config": {"workload": ps.name, "K": ps.K, "d": ps.d, "packing": args.packing, "sample_weights": M},
-        "cpu_baseline": {"value": value, "unit": UNIT, "cores": 1, "kind": "oracle", "sample": sample},
+        "cpu_baseline": {"value": value, "unit": UNIT, "cores": cores, "kind": "oracle", "sample": sample},
         "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
     }
     print(json.dumps(line), flush=True)
@@ -416,8 +449,8 @@ def run_zo(args):
         return
     cpu = None
     if world == 1 and not args.no_cpu_baseline:
-        v, dt, M, sample = time_oracle(ps, args.cpu_seconds, packing=args.packing)
-        cpu = {"value": v, "unit": UNIT, "cores": 1, "kind": "oracle", "sample": sample}
+        v, dt, M, cores, sample = time_oracle(ps, args.cpu_seconds, packing=args.packing, workers=args.cpu_workers)
+        cpu = {"value": v, "unit": UNIT, "cores": cores, "kind": "oracle", "sample": sample}
     line = {
         "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
         "warmup": args.warmup, "ms_per_step": ms_per_step, "higher_is_better": True, "scaling": "weak",

@@ -401,3 +401,35 @@ def test_quadratic_loss():
     a = W.tiny_curvatures(10000)
     want = 0.5 * math.fsum(a.astype(np.float64) * th.astype(np.float64) ** 2)
     assert oracle.quadratic_loss(th, a) == pytest.approx(want, rel=1e-13)
+
+
+@pytest.mark.parametrize("dtype", [W.DT_F32, W.DT_BF16, W.DT_F16])
+def test_element_routines_match_list_routines(dtype):
+    """The element-list routines (sampled full-size parity, the CPU baseline)
+    compute what the tensor-list routines compute at the same virtual indices."""
+    rng = np.random.default_rng(21)
+    n = 3000
+    bits = W.random_storage(rng, n, dtype)
+    g = np.arange(n, dtype=np.uint64)
+    seed, eps = 0x15E5A0004, 1e-3
+    c = rng.standard_normal(12) * 3
+
+    def widen(b):
+        if dtype == W.DT_F32:
+            return b
+        if dtype == W.DT_F16:
+            return b.view(np.float16).astype(np.float32)
+        return (b.astype(np.uint32) << 16).view(np.float32)
+
+    def narrow(out):
+        return out.view(np.float32) if dtype == W.DT_F32 else out.astype(np.uint16)
+
+    t = [bits.copy()]
+    e = bits.copy()
+    for k, s in ((0, eps), (5, -2 * eps), (9, 0.25)):
+        oracle.perturb(t, [dtype], seed, k, s)
+        e = narrow(oracle.perturb_elements(dtype, g, widen(e), seed, k, s))
+        np.testing.assert_array_equal(e.view(np.uint8), t[0].view(np.uint8))
+    oracle.update(t, [dtype], seed, c, 1e-2)
+    e = narrow(oracle.update_elements(dtype, g, widen(e), seed, c, 1e-2))
+    np.testing.assert_array_equal(e.view(np.uint8), t[0].view(np.uint8))
