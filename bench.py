@@ -57,9 +57,13 @@ def parse_args():
                     help="keep the nvidia-smi clock samples of the timed region in this file")
     ap.add_argument("--packing", type=int, default=1, choices=[1, 8],
                     help="generated bits per (weight, probe): 1 (the paper's bit packing) or 8")
-    ap.add_argument("--schedule", default="fused", choices=["fused", "alg1"],
+    ap.add_argument("--schedule", default="fused", choices=["fused", "alg1", "pair"],
                     help="fused: each restore is folded into the next probe's +eps pass and the last one into "
-                         "the update (2K+1 passes); alg1: Algorithm 1's +eps, -2eps, +eps per probe (3K+1)")
+                         "the update (2K+1 passes); alg1: Algorithm 1's +eps, -2eps, +eps per probe (3K+1); "
+                         "pair: theta +- eps z_k written out of place by one pass per probe into two extra "
+                         "copies of the weights (K+1 passes, 3 copies in device memory)")
+    ap.add_argument("--no-pair", action="store_true",
+                    help="skip the extra measurement of the out-of-place pair schedule")
     ap.add_argument("--sequential", action="store_true",
                     help="also time Algorithm 1's K sequential passes against the fused update")
     return ap.parse_args()
@@ -314,8 +318,12 @@ def run_zo(args):
     status = torch.zeros(1, dtype=torch.int32, device=dev)
     stream = torch.cuda.current_stream(dev)
     chunks = (len(params) + 1023) // 1024
+    pair = args.schedule == "pair"
+    if pair:
+        plus = zo.ParamList([torch.empty_like(t) for t in params])
+        minus = zo.ParamList([torch.empty_like(t) for t in params])
 
-    timing = {"perturb": [], "perturb2": [], "update": [], "precondition": []}
+    timing = {"perturb": [], "perturb2": [], "pair": [], "update": [], "precondition": []}
     fused = args.schedule == "fused"
 
     def timed(key, record, fn, *a, **kw):
@@ -333,7 +341,10 @@ def run_zo(args):
         +eps and each -2eps pass. The fused schedule leaves the weights at
         those points, and at the end, bit for bit as Algorithm 1's does."""
         seed = W.step_seed(s)
-        if fused:
+        if pair:
+            for k in range(K):
+                timed("pair", record, zo.perturb_pair, plist, plus, minus, seed, k, eps)
+        elif fused:
             timed("perturb", record, zo.perturb, plist, seed, 0, eps)
             for k in range(K):
                 timed("perturb", record, zo.perturb, plist, seed, k, -2 * eps)
@@ -370,8 +381,11 @@ def run_zo(args):
     clk = clocks.stop()
     elapsed_ms = ranks_max(t_start.elapsed_time(t_end))
     ms_per_step = elapsed_ms / args.steps
-    passes = 2 * K + 1 if fused else 3 * K + 1   # sweeps over the weights per step (update included)
-    launches = args.steps * ((passes - 1) * chunks + 1 + chunks)
+    passes = K + 1 if pair else (2 * K + 1 if fused else 3 * K + 1)   # sweeps over the weights, update included
+    if pair:
+        launches = args.steps * (K * chunks + 1 + chunks)
+    else:
+        launches = args.steps * ((passes - 1) * chunks + 1 + chunks)
 
     def avg_ms(key):
         v = [a.elapsed_time(b) for a, b in timing[key]]
@@ -379,6 +393,7 @@ def run_zo(args):
 
     perturb_ms = ranks_max(avg_ms("perturb"))
     perturb2_ms = ranks_max(avg_ms("perturb2"))
+    pair_ms = ranks_max(avg_ms("pair"))
     update_ms = ranks_max(avg_ms("update"))
     precond_ms = ranks_max(avg_ms("precondition"))
 
@@ -405,6 +420,45 @@ def run_zo(args):
         e2e = {"value": whole_job_rate(world, d, K, e2e_s), "unit": UNIT, "h2d_bytes_per_step": K * 3 * 8,
                "d2h_bytes_per_step": K * 8 + 4, "ms_per_step": e2e_s * 1e3}
 
+    # ---- the out-of-place pair schedule on the same weights (two more copies)
+    pair_alt = None
+    if not pair and not args.no_pair:
+        free, _ = torch.cuda.mem_get_info(dev)
+        if free > 2.05 * d * ps.bytes_per_elem:
+            plus_a = zo.ParamList([torch.empty_like(t) for t in params])
+            minus_a = zo.ParamList([torch.empty_like(t) for t in params])
+            ev = []
+
+            def pair_step(s, record):
+                seed = W.step_seed(s)
+                e = [torch.cuda.Event(enable_timing=True) for _ in range(3)]
+                e[0].record(stream)
+                for k in range(K):
+                    zo.perturb_pair(plist, plus_a, minus_a, seed, k, eps)
+                e[1].record(stream)
+                zo.precondition(losses_dev[s], eps, out=(c, status))
+                zo.update(plist, seed, c, eps, status=status)
+                e[2].record(stream)
+                if record:
+                    ev.append(e)
+
+            pair_step(0, False)
+            barrier()
+            for i in range(args.steps):
+                pair_step(args.warmup + i, True)
+            barrier()
+            step_ms = ranks_max(sum(e[0].elapsed_time(e[2]) for e in ev) / len(ev))
+            pass_ms = ranks_max(sum(e[0].elapsed_time(e[1]) for e in ev) / len(ev) / K)
+            pbytes = 3.0 * d * ps.bytes_per_elem
+            pair_alt = {"schedule": f"pair ({K + 1} passes: theta +- eps z_k written out of place into two extra "
+                                    "copies, then the preconditioner and the fused update)",
+                        "value": whole_job_rate(world, d, K, step_ms * 1e-3), "unit": UNIT, "ms_per_step": step_ms,
+                        "device_copies_of_weights": 3, "perturb_pair_ms": pass_ms,
+                        "perturb_pair_GB/s": pbytes / (pass_ms * 1e-3) / 1e9,
+                        "step_hbm_bytes": K * pbytes + 2.0 * d * ps.bytes_per_elem}
+            del plus_a, minus_a
+            torch.cuda.empty_cache()
+
     # ---- Algorithm 1's K-pass update against the fused one (same coefficients)
     seq = None
     if args.sequential:
@@ -428,17 +482,27 @@ def run_zo(args):
 
     peaks, peak_kind = measured_peaks()
     hbm_peak = float(peaks.get("hbm_gbs", FALLBACK_HBM_GBS))
+    if pair_alt is not None:
+        pair_alt["perturb_pair_frac_of_measured_hbm"] = pair_alt["perturb_pair_GB/s"] / hbm_peak
     perturb_bytes = 2.0 * d * ps.bytes_per_elem       # read + write every weight once
-    achieved = perturb_bytes / (perturb_ms * 1e-3) / 1e9
+    pair_bytes = 3.0 * d * ps.bytes_per_elem          # read theta, write plus and minus
+    achieved = perturb_bytes / (perturb_ms * 1e-3) / 1e9 if perturb_ms > 0 else None
     # the roofline is reported for the kernel with the largest share of the step
-    n1, n2 = (K + 1, K - 1) if fused else (3 * K, 0)
-    if n2 > 0 and n2 * perturb2_ms > n1 * perturb_ms:
+    n1, n2 = (K + 1, K - 1) if fused else ((0, 0) if pair else (3 * K, 0))
+    if pair:
+        dom_kernel, dom_ms, dom_launches = "perturb_pair_kernel", pair_ms, K
+        traffic = committed_traffic("perturb_pair_kernel", args.config)
+    elif n2 > 0 and n2 * perturb2_ms > n1 * perturb_ms:
         dom_kernel, dom_ms, dom_launches = "perturb_kernel<2>", perturb2_ms, n2
         traffic = committed_traffic("perturb2_kernel", args.config)
     else:
         dom_kernel, dom_ms, dom_launches = "perturb_kernel<1>", perturb_ms, n1
         traffic = committed_traffic("perturb_kernel", args.config)
-    dom_achieved = perturb_bytes / (dom_ms * 1e-3) / 1e9
+    dom_bytes = pair_bytes if pair else perturb_bytes
+    # algorithmic HBM bytes of one step: every pass reads and writes theta once,
+    # except the pair passes (read theta, write two copies)
+    step_bytes = K * pair_bytes + perturb_bytes if pair else passes * perturb_bytes
+    dom_achieved = dom_bytes / (dom_ms * 1e-3) / 1e9
     sms = torch.cuda.get_device_properties(dev).multi_processor_count
     sm_mhz = (clk or {}).get("sm_mhz") or float(peaks.get("sm_max_mhz", 2070.0))
     alu_peak = sms * LANES_PER_SM * sm_mhz * 1e6 / 1e9    # Gparam*probe/s at one instruction per pair
@@ -463,18 +527,21 @@ def run_zo(args):
                    "l2": "inputs larger than L2 (every pass streams the whole parameter set)"},
         "roofline": {"bound": "hbm", "kernel": dom_kernel, "achieved": dom_achieved, "peak": hbm_peak,
                      "unit": "GB/s", "frac": dom_achieved / hbm_peak, "traffic": traffic,
-                     "peak_source": f"{peak_kind} hbm_gbs", "bytes_per_launch": perturb_bytes,
+                     "peak_source": f"{peak_kind} hbm_gbs", "bytes_per_launch": dom_bytes,
                      "launches_per_step": dom_launches * chunks,
                      "step_share": dom_launches * dom_ms / ms_per_step},
         "kernels": {
-            "perturb": {"ms": perturb_ms, "GB/s": achieved, "frac_of_measured_hbm": achieved / hbm_peak,
-                        "frac_of_nominal_hbm": achieved / NOMINAL_HBM_GBS,
-                        "launches_per_step": (K + 1 if fused else 3 * K) * chunks},
+            "perturb": ({"ms": perturb_ms, "GB/s": achieved, "frac_of_measured_hbm": achieved / hbm_peak,
+                         "frac_of_nominal_hbm": achieved / NOMINAL_HBM_GBS,
+                         "launches_per_step": (K + 1 if fused else 3 * K) * chunks} if not pair else None),
+            "pair": ({"ms": pair_ms, "GB/s": pair_bytes / (pair_ms * 1e-3) / 1e9,
+                      "frac_of_measured_hbm": pair_bytes / (pair_ms * 1e-3) / 1e9 / hbm_peak,
+                      "bytes_per_pass": pair_bytes, "launches_per_step": K * chunks} if pair else None),
             "perturb2": ({"ms": perturb2_ms, "GB/s": perturb_bytes / (perturb2_ms * 1e-3) / 1e9,
                           "frac_of_measured_hbm": perturb_bytes / (perturb2_ms * 1e-3) / 1e9 / hbm_peak,
                           "launches_per_step": (K - 1) * chunks} if fused and K > 1 else None),
-            "step_hbm": {"passes": passes, "ideal_ms": passes * perturb_bytes / (hbm_peak * 1e9) * 1e3,
-                         "frac": passes * perturb_bytes / (hbm_peak * 1e9) / (ms_per_step * 1e-3)},
+            "step_hbm": {"passes": passes, "bytes": step_bytes, "ideal_ms": step_bytes / (hbm_peak * 1e9) * 1e3,
+                         "frac": step_bytes / (hbm_peak * 1e9) / (ms_per_step * 1e-3)},
             "update": {"ms": update_ms, "gparam_probe_per_s": upd_rate, "bound": "alu",
                        "peak_gparam_probe_per_s_1instr": alu_peak, "frac_alu_1instr": upd_rate / alu_peak,
                        "GB/s": perturb_bytes / (update_ms * 1e-3) / 1e9},
@@ -482,6 +549,7 @@ def run_zo(args):
         },
         "e2e": e2e,
         "sequential": seq,
+        "pair_schedule": pair_alt,
         "gpu_launches": launches,
         "clocks": clk,
         "cpu_baseline": cpu,

@@ -135,6 +135,26 @@ int zo_perturb(const zo_tensor* params, int32_t n_tensors, uint64_t seed, uint32
 int zo_perturb2(const zo_tensor* params, int32_t n_tensors, uint64_t seed, uint32_t probe_a, float scale_a,
                 uint32_t probe_b, float scale_b, void* stream);
 
+/* zo_perturb_pair -- both forward points of probe k in one pass, out of place:
+ *   plus  <- rn( fp32(theta) + scale * z_k )
+ *   minus <- rn( fp32(theta) - scale * z_k )
+ * for every tensor, theta left untouched (Sec. 2 / Eq. 3 evaluate the loss at
+ * theta +- eps z; Algorithm 1 reaches them in place by +eps, -2 eps, +eps).
+ * theta is read once and the two results written once: 6 bytes per 16-bit
+ * weight instead of the 8 of two in-place passes, no restore pass and no
+ * restore drift, for two extra copies of the weights in device memory.
+ * The probes are zo_perturb's: `theta` is the parameter list of the step
+ * (virtual indices from its sizes); plus and minus are lists of the same
+ * length with the same numel and dtype per entry. plus[t] may be theta[t]
+ * itself (then theta becomes theta + scale z) and so may minus[t]; plus[t]
+ * and minus[t] must be different, and any other overlap is undefined.
+ * The vectorised path needs all three pointers of a tensor 32-byte aligned.
+ * Errors: ZO_ERR_ARG (also for mismatched lists or plus[t] == minus[t]),
+ * ZO_ERR_DTYPE, ZO_ERR_ALIGN, ZO_ERR_CUDA. No counterpart in the paper as a
+ * kernel: it trades device memory for HBM traffic. */
+int zo_perturb_pair(const zo_tensor* theta, const zo_tensor* plus, const zo_tensor* minus, int32_t n_tensors,
+                    uint64_t seed, uint32_t probe, float scale, void* stream);
+
 /* ---------------------------------------------------------------------------
  * zo_precondition -- the probe-space diagonal preconditioner of Sec. 4.1 with
  * the paper's settings (alpha = 0.1, lambda_reg = 1, two-sided difference).

@@ -188,7 +188,35 @@ int run_perturb(const zo_tensor* params, int32_t n, PerturbParams& pp, DeviceInf
   return ZO_OK;
 }
 
+// Fill a pair table with tensors t0, t0+1, ... (same split rules as
+// fill_table).
+int32_t fill_pair_table(zo::PairTable& tab, const zo_tensor* theta, const zo_tensor* plus, const zo_tensor* minus,
+                        int32_t t0, int32_t n, int64_t blk_base, int64_t* nblocks) {
+  tab.n = 0;
+  tab.blk_base = blk_base;
+  int64_t b = 0;
+  int32_t t = t0;
+  for (; t < n && tab.n < zo::kMaxTensorsPerLaunch; ++t) {
+    const int64_t nb = (theta[t].numel + 15) / 16;
+    if (tab.n > 0 && b + nb >= zo::kMaxLaunchBlocks) break;
+    const int i = tab.n++;
+    b += nb;
+    tab.blk_end[i] = static_cast<uint32_t>(b);
+    tab.src[i] = reinterpret_cast<uint64_t>(theta[t].ptr);
+    tab.plus[i] = reinterpret_cast<uint64_t>(plus[t].ptr);
+    tab.minus[i] = reinterpret_cast<uint64_t>(minus[t].ptr);
+    tab.last[i] = static_cast<uint8_t>(theta[t].numel - 16 * (nb > 0 ? nb - 1 : 0));  // 1..16 (0 if empty)
+    uint8_t fl = static_cast<uint8_t>(theta[t].dtype);
+    if ((tab.src[i] | tab.plus[i] | tab.minus[i]) % 32 == 0) fl |= zo::kVec32;
+    tab.flags[i] = fl;
+  }
+  tab.blk_total = static_cast<uint32_t>(b);
+  *nblocks = b;
+  return t;
+}
+
 thread_local PerturbParams tl_perturb;
+thread_local zo::PairParams tl_pair;
 thread_local UpdateParams tl_update;
 
 }  // namespace
@@ -211,7 +239,7 @@ const char* zo_status_string(int status) {
 
 const char* zo_last_cuda_error(void) { return g_last_cuda_error; }
 
-int zo_version(void) { return 10200; }
+int zo_version(void) { return 10300; }
 
 int zo_set_packing(int32_t bits_per_value) {
   if (bits_per_value != zo::kPacking1 && bits_per_value != zo::kPacking8) return ZO_ERR_ARG;
@@ -260,6 +288,38 @@ int zo_perturb2(const zo_tensor* params, int32_t n_tensors, uint64_t seed, uint3
   pp.coef_mul = 0.0;
   pp.status = nullptr;
   return run_perturb(params, n_tensors, pp, d, static_cast<cudaStream_t>(stream));
+}
+
+int zo_perturb_pair(const zo_tensor* theta, const zo_tensor* plus, const zo_tensor* minus, int32_t n_tensors,
+                    uint64_t seed, uint32_t probe, float scale, void* stream) {
+  int rc = validate_params(theta, n_tensors);
+  if (rc != ZO_OK) return rc;
+  if ((rc = validate_params(plus, n_tensors)) != ZO_OK) return rc;
+  if ((rc = validate_params(minus, n_tensors)) != ZO_OK) return rc;
+  if (!std::isfinite(scale)) return ZO_ERR_ARG;
+  for (int32_t t = 0; t < n_tensors; ++t) {
+    if (plus[t].numel != theta[t].numel || minus[t].numel != theta[t].numel) return ZO_ERR_ARG;
+    if (plus[t].dtype != theta[t].dtype || minus[t].dtype != theta[t].dtype) return ZO_ERR_ARG;
+    if (theta[t].numel > 0 && plus[t].ptr == minus[t].ptr) return ZO_ERR_ARG;
+  }
+  if (n_tensors == 0) return ZO_OK;
+  DeviceInfo* d = nullptr;
+  if ((rc = device_info(&d)) != ZO_OK) return rc;
+  zo::PairParams& pp = tl_pair;
+  pp.keys = expand_keys(seed);
+  pp.op = make_op(probe, scale, g_packing.load());
+  int64_t blk = 0;
+  for (int32_t t0 = 0; t0 < n_tensors;) {
+    int64_t nb = 0;
+    t0 = fill_pair_table(pp.tab, theta, plus, minus, t0, n_tensors, blk, &nb);
+    if (nb > 0) {
+      cudaError_t e = zo::launch_perturb_pair(pp, grid_for(nb, d->sms, d->perturb_bps),
+                                              static_cast<cudaStream_t>(stream));
+      if (e != cudaSuccess) return cuda_fail(e, "perturb_pair_kernel");
+    }
+    blk += nb;
+  }
+  return ZO_OK;
 }
 
 static int check_update_args(const zo_tensor* params, int32_t n, const double* c, int32_t K, double lr) {

@@ -17,6 +17,7 @@ constexpr int kStaticLossPartials = 4096;   // fixed scratch of the allocation-f
 constexpr int64_t kStaticLossSlice = 2048;  // elements per partial in that variant
 
 cudaError_t launch_perturb(const PerturbParams& p, int grid, cudaStream_t stream);
+cudaError_t launch_perturb_pair(const PairParams& p, int grid, cudaStream_t stream);
 cudaError_t launch_update(const UpdateParams& p, int grid, cudaStream_t stream);
 size_t update_smem_bytes(int groups);
 cudaError_t perturb_blocks_per_sm(int* out);

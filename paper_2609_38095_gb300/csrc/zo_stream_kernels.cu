@@ -180,6 +180,102 @@ __global__ void __launch_bounds__(256) perturb_kernel(const __grid_constant__ Pe
 }
 
 // ---------------------------------------------------------------------------
+// Out-of-place pair: plus <- rn(fp32(theta) + v), minus <- rn(fp32(theta) - v)
+// with v = scale z_k[g] (exact), theta untouched. One read of theta and two
+// writes instead of the three read-modify-write passes of +eps / -2 eps /
+// +eps, and both forward points are one rounding away from theta.
+// ---------------------------------------------------------------------------
+template <uint8_t DT>
+__device__ __forceinline__ void pair_regs16(const uint32_t (&v)[8], const uint4& x, const PerturbOp& op,
+                                            uint32_t (&p)[8], uint32_t (&m)[8]) {
+#pragma unroll
+  for (int r = 0; r < 8; ++r) {
+    const float2 f = unpack2<DT>(v[r]);
+    const float d0 = __uint_as_float(op.nscale_bits ^ sign_bit(x, 2 * r, op.bit));
+    const float d1 = __uint_as_float(op.nscale_bits ^ sign_bit(x, 2 * r + 1, op.bit));
+    p[r] = pack2<DT>(__fadd_rn(f.x, d0), __fadd_rn(f.y, d1));
+    m[r] = pack2<DT>(__fsub_rn(f.x, d0), __fsub_rn(f.y, d1));
+  }
+}
+
+// n full, 32-byte aligned 16-bit blocks, pipelined like perturb_run16.
+template <uint8_t DT>
+__device__ __forceinline__ void pair_run16(const uint16_t* s, uint16_t* pp, uint16_t* mp, uint32_t n, size_t pstride,
+                                           int64_t vb, uint32_t stride, const PerturbOp& op, const RoundKeys& keys) {
+  uint32_t v[8];
+  ld256(s, v);
+  for (uint32_t i = 0; i < n; ++i) {
+    const uint16_t* sn = s + pstride;
+    uint32_t vn[8];
+    if (i + 1 < n) ld256(sn, vn);
+    const uint4 x = block_bits(vb, op.ctr2, keys);
+    uint32_t p[8], m[8];
+    pair_regs16<DT>(v, x, op, p, m);
+    st256(pp, p);
+    st256(mp, m);
+    s = sn;
+    pp += pstride;
+    mp += pstride;
+    vb += stride;
+#pragma unroll
+    for (int r = 0; r < 8; ++r) v[r] = vn[r];
+  }
+}
+
+__device__ __noinline__ void pair_block_other(const PairTable& tab, int t, uint32_t b, uint4 x, PerturbOp op) {
+  const uint32_t tb = t == 0 ? 0u : tab.blk_end[t - 1];
+  const int64_t e0 = static_cast<int64_t>(b - tb) * 16;
+  const int cnt = b + 1 == tab.blk_end[t] ? tab.last[t] : 16;
+  const uint8_t dt = tab.flags[t] & kDtypeMask;
+  const void* src = reinterpret_cast<const void*>(tab.src[t]);
+  void* pl = reinterpret_cast<void*>(tab.plus[t]);
+  void* mi = reinterpret_cast<void*>(tab.minus[t]);
+  for (int i = 0; i < cnt; ++i) {
+    const float th = load_elem(src, dt, e0 + i);
+    const float d = __uint_as_float(op.nscale_bits ^ sign_bit(x, i, op.bit));
+    store_elem(pl, dt, e0 + i, __fadd_rn(th, d));
+    store_elem(mi, dt, e0 + i, __fsub_rn(th, d));
+  }
+}
+
+__global__ void __launch_bounds__(256, 4) perturb_pair_kernel(const __grid_constant__ PairParams P) {
+  const PairTable& tab = P.tab;
+  const PerturbOp op = P.op;
+  const uint32_t stride = gridDim.x * blockDim.x;
+  uint32_t b = blockIdx.x * blockDim.x + threadIdx.x;  // < 2^31 + stride: never wraps
+  int t = 0;
+  uint32_t tb = 0, te = 0, tfe = 0;
+  uint8_t dt = 0;
+  bool seeked = false;
+  while (b < tab.blk_total) {
+    if (!seeked || b >= te) {
+      while (b >= tab.blk_end[t]) ++t;
+      tb = t == 0 ? 0u : tab.blk_end[t - 1];
+      te = tab.blk_end[t];
+      dt = tab.flags[t] & kDtypeMask;
+      tfe = ((tab.flags[t] & kVec32) && dt != kF32) ? te - (tab.last[t] < 16 ? 1u : 0u) : tb;  // full blocks
+      seeked = true;
+    }
+    const int64_t vb = tab.blk_base + b;
+    if (b < tfe) {
+      const uint32_t n = (tfe - b + stride - 1) / stride;
+      const size_t off = static_cast<size_t>(b - tb) * 16, pstride = static_cast<size_t>(stride) * 16;
+      const uint16_t* s = reinterpret_cast<const uint16_t*>(tab.src[t]) + off;
+      uint16_t* pp = reinterpret_cast<uint16_t*>(tab.plus[t]) + off;
+      uint16_t* mp = reinterpret_cast<uint16_t*>(tab.minus[t]) + off;
+      if (dt == kBF16)
+        pair_run16<kBF16>(s, pp, mp, n, pstride, vb, stride, op, P.keys);
+      else
+        pair_run16<kF16>(s, pp, mp, n, pstride, vb, stride, op, P.keys);
+      b += n * stride;
+    } else {
+      pair_block_other(tab, t, b, block_bits(vb, op.ctr2, P.keys), op);
+      b += stride;
+    }
+  }
+}
+
+// ---------------------------------------------------------------------------
 // Fused K-probe update: theta <- rn(fp32(theta) + sum_k a_k z_k[g]).
 //
 // Byte m of Philox(b, q) holds the signs of probes 8q..8q+7 for element
@@ -450,6 +546,15 @@ cudaError_t launch_perturb(const PerturbParams& p, int grid, cudaStream_t stream
     perturb_kernel<2><<<grid, kThreads, 0, stream>>>(p);
   else
     perturb_kernel<1><<<grid, kThreads, 0, stream>>>(p);
+  return cudaGetLastError();
+}
+
+static_assert(sizeof(PairParams) <= 32764, "pair table exceeds the kernel parameter space");
+static_assert(sizeof(PerturbParams) <= 32764 && sizeof(UpdateParams) <= 32764,
+              "tensor table exceeds the kernel parameter space");
+
+cudaError_t launch_perturb_pair(const PairParams& p, int grid, cudaStream_t stream) {
+  perturb_pair_kernel<<<grid, kThreads, 0, stream>>>(p);
   return cudaGetLastError();
 }
 

@@ -28,7 +28,7 @@ ZO_PRECOND_RELATIVE_CURVATURE = 2
 DTYPE_CODE = {torch.float32: 0, torch.bfloat16: 1, torch.float16: 2}
 
 EXPORTS = ["zo_status_string", "zo_last_cuda_error", "zo_version", "zo_set_packing", "zo_get_packing",
-           "zo_perturb", "zo_perturb2", "zo_precondition",
+           "zo_perturb", "zo_perturb2", "zo_perturb_pair", "zo_precondition",
            "zo_precondition_ex", "zo_update", "zo_update_ex", "zo_update_sequential", "zo_probe_bytes", "zo_probe_signs",
            "zo_quadratic_loss_workspace_size", "zo_quadratic_loss", "zo_quadratic_loss_static"]
 ZO_QUADRATIC_LOSS_STATIC_MAX_N = 8388608
@@ -68,6 +68,7 @@ def _lib():
             "zo_get_packing": ([], c.c_int),
             "zo_perturb": ([vp, i32, u64, u32, f32, vp], c.c_int),
             "zo_perturb2": ([vp, i32, u64, u32, f32, u32, f32, vp], c.c_int),
+            "zo_perturb_pair": ([vp, vp, vp, i32, u64, u32, f32, vp], c.c_int),
             "zo_update_ex": ([vp, i32, u64, vp, i32, f64, vp, i32, u32, f32, vp], c.c_int),
             "zo_precondition": ([vp, i32, f64, vp, vp, vp], c.c_int),
             "zo_precondition_ex": ([vp, i32, f64, f64, f64, i32, vp, vp, vp, vp, vp], c.c_int),
@@ -195,6 +196,20 @@ def perturb2(params, seed: int, probe_a: int, scale_a: float, probe_b: int, scal
     with torch.cuda.device(p.device):
         _check("zo_perturb2", _lib().zo_perturb2(p._arr, p.n, seed, probe_a, scale_a, probe_b, scale_b,
                                                  _stream(p.device)))
+
+
+def perturb_pair(params, plus, minus, seed: int, probe: int, scale: float):
+    """plus <- theta + scale z_k and minus <- theta - scale z_k, both rounded
+    once to storage, theta untouched, in one pass (zo_perturb_pair). plus and
+    minus are lists of tensors shaped like params (same numel and dtype)."""
+    p, pl, mi = _plist(params), _plist(plus), _plist(minus)
+    if not (pl.n == mi.n == p.n):
+        raise ValueError("plus and minus must have one tensor per parameter")
+    if (pl.n and pl.device != p.device) or (mi.n and mi.device != p.device):
+        raise ValueError("plus and minus must live on the parameters' device")
+    with torch.cuda.device(p.device):
+        _check("zo_perturb_pair", _lib().zo_perturb_pair(p._arr, pl._arr, mi._arr, p.n, seed, probe, scale,
+                                                         _stream(p.device)))
 
 
 def precondition(losses, eps: float, alpha: float = 0.1, lambda_reg: float = 1.0, one_sided: bool = False,

@@ -100,3 +100,37 @@ def assert_update_close(got_bits, want_bits, dt, c, lr, context="", min_one_ulp=
     if dt != W.DT_F32 and g.size >= 1000:   # the one-ulp bar is stated for bf16 / fp16 storage
         one = ulp_distance16(got_bits, want_bits) <= 1
         assert np.mean(one) >= min_one_ulp, (context, float(np.mean(one)))
+
+
+def sample_positions(numels, n_random=1 << 16, seed=0):
+    """(tensor index, element index) pairs: ends of every tensor + uniform."""
+    numels = np.asarray(numels, dtype=np.int64)
+    cum = np.concatenate([[0], np.cumsum(numels)])
+    rng = np.random.default_rng(seed)
+    flat = rng.integers(0, cum[-1], n_random)
+    t_r = np.searchsorted(cum, flat, side="right") - 1
+    i_r = flat - cum[t_r]
+    ts, is_ = [t_r], [i_r]
+    for t, n in enumerate(numels):
+        if n == 0:
+            continue
+        e = np.unique(np.concatenate([np.arange(min(16, n)), np.arange(max(0, n - 16), n)]))
+        ts.append(np.full(e.size, t))
+        is_.append(e)
+    t_all = np.concatenate(ts)
+    i_all = np.concatenate(is_)
+    order = np.lexsort((i_all, t_all))
+    return t_all[order], i_all[order]
+
+
+def gather(params, t_idx, i_idx):
+    """Storage bits and fp32 values of the sampled elements."""
+    out_bits, out_f32 = [], []
+    bounds = np.flatnonzero(np.diff(np.concatenate([[-1], t_idx, [len(params)]])))
+    for a, b in zip(bounds[:-1], bounds[1:]):
+        t = int(t_idx[a])
+        idx = torch.from_numpy(i_idx[a:b]).to(params[t].device)
+        v = params[t][idx]
+        out_f32.append(v.float().cpu().numpy())
+        out_bits.append(storage_bits(v))
+    return np.concatenate(out_bits), np.concatenate(out_f32)

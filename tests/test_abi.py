@@ -34,7 +34,7 @@ def test_exports_every_declared_symbol(L):
 
 
 def test_version_and_strings(L):
-    assert zo.version() == 10200
+    assert zo.version() == 10300
     for s in (0, -1, -2, -3, -4, -5, -6, -7):
         assert zo.status_string(s).startswith("ZO_")
     assert "unknown" in zo.status_string(99)
@@ -66,6 +66,22 @@ def test_perturb_validation(L):
     bad_res[0].reserved = 1
     assert L.zo_perturb(bad_res, 1, 1, 0, 1e-3, None) == zo.ZO_ERR_ARG
     assert L.zo_perturb(None, 0, 1, 0, 1e-3, None) == zo.ZO_OK  # empty list: nothing to do
+
+
+def test_perturb_pair_validation(L):
+    th = tensors((FAKE, 16, 1), (FAKE + 64, 40, 2))
+    pl = tensors((FAKE + 4096, 16, 1), (FAKE + 8192, 40, 2))
+    mi = tensors((FAKE + 16384, 16, 1), (FAKE + 32768, 40, 2))
+    f = L.zo_perturb_pair
+    assert f(th, pl, mi, -1, 1, 0, 1e-3, None) == zo.ZO_ERR_ARG
+    assert f(th, None, mi, 2, 1, 0, 1e-3, None) == zo.ZO_ERR_ARG
+    assert f(th, pl, mi, 2, 1, 0, float("nan"), None) == zo.ZO_ERR_ARG
+    assert f(th, tensors((FAKE + 4096, 16, 1), (FAKE + 8192, 41, 2)), mi, 2, 1, 0, 1e-3, None) == zo.ZO_ERR_ARG
+    assert f(th, pl, tensors((FAKE + 16384, 16, 1), (FAKE + 32768, 40, 1)), 2, 1, 0, 1e-3, None) == zo.ZO_ERR_ARG
+    assert f(th, pl, tensors((FAKE + 4096, 16, 1), (FAKE + 32768, 40, 2)), 2, 1, 0, 1e-3, None) == zo.ZO_ERR_ARG
+    assert f(th, pl, tensors((FAKE + 16385, 16, 1), (FAKE + 32768, 40, 2)), 2, 1, 0, 1e-3, None) == zo.ZO_ERR_ALIGN
+    assert f(th, pl, tensors((FAKE + 16384, 16, 3), (FAKE + 32768, 40, 2)), 2, 1, 0, 1e-3, None) == zo.ZO_ERR_DTYPE
+    assert f(None, None, None, 0, 1, 0, 1e-3, None) == zo.ZO_OK
 
 
 def test_update_validation(L):

@@ -14,7 +14,7 @@ from paper_2609_38095_gb300 import build as zo_build
 from paper_2609_38095_gb300 import workloads as W
 from paper_2609_38095_gb300 import zo
 
-from gpu_helpers import assert_update_close, storage_bits
+from gpu_helpers import assert_update_close, gather, sample_positions
 
 pytestmark = pytest.mark.gpu
 
@@ -25,40 +25,6 @@ def _built():
         pytest.skip("no CUDA device")
     zo_build.build()
     oracle.lib()
-
-
-def sample_positions(numels, n_random=1 << 16, seed=0):
-    """(tensor index, element index) pairs: ends of every tensor + uniform."""
-    numels = np.asarray(numels, dtype=np.int64)
-    cum = np.concatenate([[0], np.cumsum(numels)])
-    rng = np.random.default_rng(seed)
-    flat = rng.integers(0, cum[-1], n_random)
-    t_r = np.searchsorted(cum, flat, side="right") - 1
-    i_r = flat - cum[t_r]
-    ts, is_ = [t_r], [i_r]
-    for t, n in enumerate(numels):
-        if n == 0:
-            continue
-        e = np.unique(np.concatenate([np.arange(min(16, n)), np.arange(max(0, n - 16), n)]))
-        ts.append(np.full(e.size, t))
-        is_.append(e)
-    t_all = np.concatenate(ts)
-    i_all = np.concatenate(is_)
-    order = np.lexsort((i_all, t_all))
-    return t_all[order], i_all[order]
-
-
-def gather(params, t_idx, i_idx):
-    """Storage bits and fp32 values of the sampled elements."""
-    out_bits, out_f32 = [], []
-    bounds = np.flatnonzero(np.diff(np.concatenate([[-1], t_idx, [len(params)]])))
-    for a, b in zip(bounds[:-1], bounds[1:]):
-        t = int(t_idx[a])
-        idx = torch.from_numpy(i_idx[a:b]).to(params[t].device)
-        v = params[t][idx]
-        out_f32.append(v.float().cpu().numpy())
-        out_bits.append(storage_bits(v))
-    return np.concatenate(out_bits), np.concatenate(out_f32)
 
 
 @pytest.mark.parametrize("key", ["opt-1.3b", "qwen3-8b", "opt-13b", "opt-30b"])

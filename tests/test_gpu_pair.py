@@ -1,0 +1,204 @@
+"""GPU parity of zo_perturb_pair (both forward points of a probe, out of
+place) against the CPU oracle: plus and minus must equal the oracle's
+perturbation of a copy of theta by +scale and -scale, bit for bit, and theta
+must stay untouched. Also the schedule built on it: K pair passes, the
+preconditioner and the fused update leave theta where the oracle's update of
+the unperturbed theta puts it."""
+import gc
+
+import numpy as np
+import pytest
+import torch
+
+import oracle
+from paper_2609_38095_gb300 import build as zo_build
+from paper_2609_38095_gb300 import workloads as W
+from paper_2609_38095_gb300 import zo
+
+from gpu_helpers import (TORCH_TO_DT, assert_update_close, gather, sample_positions, storage_bits, storage_np,
+                         to_torch)
+
+pytestmark = pytest.mark.gpu
+
+DTS = [torch.float32, torch.bfloat16, torch.float16]
+NUMELS = [1, 15, 16, 17, 31, 33, 0, 255, 4096, 4099, 100003, 7, 65536 + 5]
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _built():
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    zo_build.build()
+    oracle.lib()
+
+
+def make(numels, dtypes, seed):
+    rng = np.random.default_rng(seed)
+    host = [W.random_storage(rng, n, TORCH_TO_DT[dt]) for n, dt in zip(numels, dtypes)]
+    return host, [to_torch(h, dt) for h, dt in zip(host, dtypes)]
+
+
+def like(dev, fill_seed):
+    """Buffers shaped like dev, filled with unrelated bits (the kernel must
+    overwrite every element)."""
+    g = torch.Generator(device="cuda").manual_seed(fill_seed)
+    out = []
+    for t in dev:
+        b = torch.empty_like(t)
+        if b.numel():
+            b.view(torch.uint8).copy_(torch.randint(0, 256, (b.numel() * b.element_size(),), generator=g,
+                                                    device="cuda", dtype=torch.uint8))
+        out.append(b)
+    return out
+
+
+def expect(host, dts, seed, k, scale):
+    plus = [h.copy() for h in host]
+    minus = [h.copy() for h in host]
+    oracle.perturb(plus, dts, seed, k, scale)
+    oracle.perturb(minus, dts, seed, k, -scale)
+    return plus, minus
+
+
+def assert_equal(dev, host, what):
+    for i, (d, h) in enumerate(zip(dev, host)):
+        got = storage_np(d)
+        view = np.uint32 if h.dtype == np.float32 else np.uint16
+        np.testing.assert_array_equal(got.view(view), h.view(view), err_msg=f"{what} tensor {i} numel {h.size}")
+
+
+@pytest.mark.parametrize("k,scale", [(0, 1e-3), (9, 1e-3), (255, 0.25), (1023, -3e-8)])
+def test_pair_bit_exact_mixed(k, scale, packing_mode):
+    dtypes = [DTS[i % 3] for i in range(len(NUMELS))]
+    dts = [TORCH_TO_DT[d] for d in dtypes]
+    host, dev = make(NUMELS, dtypes, seed=k)
+    plus, minus = like(dev, 1), like(dev, 2)
+    seed = W.step_seed(4)
+    zo.perturb_pair(dev, plus, minus, seed, k, scale)
+    want_p, want_m = expect(host, dts, seed, k, scale)
+    assert_equal(plus, want_p, "plus")
+    assert_equal(minus, want_m, "minus")
+    assert_equal(dev, host, "theta untouched")
+
+
+@pytest.mark.parametrize("which", ["theta", "plus", "minus"])
+@pytest.mark.parametrize("offset", [1, 8, 16])
+@pytest.mark.parametrize("dtype", [torch.bfloat16, torch.float16, torch.float32])
+def test_pair_unaligned(which, offset, dtype):
+    """Any one of the three pointers off the 32-byte grid sends the tensor to
+    the element-wise path; results are identical and nothing outside the views
+    is written."""
+    n = 4096 + 37
+    dt = TORCH_TO_DT[dtype]
+    rng = np.random.default_rng(offset)
+    bases = {}
+    views = {}
+    for name in ("theta", "plus", "minus"):
+        off = offset if name == which else 0
+        h = W.random_storage(rng, n + off + 64, dt)
+        bases[name] = (h, to_torch(h, dtype), off)
+        views[name] = bases[name][1][off:off + n]
+    host = [bases["theta"][0][bases["theta"][2]:bases["theta"][2] + n].copy()]
+    seed = W.step_seed(7)
+    zo.perturb_pair([views["theta"]], [views["plus"]], [views["minus"]], seed, 21, 1e-3)
+    want_p, want_m = expect(host, [dt], seed, 21, 1e-3)
+    assert_equal([views["plus"]], want_p, "plus")
+    assert_equal([views["minus"]], want_m, "minus")
+    for name in ("plus", "minus", "theta"):
+        h, d, off = bases[name]
+        after = storage_np(d)
+        np.testing.assert_array_equal(after[:off], h[:off])
+        np.testing.assert_array_equal(after[off + n:], h[off + n:])
+
+
+def test_pair_split_launches(packing_mode):
+    """More tensors than one launch holds (1024)."""
+    rng = np.random.default_rng(31)
+    numels = [int(x) for x in rng.integers(0, 300, 2300)]
+    dtypes = [DTS[int(x)] for x in rng.integers(0, 3, 2300)]
+    dts = [TORCH_TO_DT[d] for d in dtypes]
+    host, dev = make(numels, dtypes, seed=31)
+    plus, minus = like(dev, 3), like(dev, 4)
+    seed = W.step_seed(8)
+    zo.perturb_pair(dev, plus, minus, seed, 77, 2e-3)
+    want_p, want_m = expect(host, dts, seed, 77, 2e-3)
+    assert_equal(plus, want_p, "plus")
+    assert_equal(minus, want_m, "minus")
+
+
+def test_pair_matches_in_place_perturb():
+    """plus equals zo_perturb(+scale) of a copy and minus zo_perturb(-scale),
+    on the GPU, bit for bit; plus may alias theta."""
+    dtypes = [DTS[i % 3] for i in range(len(NUMELS))]
+    _, dev = make(NUMELS, dtypes, seed=5)
+    a = [t.clone() for t in dev]
+    b = [t.clone() for t in dev]
+    seed = W.step_seed(2)
+    zo.perturb(a, seed, 14, 1e-3)
+    zo.perturb(b, seed, 14, -1e-3)
+    minus = like(dev, 6)
+    zo.perturb_pair(dev, dev, minus, seed, 14, 1e-3)      # plus aliases theta
+    assert_equal(dev, [storage_np(t) for t in a], "plus (aliasing theta) vs zo_perturb(+scale)")
+    assert_equal(minus, [storage_np(t) for t in b], "minus vs zo_perturb(-scale)")
+
+
+def test_pair_rejects_same_plus_and_minus():
+    _, dev = make([64], [torch.bfloat16], seed=1)
+    buf = like(dev, 7)
+    with pytest.raises(zo.ZoError):
+        zo.perturb_pair(dev, buf, buf, 1, 0, 1e-3)
+
+
+@pytest.mark.parametrize("K", [8, 19])
+def test_pair_schedule_step(K, packing_mode):
+    """K pair passes (theta untouched), the preconditioner, the fused update:
+    theta ends where the oracle's update of the unperturbed theta puts it, and
+    every pair matched the oracle's theta +- eps z_k."""
+    dtypes = [torch.bfloat16, torch.float16, torch.float32, torch.bfloat16]
+    numels = [5000, 4096 * 3 + 5, 777, 65536]
+    dts = [TORCH_TO_DT[d] for d in dtypes]
+    host, dev = make(numels, dtypes, seed=K)
+    plus, minus = like(dev, 8), like(dev, 9)
+    seed, eps = W.step_seed(K), 1e-3
+    for k in range(K):
+        zo.perturb_pair(dev, plus, minus, seed, k, eps)
+        if k in (0, K - 1):
+            want_p, want_m = expect(host, dts, seed, k, eps)
+            assert_equal(plus, want_p, f"plus k={k}")
+            assert_equal(minus, want_m, f"minus k={k}")
+    assert_equal(dev, host, "theta untouched by the pair passes")
+    L = W.synthetic_losses(K, step=K)
+    c, st = zo.precondition(torch.tensor(L, device="cuda"), eps)
+    zo.update(dev, seed, c, eps, status=st)
+    c_h = c.cpu().numpy()
+    oracle.update(host, dts, seed, c_h, eps)
+    for d, h, dt in zip(dev, host, dts):
+        assert_update_close(storage_bits(d), storage_bits(h), dt, c_h, eps, context="pair schedule")
+
+
+def test_pair_fullsize_sampled_opt13b():
+    """The OPT-13B-shaped set (25.7 GB, three copies on the device): sampled
+    elements of plus and minus against the oracle."""
+    ps = W.BY_KEY["opt-13b"]
+    free, _ = torch.cuda.mem_get_info()
+    if free < 3 * ps.d * ps.bytes_per_elem * 1.1:
+        pytest.skip("needs three copies of the OPT-13B-shaped set")
+    params = W.allocate_params(ps)
+    plus = [torch.empty_like(t) for t in params]
+    minus = [torch.empty_like(t) for t in params]
+    try:
+        S = oracle.virtual_offsets(ps.numels)
+        t_idx, i_idx = sample_positions(ps.numels)
+        g = (S[t_idx] + i_idx).astype(np.uint64)
+        seed, k = W.step_seed(1), ps.K - 1
+        bits0, f0 = gather(params, t_idx, i_idx)
+        zo.perturb_pair(zo.ParamList(params), zo.ParamList(plus), zo.ParamList(minus), seed, k, ps.eps)
+        bp, _ = gather(plus, t_idx, i_idx)
+        bm, _ = gather(minus, t_idx, i_idx)
+        np.testing.assert_array_equal(bp, oracle.perturb_elements(ps.dtype, g, f0, seed, k, ps.eps))
+        np.testing.assert_array_equal(bm, oracle.perturb_elements(ps.dtype, g, f0, seed, k, -ps.eps))
+        np.testing.assert_array_equal(gather(params, t_idx, i_idx)[0], bits0)   # theta untouched
+    finally:
+        del params, plus, minus
+        gc.collect()
+        torch.cuda.empty_cache()
