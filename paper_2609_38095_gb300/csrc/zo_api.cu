@@ -63,14 +63,18 @@ zo::PerturbOp make_op(uint32_t k, float scale, int packing) {
   uint32_t u;
   std::memcpy(&u, &scale, sizeof(u));
   op.nscale_bits = u ^ 0x80000000u;  // -scale: the probe bit flips it to +scale
+  for (uint32_t m = 0; m < 4; ++m) op.mul[m] = 1u << (31u - 8u * m - op.bit);
   return op;
 }
 
-// Resident perturb blocks per SM. The pass is HBM-bound and each thread keeps
-// two 32-byte loads in flight; on GB300 four 256-thread blocks per SM stream
-// fastest (measured: 3 -> 90.6 %, 4 -> 97.7 %, 5 -> 93.0 % of the copy
-// bandwidth on the 60 GB OPT-30B-shaped set), so the grid is capped there.
-constexpr int kPerturbBlocksPerSm = 4;
+// Resident perturb blocks per SM, by kernel. The passes are HBM-bound and each
+// thread keeps two 32-byte loads in flight. The single-op pass streams fastest
+// with four 256-thread blocks per SM (3 -> 90.6 %, 4 -> 97.7 %, 5 -> 93.0 % of
+// the copy bandwidth on the 60 GB OPT-30B-shaped set); the two-op and the
+// out-of-place pair passes, with more arithmetic per element and 80
+// registers, with three (two-op: 93.2 % at four, 96.5 % at three).
+constexpr int kPerturbBlocksPerSm[2] = {4, 3};  // by number of operations
+constexpr int kPairBlocksPerSm = 3;
 
 // The update is issue-bound; four waves of its blocks per SM keep more warps
 // eligible than one persistent wave (measured +3 % at K = 64 and 256).
@@ -79,7 +83,8 @@ constexpr int kUpdateWaves = 4;
 // Per-device launch facts, filled once per device.
 struct DeviceInfo {
   int sms = 0;
-  int perturb_bps = 0;                    // resident perturb blocks per SM
+  int perturb_bps[2] = {0, 0};            // perturb blocks per SM, single-op and two-op kernel
+  int pair_bps = 0;                       // perturb_pair blocks per SM
   int update_bps[2][zo::kMaxGroups + 1] = {};  // by packing (1, 8) and probe-group count
 };
 constexpr int kMaxDevices = 64;
@@ -98,9 +103,15 @@ int device_info(DeviceInfo** out) {
     e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
     if (e != cudaSuccess) return cuda_fail(e, "cudaDeviceGetAttribute");
     int bps = 0;
-    e = zo::perturb_blocks_per_sm(&bps);
-    if (e != cudaSuccess) return cuda_fail(e, "occupancy(perturb)");
-    d.perturb_bps = bps < 1 ? 1 : (bps < kPerturbBlocksPerSm ? bps : kPerturbBlocksPerSm);
+    for (int nops = 1; nops <= 2; ++nops) {
+      e = zo::perturb_blocks_per_sm(nops, &bps);
+      if (e != cudaSuccess) return cuda_fail(e, "occupancy(perturb)");
+      const int cap = kPerturbBlocksPerSm[nops - 1];
+      d.perturb_bps[nops - 1] = bps < 1 ? 1 : (bps < cap ? bps : cap);
+    }
+    e = zo::pair_blocks_per_sm(&bps);
+    if (e != cudaSuccess) return cuda_fail(e, "occupancy(perturb_pair)");
+    d.pair_bps = bps < 1 ? 1 : (bps < kPairBlocksPerSm ? bps : kPairBlocksPerSm);
     d.sms = sms;
   }
   *out = &d;
@@ -180,7 +191,7 @@ int run_perturb(const zo_tensor* params, int32_t n, PerturbParams& pp, DeviceInf
     int64_t nb = 0;
     t0 = fill_table(pp.tab, params, t0, n, blk, &nb);
     if (nb > 0) {
-      cudaError_t e = zo::launch_perturb(pp, grid_for(nb, d->sms, d->perturb_bps), s);
+      cudaError_t e = zo::launch_perturb(pp, grid_for(nb, d->sms, d->perturb_bps[pp.nops == 2 ? 1 : 0]), s);
       if (e != cudaSuccess) return cuda_fail(e, "perturb_kernel");
     }
     blk += nb;
@@ -313,7 +324,7 @@ int zo_perturb_pair(const zo_tensor* theta, const zo_tensor* plus, const zo_tens
     int64_t nb = 0;
     t0 = fill_pair_table(pp.tab, theta, plus, minus, t0, n_tensors, blk, &nb);
     if (nb > 0) {
-      cudaError_t e = zo::launch_perturb_pair(pp, grid_for(nb, d->sms, d->perturb_bps),
+      cudaError_t e = zo::launch_perturb_pair(pp, grid_for(nb, d->sms, d->pair_bps),
                                               static_cast<cudaStream_t>(stream));
       if (e != cudaSuccess) return cuda_fail(e, "perturb_pair_kernel");
     }

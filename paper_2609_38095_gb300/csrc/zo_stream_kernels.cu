@@ -34,6 +34,18 @@ __device__ __forceinline__ float add_signed(float th, const uint4& x, int i, con
   return __fadd_rn(th, __uint_as_float(op.nscale_bits ^ sign_bit(x, i, op.bit)));
 }
 
+// The same with the sign moved by a multiply (PerturbOp::mul), in the vector
+// loops: it moves half of the sign injection from the integer ALU, the busiest
+// pipe of these loops, to the multiply-add pipe (measured: single-op pass
+// -1.1 to -1.7 % time on the OPT-30B / OPT-13B-shaped sets).
+__device__ __forceinline__ uint32_t sign_bit_mul(const uint4& x, int i, const PerturbOp& op) {
+  return (word_of(x, i >> 2) * op.mul[i & 3]) & 0x80000000u;
+}
+
+__device__ __forceinline__ float add_signed_mul(float th, const uint4& x, int i, const PerturbOp& op) {
+  return __fadd_rn(th, __uint_as_float(op.nscale_bits ^ sign_bit_mul(x, i, op)));
+}
+
 __device__ __forceinline__ uint4 block_bits(int64_t b, uint32_t ctr2, const RoundKeys& keys) {
   return philox10(static_cast<uint32_t>(b), static_cast<uint32_t>(static_cast<uint64_t>(b) >> 32), ctr2, 0u, keys);
 }
@@ -46,7 +58,7 @@ __device__ __forceinline__ void perturb_regs16(uint32_t (&v)[8], const uint4 (&x
 #pragma unroll
     for (int o = 0; o < NOPS; ++o) {
       const float2 f = unpack2<DT>(v[r]);
-      v[r] = pack2<DT>(add_signed(f.x, x[o], 2 * r, op[o]), add_signed(f.y, x[o], 2 * r + 1, op[o]));
+      v[r] = pack2<DT>(add_signed_mul(f.x, x[o], 2 * r, op[o]), add_signed_mul(f.y, x[o], 2 * r + 1, op[o]));
     }
   }
 }
@@ -187,12 +199,12 @@ __global__ void __launch_bounds__(256) perturb_kernel(const __grid_constant__ Pe
 // ---------------------------------------------------------------------------
 template <uint8_t DT>
 __device__ __forceinline__ void pair_regs16(const uint32_t (&v)[8], const uint4& x, const PerturbOp& op,
-                                            uint32_t (&p)[8], uint32_t (&m)[8]) {
+                                            uint32_t (&p)[8], uint32_t (&m)[8]) {  // p may alias v
 #pragma unroll
   for (int r = 0; r < 8; ++r) {
     const float2 f = unpack2<DT>(v[r]);
-    const float d0 = __uint_as_float(op.nscale_bits ^ sign_bit(x, 2 * r, op.bit));
-    const float d1 = __uint_as_float(op.nscale_bits ^ sign_bit(x, 2 * r + 1, op.bit));
+    const float d0 = __uint_as_float(op.nscale_bits ^ sign_bit_mul(x, 2 * r, op));
+    const float d1 = __uint_as_float(op.nscale_bits ^ sign_bit_mul(x, 2 * r + 1, op));
     p[r] = pack2<DT>(__fadd_rn(f.x, d0), __fadd_rn(f.y, d1));
     m[r] = pack2<DT>(__fsub_rn(f.x, d0), __fsub_rn(f.y, d1));
   }
@@ -209,9 +221,9 @@ __device__ __forceinline__ void pair_run16(const uint16_t* s, uint16_t* pp, uint
     uint32_t vn[8];
     if (i + 1 < n) ld256(sn, vn);
     const uint4 x = block_bits(vb, op.ctr2, keys);
-    uint32_t p[8], m[8];
-    pair_regs16<DT>(v, x, op, p, m);
-    st256(pp, p);
+    uint32_t m[8];
+    pair_regs16<DT>(v, x, op, v, m);  // plus overwrites the loaded values
+    st256(pp, v);
     st256(mp, m);
     s = sn;
     pp += pstride;
@@ -238,7 +250,7 @@ __device__ __noinline__ void pair_block_other(const PairTable& tab, int t, uint3
   }
 }
 
-__global__ void __launch_bounds__(256, 4) perturb_pair_kernel(const __grid_constant__ PairParams P) {
+__global__ void __launch_bounds__(256) perturb_pair_kernel(const __grid_constant__ PairParams P) {
   const PairTable& tab = P.tab;
   const PerturbOp op = P.op;
   const uint32_t stride = gridDim.x * blockDim.x;
@@ -569,18 +581,13 @@ cudaError_t launch_update(const UpdateParams& p, int grid, cudaStream_t stream) 
   return cudaGetLastError();
 }
 
-cudaError_t perturb_blocks_per_sm(int* out) {
-  int m = 1 << 30;
-  const void* kernels[2] = {reinterpret_cast<const void*>(perturb_kernel<1>),
-                            reinterpret_cast<const void*>(perturb_kernel<2>)};
-  for (const void* k : kernels) {
-    int a = 0;
-    cudaError_t e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&a, k, kThreads, 0);
-    if (e != cudaSuccess) return e;
-    m = a < m ? a : m;
-  }
-  *out = m;
-  return cudaSuccess;
+cudaError_t perturb_blocks_per_sm(int nops, int* out) {
+  if (nops == 2) return cudaOccupancyMaxActiveBlocksPerMultiprocessor(out, perturb_kernel<2>, kThreads, 0);
+  return cudaOccupancyMaxActiveBlocksPerMultiprocessor(out, perturb_kernel<1>, kThreads, 0);
+}
+
+cudaError_t pair_blocks_per_sm(int* out) {
+  return cudaOccupancyMaxActiveBlocksPerMultiprocessor(out, perturb_pair_kernel, kThreads, 0);
 }
 
 cudaError_t update_blocks_per_sm(int groups, int packing, int* out) {
