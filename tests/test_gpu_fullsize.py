@@ -1,8 +1,9 @@
 """Parity at the full parameter-set sizes (OPT-1.3B/13B/30B- and Qwen3-8B-
-shaped), through the same ParamList / zo_perturb / zo_precondition /
-zo_update calls the benchmark times. The oracle recomputes sampled elements
-one by one (the generator is counter-based): every tensor's first and last 16
-elements plus 2^16 elements drawn uniformly over the whole set."""
+shaped), through the same ParamList / zo_perturb / zo_perturb2 /
+zo_precondition / zo_update(_ex) calls the benchmark times. The oracle
+recomputes sampled elements one by one (the generator is counter-based): every
+tensor's first and last 16 elements plus 2^16 elements drawn uniformly over
+the whole set."""
 import gc
 
 import numpy as np
@@ -14,7 +15,7 @@ from paper_2609_38095_gb300 import build as zo_build
 from paper_2609_38095_gb300 import workloads as W
 from paper_2609_38095_gb300 import zo
 
-from gpu_helpers import assert_update_close, gather, sample_positions
+from gpu_helpers import assert_update_close, bits_to_f64, gather, sample_positions
 
 pytestmark = pytest.mark.gpu
 
@@ -36,6 +37,10 @@ def test_fullsize_sampled_parity_packing8():
     """The 8-bit packing on the largest set (60 GB fp16, K = 256)."""
     with oracle.packing(8), zo.packing(8):
         run_fullsize("opt-30b")
+
+
+def bits_to_f32(bits, dt):
+    return bits_to_f64(bits, dt).astype(np.float32)
 
 
 def run_fullsize(key):
@@ -68,10 +73,23 @@ def run_fullsize(key):
         c_h = c.cpu().numpy()
         np.testing.assert_allclose(c_h, c_o, rtol=1e-6)
 
-        # fused K-probe update with lr = eps (tied, as in the paper)
-        zo.update(plist, seed, c, eps, status=st)
+        # two-op passes as the fused schedule launches them: probes in one
+        # group of 8 (one Philox call) and in two groups: bit-exact
+        f = f1
+        for (ka, sa, kb, sb) in ((k, -2 * eps, k - 1, eps), (K - 9, eps, K - 8, -eps)):
+            zo.perturb2(plist, seed, ka, sa, kb, sb)
+            bits_p2, f_next = gather(params, t_idx, i_idx)
+            mid = oracle.perturb_elements(ps.dtype, g, f, seed, ka, sa)
+            want_p2 = oracle.perturb_elements(ps.dtype, g, bits_to_f32(mid, ps.dtype), seed, kb, sb)
+            np.testing.assert_array_equal(bits_p2, want_p2, err_msg=f"perturb2 {ka},{kb}")
+            f = f_next
+
+        # fused K-probe update with lr = eps (tied, as in the paper), carrying a
+        # leading perturbation (the last restore) as the bench's schedule does
+        zo.update(plist, seed, c, eps, status=st, pre=(k, eps))
         bits2, _ = gather(params, t_idx, i_idx)
-        want2 = oracle.update_elements(ps.dtype, g, f1, seed, c_h, eps)
+        pre = bits_to_f32(oracle.perturb_elements(ps.dtype, g, f, seed, k, eps), ps.dtype)
+        want2 = oracle.update_elements(ps.dtype, g, pre, seed, c_h, eps)
         assert_update_close(bits2, want2, ps.dtype, c_h, eps, context=key)
         assert np.mean(bits2 == want2) > 0.95
     finally:

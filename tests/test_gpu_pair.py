@@ -176,13 +176,14 @@ def test_pair_schedule_step(K, packing_mode):
         assert_update_close(storage_bits(d), storage_bits(h), dt, c_h, eps, context="pair schedule")
 
 
-def test_pair_fullsize_sampled_opt13b():
-    """The OPT-13B-shaped set (25.7 GB, three copies on the device): sampled
-    elements of plus and minus against the oracle."""
-    ps = W.BY_KEY["opt-13b"]
+@pytest.mark.parametrize("key", ["opt-13b", "opt-30b"])
+def test_pair_fullsize_sampled(key):
+    """Full-size sets with three copies on the device (77 GB, 180 GB): sampled
+    elements of plus and minus against the oracle, theta untouched."""
+    ps = W.BY_KEY[key]
     free, _ = torch.cuda.mem_get_info()
-    if free < 3 * ps.d * ps.bytes_per_elem * 1.1:
-        pytest.skip("needs three copies of the OPT-13B-shaped set")
+    if free < 3 * ps.d * ps.bytes_per_elem * 1.05:
+        pytest.skip(f"needs three copies of the {key}-shaped set")
     params = W.allocate_params(ps)
     plus = [torch.empty_like(t) for t in params]
     minus = [torch.empty_like(t) for t in params]
