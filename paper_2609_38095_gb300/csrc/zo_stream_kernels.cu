@@ -1,6 +1,7 @@
 // zo_stream_kernels.cu -- the HBM-streaming kernels of the 1.5-SPSA step:
-// fused perturb (Algorithm 1, ApplyPackedPerturbation), fused K-probe update
-// (Sec. 4.2, Eqs. 5-6) and the debug views of a probe.
+// fused perturb (Algorithm 1, ApplyPackedPerturbation), the out-of-place pair
+// of perturbations, fused K-probe update (Sec. 4.2, Eqs. 5-6) and the debug
+// views of a probe.
 //
 // Work unit: one thread owns one 16-element Philox block at a time (grid-
 // stride over the virtual block space of the launch's tensor table). A block
