@@ -147,18 +147,67 @@ __device__ __forceinline__ void perturb_run16(uint16_t* p, uint32_t n, size_t ps
   }
 }
 
-// Grid-stride over the launch's blocks. While a thread's next blocks lie in
-// the full, aligned 16-bit region of its current tensor they go through
-// perturb_run16; any other block (fp32, a partial last block, an unaligned
-// tensor) is handled on its own.
+// Grid-stride over the launch's blocks, one block per iteration: the load of
+// the thread's next block (through the cursor, in whatever tensor it lies) is
+// issued before the current block is computed and stored. Every lane of a
+// warp runs the same number of iterations, whatever the tensor sizes.
 template <int NOPS>
-__global__ void __launch_bounds__(256) perturb_kernel(const __grid_constant__ PerturbParams P) {
-  if (P.status != nullptr && *P.status != 0) return;
-  PerturbOp op[2] = {P.op[0], P.op[1]};
-  if (P.coef != nullptr)
-    op[0].nscale_bits = __float_as_uint(__double2float_rn(P.coef_mul * P.coef[P.probe])) ^ 0x80000000u;
-  const bool same_ctr = op[1].ctr2 == op[0].ctr2;
+__device__ __forceinline__ void perturb_blocks(const PerturbParams& P, const PerturbOp (&op)[2], bool same_ctr) {
+  const TensorTable& tab = P.tab;
+  const uint32_t blk_total = tab.blk_total;
+  const uint32_t stride = gridDim.x * blockDim.x;
+  uint32_t b = blockIdx.x * blockDim.x + threadIdx.x;  // launch-relative; < 2^31 + stride never wraps
+  if (b >= blk_total) return;
+  Cursor c;
+  c.t = 0;
+  cursor_seek(tab, c, b);
+  int t = c.t;  // tensor and dtype of the current block
+  uint8_t dt = c.dt;
+  uint16_t* p = b < c.tfe ? c.tp + static_cast<size_t>(b - c.tb) * 16 : nullptr;
+  uint32_t v[8];
+  if (p != nullptr) ld256(p, v);
+  while (true) {
+    const uint32_t bn = b + stride;
+    uint16_t* pn = nullptr;
+    uint32_t vn[8];
+    if (bn < blk_total) {
+      if (bn >= c.te) cursor_seek(tab, c, bn);
+      pn = bn < c.tfe ? c.tp + static_cast<size_t>(bn - c.tb) * 16 : nullptr;
+      if (pn != nullptr) ld256(pn, vn);
+    }
+    const int64_t vb = tab.blk_base + b;  // virtual block: the Philox counter
+    uint4 x[2];
+    x[0] = block_bits(vb, op[0].ctr2, P.keys);
+    x[1] = x[0];
+    if (NOPS == 2 && !same_ctr) x[1] = block_bits(vb, op[1].ctr2, P.keys);
+    if (p != nullptr) {
+      if (dt == kBF16)
+        perturb_regs16<kBF16, NOPS>(v, x, op);
+      else
+        perturb_regs16<kF16, NOPS>(v, x, op);
+      st256(p, v);
+    } else {
+      perturb_block_other<NOPS>(tab, t, b, x[0], x[1], op[0], op[1]);
+    }
+    if (bn >= blk_total) break;
+    b = bn;
+    t = c.t;
+    dt = c.dt;
+    p = pn;
+#pragma unroll
+    for (int r = 0; r < 8; ++r) v[r] = vn[r];
+  }
+}
 
+// Grid-stride by runs: while a thread's next blocks lie in the full, aligned
+// 16-bit region of its current tensor they go through the tight loop of
+// perturb_run16; any other block (fp32, a partial last block, an unaligned
+// tensor) is handled on its own. Fewer instructions per block than
+// perturb_blocks, but the lanes of a warp leave a run up to one iteration
+// apart, which costs most where runs are short (tensors of a few blocks per
+// thread).
+template <int NOPS>
+__device__ __forceinline__ void perturb_runs(const PerturbParams& P, const PerturbOp (&op)[2], bool same_ctr) {
   const TensorTable& tab = P.tab;
   const uint32_t blk_total = tab.blk_total;
   const uint32_t stride = gridDim.x * blockDim.x;
@@ -190,6 +239,24 @@ __global__ void __launch_bounds__(256) perturb_kernel(const __grid_constant__ Pe
       b += stride;
     }
   }
+}
+
+// The single-op pass (zo_perturb) walks block by block; the two-op pass
+// (zo_perturb2), with twice the arithmetic per element, by runs (measured on
+// the benchmark sets: single-op per-block 4.99 ms against 5.56 ms by runs on
+// the Qwen3-8B-shaped set and equal elsewhere; two-op by runs 18.39 ms
+// against 20.04 ms per-block on the OPT-30B-shaped set).
+template <int NOPS>
+__global__ void __launch_bounds__(256) perturb_kernel(const __grid_constant__ PerturbParams P) {
+  if (P.status != nullptr && *P.status != 0) return;
+  PerturbOp op[2] = {P.op[0], P.op[1]};
+  if (P.coef != nullptr)
+    op[0].nscale_bits = __float_as_uint(__double2float_rn(P.coef_mul * P.coef[P.probe])) ^ 0x80000000u;
+  const bool same_ctr = op[1].ctr2 == op[0].ctr2;
+  if (NOPS == 1)
+    perturb_blocks<NOPS>(P, op, same_ctr);
+  else
+    perturb_runs<NOPS>(P, op, same_ctr);
 }
 
 // ---------------------------------------------------------------------------
