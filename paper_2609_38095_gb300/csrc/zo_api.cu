@@ -6,6 +6,7 @@
 #include <cstdio>
 #include <cstring>
 #include <mutex>
+#include <vector>
 
 #include <cuda_runtime.h>
 
@@ -67,14 +68,17 @@ zo::PerturbOp make_op(uint32_t k, float scale, int packing) {
   return op;
 }
 
-// Resident perturb blocks per SM, by kernel. The passes are HBM-bound and each
-// thread keeps two 32-byte loads in flight. The single-op pass streams fastest
-// with four 256-thread blocks per SM (3 -> 90.6 %, 4 -> 97.7 %, 5 -> 93.0 % of
-// the copy bandwidth on the 60 GB OPT-30B-shaped set); the two-op and the
-// out-of-place pair passes, with more arithmetic per element and 80
-// registers, with three (two-op: 93.2 % at four, 96.5 % at three).
-constexpr int kPerturbBlocksPerSm[2] = {4, 3};  // by number of operations
+// Resident perturb blocks per SM. The passes are HBM-bound and each thread
+// keeps two 32-byte loads in flight. The single-op pass streams fastest with
+// four 256-thread blocks per SM (3 -> 90.6 %, 4 -> 97.7 %, 5 -> 93.0 % of the
+// copy bandwidth on the 60 GB OPT-30B-shaped set), the out-of-place pair pass
+// with three. The two-op pass has three candidate (loop, blocks per SM)
+// configurations, timed on the caller's list (TwoOpTuner below).
+constexpr int kPerturbBlocksPerSm = 4;
 constexpr int kPairBlocksPerSm = 3;
+constexpr int kTwoOpCandidates = 3;
+constexpr int kTwoOpLoop[kTwoOpCandidates] = {zo::kLoopRuns, zo::kLoopRuns, zo::kLoopBlocks};
+constexpr int kTwoOpBlocksPerSm[kTwoOpCandidates] = {3, 4, 4};
 
 // The update is issue-bound; four waves of its blocks per SM keep more warps
 // eligible than one persistent wave (measured +3 % at K = 64 and 256).
@@ -83,7 +87,8 @@ constexpr int kUpdateWaves = 4;
 // Per-device launch facts, filled once per device.
 struct DeviceInfo {
   int sms = 0;
-  int perturb_bps[2] = {0, 0};            // perturb blocks per SM, single-op and two-op kernel
+  int perturb_bps = 0;                    // single-op perturb blocks per SM
+  int two_op_bps[kTwoOpCandidates] = {};  // two-op perturb blocks per SM, by candidate
   int pair_bps = 0;                       // perturb_pair blocks per SM
   int update_bps[2][zo::kMaxGroups + 1] = {};  // by packing (1, 8) and probe-group count
 };
@@ -103,11 +108,13 @@ int device_info(DeviceInfo** out) {
     e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
     if (e != cudaSuccess) return cuda_fail(e, "cudaDeviceGetAttribute");
     int bps = 0;
-    for (int nops = 1; nops <= 2; ++nops) {
-      e = zo::perturb_blocks_per_sm(nops, &bps);
-      if (e != cudaSuccess) return cuda_fail(e, "occupancy(perturb)");
-      const int cap = kPerturbBlocksPerSm[nops - 1];
-      d.perturb_bps[nops - 1] = bps < 1 ? 1 : (bps < cap ? bps : cap);
+    e = zo::perturb_blocks_per_sm(1, zo::kLoopBlocks, &bps);
+    if (e != cudaSuccess) return cuda_fail(e, "occupancy(perturb)");
+    d.perturb_bps = bps < 1 ? 1 : (bps < kPerturbBlocksPerSm ? bps : kPerturbBlocksPerSm);
+    for (int i = 0; i < kTwoOpCandidates; ++i) {
+      e = zo::perturb_blocks_per_sm(2, kTwoOpLoop[i], &bps);
+      if (e != cudaSuccess) return cuda_fail(e, "occupancy(perturb2)");
+      d.two_op_bps[i] = bps < 1 ? 1 : (bps < kTwoOpBlocksPerSm[i] ? bps : kTwoOpBlocksPerSm[i]);
     }
     e = zo::pair_blocks_per_sm(&bps);
     if (e != cudaSuccess) return cuda_fail(e, "occupancy(perturb_pair)");
@@ -184,18 +191,157 @@ int grid_for(int64_t blocks, int sms, int bps) {
   return static_cast<int>(g < 1 ? 1 : g);
 }
 
+// Choice of the two-op configuration per parameter list. All candidates give
+// the same bits; which is fastest depends on the tensor sizes (measured: runs
+// with 3 blocks per SM on the OPT-30B-shaped set, one block per iteration with
+// 4 on the Qwen3-8B-shaped one, runs with 4 on the OPT-1.3B-shaped one, the
+// spread between candidates from 1 % to 12 %). The first kTrials calls on a
+// list (keyed by its sizes, dtypes, alignments and device) run the candidates
+// in turn, kRounds times each, each call between two events on the caller's
+// stream; once all those events have completed (polled, never waited for),
+// later calls use the candidate with the shortest time. Calls made while the
+// stream is being captured into a graph, or before a decision, use
+// candidate 0.
+class TwoOpTuner {
+ public:
+  // Candidate for this call; *slot receives the trial index when the call's
+  // launches must be bracketed by that trial's events, else -1.
+  int pick(uint64_t key, cudaStream_t s, int* slot) {
+    *slot = -1;
+    cudaStreamCaptureStatus cap = cudaStreamCaptureStatusNone;
+    if (cudaStreamIsCapturing(s, &cap) != cudaSuccess || cap != cudaStreamCaptureStatusNone) {
+      cudaGetLastError();
+      return 0;
+    }
+    std::lock_guard<std::mutex> lock(mu_);
+    Entry* e = find(key);
+    if (e == nullptr) return 0;
+    if (e->chosen >= 0) return e->chosen;
+    decide(*e);
+    if (e->chosen >= 0) return e->chosen;
+    if (e->next < kTrials) {
+      *slot = e->next++;
+      return *slot % kTwoOpCandidates;
+    }
+    return 0;
+  }
+
+  void record(uint64_t key, int slot, int which, cudaStream_t s) {
+    std::lock_guard<std::mutex> lock(mu_);
+    Entry* e = find(key);
+    if (e == nullptr || e->ev[slot][which] == nullptr) return;
+    if (cudaEventRecord(e->ev[slot][which], s) != cudaSuccess) {
+      cudaGetLastError();
+      e->failed = true;
+    }
+  }
+
+ private:
+  static constexpr int kRounds = 3;
+  static constexpr int kTrials = kRounds * kTwoOpCandidates;
+
+  struct Entry {
+    uint64_t key = 0;
+    int chosen = -1;
+    int next = 0;  // next trial; trial i runs candidate i % kTwoOpCandidates
+    bool failed = false;
+    cudaEvent_t ev[kTrials][2] = {};
+  };
+
+  // Entry of `key`, created with its events on first use (nullptr when the
+  // table is full or events cannot be created: then candidate 0 is used).
+  Entry* find(uint64_t key) {
+    for (Entry& e : entries_)
+      if (e.key == key) return &e;
+    if (entries_.size() >= kMaxEntries) return nullptr;
+    Entry e;
+    e.key = key;
+    for (auto& pair : e.ev)
+      for (cudaEvent_t& ev : pair)
+        if (cudaEventCreate(&ev) != cudaSuccess) {
+          cudaGetLastError();
+          e.chosen = 0;
+        }
+    entries_.push_back(e);
+    return &entries_.back();
+  }
+
+  void decide(Entry& e) {
+    if (e.failed) {
+      e.chosen = 0;
+      return;
+    }
+    if (e.next < kTrials) return;
+    float best[kTwoOpCandidates];
+    for (int i = 0; i < kTrials; ++i) {
+      if (cudaEventQuery(e.ev[i][1]) != cudaSuccess) {  // not done yet (or failed): decide later
+        cudaGetLastError();
+        return;
+      }
+      float ms = 0.0f;
+      if (cudaEventElapsedTime(&ms, e.ev[i][0], e.ev[i][1]) != cudaSuccess) {
+        cudaGetLastError();
+        e.chosen = 0;
+        return;
+      }
+      const int c = i % kTwoOpCandidates;
+      if (i < kTwoOpCandidates || ms < best[c]) best[c] = ms;  // shortest of its rounds
+    }
+    int arg = 0;
+    for (int c = 1; c < kTwoOpCandidates; ++c)
+      if (best[c] < best[arg]) arg = c;
+    e.chosen = arg;
+  }
+
+  static constexpr size_t kMaxEntries = 64;
+  std::mutex mu_;
+  std::vector<Entry> entries_;
+};
+TwoOpTuner g_two_op_tuner;
+
+// FNV-1a over what decides the two-op pass's speed: device, sizes, dtypes,
+// 32-byte alignment.
+uint64_t list_key(const zo_tensor* params, int32_t n) {
+  uint64_t h = 0xcbf29ce484222325ull;
+  auto mix = [&h](uint64_t v) {
+    for (int i = 0; i < 8; ++i) {
+      h ^= (v >> (8 * i)) & 0xFFu;
+      h *= 0x100000001b3ull;
+    }
+  };
+  int dev = 0;
+  cudaGetDevice(&dev);
+  mix(static_cast<uint64_t>(dev));
+  mix(static_cast<uint64_t>(n));
+  for (int32_t t = 0; t < n; ++t) {
+    mix(static_cast<uint64_t>(params[t].numel));
+    mix(static_cast<uint64_t>(params[t].dtype) | (reinterpret_cast<uintptr_t>(params[t].ptr) % 32 == 0 ? 0x100u : 0u));
+  }
+  return h;
+}
+
 // Enqueue perturb launches over the whole parameter list.
 int run_perturb(const zo_tensor* params, int32_t n, PerturbParams& pp, DeviceInfo* d, cudaStream_t s) {
+  int loop = zo::kLoopBlocks, bps = d->perturb_bps, slot = -1;
+  uint64_t key = 0;
+  if (pp.nops == 2) {
+    key = list_key(params, n);
+    const int c = g_two_op_tuner.pick(key, s, &slot);
+    loop = kTwoOpLoop[c];
+    bps = d->two_op_bps[c];
+  }
+  if (slot >= 0) g_two_op_tuner.record(key, slot, 0, s);
   int64_t blk = 0;
   for (int32_t t0 = 0; t0 < n;) {
     int64_t nb = 0;
     t0 = fill_table(pp.tab, params, t0, n, blk, &nb);
     if (nb > 0) {
-      cudaError_t e = zo::launch_perturb(pp, grid_for(nb, d->sms, d->perturb_bps[pp.nops == 2 ? 1 : 0]), s);
+      cudaError_t e = zo::launch_perturb(pp, grid_for(nb, d->sms, bps), loop, s);
       if (e != cudaSuccess) return cuda_fail(e, "perturb_kernel");
     }
     blk += nb;
   }
+  if (slot >= 0) g_two_op_tuner.record(key, slot, 1, s);
   return ZO_OK;
 }
 

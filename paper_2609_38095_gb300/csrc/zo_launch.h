@@ -16,11 +16,11 @@ constexpr int kMaxLossPartials = 2048;
 constexpr int kStaticLossPartials = 4096;   // fixed scratch of the allocation-free loss (32 KB)
 constexpr int64_t kStaticLossSlice = 2048;  // elements per partial in that variant
 
-cudaError_t launch_perturb(const PerturbParams& p, int grid, cudaStream_t stream);
+cudaError_t launch_perturb(const PerturbParams& p, int grid, int loop, cudaStream_t stream);
 cudaError_t launch_perturb_pair(const PairParams& p, int grid, cudaStream_t stream);
 cudaError_t launch_update(const UpdateParams& p, int grid, cudaStream_t stream);
 size_t update_smem_bytes(int groups);
-cudaError_t perturb_blocks_per_sm(int nops, int* out);
+cudaError_t perturb_blocks_per_sm(int nops, int loop, int* out);
 cudaError_t pair_blocks_per_sm(int* out);
 cudaError_t update_blocks_per_sm(int groups, int packing, int* out);
 cudaError_t launch_probe_bytes(const RoundKeys& keys, uint32_t ctr2, uint32_t bit, int64_t first, int64_t n,

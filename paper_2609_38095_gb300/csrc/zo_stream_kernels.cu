@@ -87,8 +87,10 @@ __device__ __forceinline__ void cursor_seek(const TensorTable& tab, Cursor& c, u
   c.tp = reinterpret_cast<uint16_t*>(tab.ptr[c.t]);
 }
 
-// Any other block: fp32, a partial last block, or an unaligned tensor.
-template <int NOPS>
+// Any other block: fp32, a partial last block, or an unaligned tensor. One
+// instantiation per calling loop (LOOP): ptxas 13.0 crashes when two kernels
+// share this non-inlined function.
+template <int NOPS, int LOOP>
 __device__ __noinline__ void perturb_block_other(const TensorTable& tab, int t, uint32_t b, uint4 x0, uint4 x1,
                                                  PerturbOp op0, PerturbOp op1) {
   const int64_t e0 = static_cast<int64_t>(b - tensor_blk_begin(tab, t)) * 16;
@@ -187,7 +189,7 @@ __device__ __forceinline__ void perturb_blocks(const PerturbParams& P, const Per
         perturb_regs16<kF16, NOPS>(v, x, op);
       st256(p, v);
     } else {
-      perturb_block_other<NOPS>(tab, t, b, x[0], x[1], op[0], op[1]);
+      perturb_block_other<NOPS, kLoopBlocks>(tab, t, b, x[0], x[1], op[0], op[1]);
     }
     if (bn >= blk_total) break;
     b = bn;
@@ -235,25 +237,27 @@ __device__ __forceinline__ void perturb_runs(const PerturbParams& P, const Pertu
       x[0] = block_bits(vb, op[0].ctr2, P.keys);
       x[1] = x[0];
       if (NOPS == 2 && !same_ctr) x[1] = block_bits(vb, op[1].ctr2, P.keys);
-      perturb_block_other<NOPS>(tab, c.t, b, x[0], x[1], op[0], op[1]);
+      perturb_block_other<NOPS, kLoopRuns>(tab, c.t, b, x[0], x[1], op[0], op[1]);
       b += stride;
     }
   }
 }
 
-// The single-op pass (zo_perturb) walks block by block; the two-op pass
-// (zo_perturb2), with twice the arithmetic per element, by runs (measured on
-// the benchmark sets: single-op per-block 4.99 ms against 5.56 ms by runs on
-// the Qwen3-8B-shaped set and equal elsewhere; two-op by runs 18.39 ms
-// against 20.04 ms per-block on the OPT-30B-shaped set).
-template <int NOPS>
+// LOOP selects perturb_blocks (kLoopBlocks) or perturb_runs (kLoopRuns). The
+// single-op pass (zo_perturb) always walks block by block (4.99 ms against
+// 5.56 ms by runs on the Qwen3-8B-shaped set, equal elsewhere). For the two-op
+// pass (zo_perturb2) the faster loop and grid depend on the parameter list
+// (OPT-30B-shaped: runs with 3 blocks per SM 18.54 ms, per block with 4
+// 18.72 ms; Qwen3-8B-shaped: 5.96 ms against 5.27 ms), so the host times the
+// candidates on the caller's own list; all give the same bits.
+template <int NOPS, int LOOP>
 __global__ void __launch_bounds__(256) perturb_kernel(const __grid_constant__ PerturbParams P) {
   if (P.status != nullptr && *P.status != 0) return;
   PerturbOp op[2] = {P.op[0], P.op[1]};
   if (P.coef != nullptr)
     op[0].nscale_bits = __float_as_uint(__double2float_rn(P.coef_mul * P.coef[P.probe])) ^ 0x80000000u;
   const bool same_ctr = op[1].ctr2 == op[0].ctr2;
-  if (NOPS == 1)
+  if (LOOP == kLoopBlocks)
     perturb_blocks<NOPS>(P, op, same_ctr);
   else
     perturb_runs<NOPS>(P, op, same_ctr);
@@ -278,30 +282,6 @@ __device__ __forceinline__ void pair_regs16(const uint32_t (&v)[8], const uint4&
   }
 }
 
-// n full, 32-byte aligned 16-bit blocks, pipelined like perturb_run16.
-template <uint8_t DT>
-__device__ __forceinline__ void pair_run16(const uint16_t* s, uint16_t* pp, uint16_t* mp, uint32_t n, size_t pstride,
-                                           int64_t vb, uint32_t stride, const PerturbOp& op, const RoundKeys& keys) {
-  uint32_t v[8];
-  ld256(s, v);
-  for (uint32_t i = 0; i < n; ++i) {
-    const uint16_t* sn = s + pstride;
-    uint32_t vn[8];
-    if (i + 1 < n) ld256(sn, vn);
-    const uint4 x = block_bits(vb, op.ctr2, keys);
-    uint32_t m[8];
-    pair_regs16<DT>(v, x, op, v, m);  // plus overwrites the loaded values
-    st256(pp, v);
-    st256(mp, m);
-    s = sn;
-    pp += pstride;
-    mp += pstride;
-    vb += stride;
-#pragma unroll
-    for (int r = 0; r < 8; ++r) v[r] = vn[r];
-  }
-}
-
 __device__ __noinline__ void pair_block_other(const PairTable& tab, int t, uint32_t b, uint4 x, PerturbOp op) {
   const uint32_t tb = t == 0 ? 0u : tab.blk_end[t - 1];
   const int64_t e0 = static_cast<int64_t>(b - tb) * 16;
@@ -318,40 +298,70 @@ __device__ __noinline__ void pair_block_other(const PairTable& tab, int t, uint3
   }
 }
 
+// A thread's position in a pair table (as Cursor for TensorTable).
+struct PairCursor {
+  int t;
+  uint32_t tb, te, tfe;  // first block, one past the last, one past the last full vector block (else tb)
+  uint8_t dt;
+};
+
+__device__ __forceinline__ void pair_seek(const PairTable& tab, PairCursor& c, uint32_t b) {
+  while (b >= tab.blk_end[c.t]) ++c.t;
+  c.tb = c.t == 0 ? 0u : tab.blk_end[c.t - 1];
+  c.te = tab.blk_end[c.t];
+  c.dt = tab.flags[c.t] & kDtypeMask;
+  c.tfe = ((tab.flags[c.t] & kVec32) && c.dt != kF32) ? c.te - (tab.last[c.t] < 16 ? 1u : 0u) : c.tb;
+}
+
+// Grid-stride one block per iteration, the next block's theta load issued
+// before the current block is computed (the single-op perturb's loop).
 __global__ void __launch_bounds__(256) perturb_pair_kernel(const __grid_constant__ PairParams P) {
   const PairTable& tab = P.tab;
   const PerturbOp op = P.op;
   const uint32_t stride = gridDim.x * blockDim.x;
-  uint32_t b = blockIdx.x * blockDim.x + threadIdx.x;  // < 2^31 + stride: never wraps
-  int t = 0;
-  uint32_t tb = 0, te = 0, tfe = 0;
-  uint8_t dt = 0;
-  bool seeked = false;
-  while (b < tab.blk_total) {
-    if (!seeked || b >= te) {
-      while (b >= tab.blk_end[t]) ++t;
-      tb = t == 0 ? 0u : tab.blk_end[t - 1];
-      te = tab.blk_end[t];
-      dt = tab.flags[t] & kDtypeMask;
-      tfe = ((tab.flags[t] & kVec32) && dt != kF32) ? te - (tab.last[t] < 16 ? 1u : 0u) : tb;  // full blocks
-      seeked = true;
+  uint32_t b = blockIdx.x * blockDim.x + threadIdx.x;
+  if (b >= tab.blk_total) return;
+  PairCursor c;
+  c.t = 0;
+  pair_seek(tab, c, b);
+  int t = c.t;
+  uint8_t dt = c.dt;
+  size_t off = static_cast<size_t>(b - c.tb) * 16;
+  bool vec = b < c.tfe;
+  uint32_t v[8];
+  if (vec) ld256(reinterpret_cast<const uint16_t*>(tab.src[t]) + off, v);
+  while (true) {
+    const uint32_t bn = b + stride;
+    bool vecn = false;
+    size_t offn = 0;
+    uint32_t vn[8];
+    if (bn < tab.blk_total) {
+      if (bn >= c.te) pair_seek(tab, c, bn);
+      vecn = bn < c.tfe;
+      offn = static_cast<size_t>(bn - c.tb) * 16;
+      if (vecn) ld256(reinterpret_cast<const uint16_t*>(tab.src[c.t]) + offn, vn);
     }
     const int64_t vb = tab.blk_base + b;
-    if (b < tfe) {
-      const uint32_t n = (tfe - b + stride - 1) / stride;
-      const size_t off = static_cast<size_t>(b - tb) * 16, pstride = static_cast<size_t>(stride) * 16;
-      const uint16_t* s = reinterpret_cast<const uint16_t*>(tab.src[t]) + off;
-      uint16_t* pp = reinterpret_cast<uint16_t*>(tab.plus[t]) + off;
-      uint16_t* mp = reinterpret_cast<uint16_t*>(tab.minus[t]) + off;
+    const uint4 x = block_bits(vb, op.ctr2, P.keys);
+    if (vec) {
+      uint32_t m[8];
       if (dt == kBF16)
-        pair_run16<kBF16>(s, pp, mp, n, pstride, vb, stride, op, P.keys);
+        pair_regs16<kBF16>(v, x, op, v, m);
       else
-        pair_run16<kF16>(s, pp, mp, n, pstride, vb, stride, op, P.keys);
-      b += n * stride;
+        pair_regs16<kF16>(v, x, op, v, m);
+      st256(reinterpret_cast<uint16_t*>(tab.plus[t]) + off, v);
+      st256(reinterpret_cast<uint16_t*>(tab.minus[t]) + off, m);
     } else {
-      pair_block_other(tab, t, b, block_bits(vb, op.ctr2, P.keys), op);
-      b += stride;
+      pair_block_other(tab, t, b, x, op);
     }
+    if (bn >= tab.blk_total) break;
+    b = bn;
+    t = c.t;
+    dt = c.dt;
+    off = offn;
+    vec = vecn;
+#pragma unroll
+    for (int r = 0; r < 8; ++r) v[r] = vn[r];
   }
 }
 
@@ -621,11 +631,13 @@ __global__ void probe_signs_kernel(RoundKeys keys, uint32_t q, uint32_t j, int64
 
 namespace zo {
 
-cudaError_t launch_perturb(const PerturbParams& p, int grid, cudaStream_t stream) {
-  if (p.nops == 2)
-    perturb_kernel<2><<<grid, kThreads, 0, stream>>>(p);
+cudaError_t launch_perturb(const PerturbParams& p, int grid, int loop, cudaStream_t stream) {
+  if (p.nops == 1)
+    perturb_kernel<1, kLoopBlocks><<<grid, kThreads, 0, stream>>>(p);
+  else if (loop == kLoopRuns)
+    perturb_kernel<2, kLoopRuns><<<grid, kThreads, 0, stream>>>(p);
   else
-    perturb_kernel<1><<<grid, kThreads, 0, stream>>>(p);
+    perturb_kernel<2, kLoopBlocks><<<grid, kThreads, 0, stream>>>(p);
   return cudaGetLastError();
 }
 
@@ -649,9 +661,12 @@ cudaError_t launch_update(const UpdateParams& p, int grid, cudaStream_t stream) 
   return cudaGetLastError();
 }
 
-cudaError_t perturb_blocks_per_sm(int nops, int* out) {
-  if (nops == 2) return cudaOccupancyMaxActiveBlocksPerMultiprocessor(out, perturb_kernel<2>, kThreads, 0);
-  return cudaOccupancyMaxActiveBlocksPerMultiprocessor(out, perturb_kernel<1>, kThreads, 0);
+cudaError_t perturb_blocks_per_sm(int nops, int loop, int* out) {
+  if (nops == 1)
+    return cudaOccupancyMaxActiveBlocksPerMultiprocessor(out, perturb_kernel<1, kLoopBlocks>, kThreads, 0);
+  if (loop == kLoopRuns)
+    return cudaOccupancyMaxActiveBlocksPerMultiprocessor(out, perturb_kernel<2, kLoopRuns>, kThreads, 0);
+  return cudaOccupancyMaxActiveBlocksPerMultiprocessor(out, perturb_kernel<2, kLoopBlocks>, kThreads, 0);
 }
 
 cudaError_t pair_blocks_per_sm(int* out) {

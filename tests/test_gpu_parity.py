@@ -379,6 +379,72 @@ def test_perturb2_is_two_perturbs(a, b, packing_mode):
     assert_storage_equal(dev, host)
 
 
+def test_perturb2_every_tuned_configuration():
+    """zo_perturb2 times its candidate configurations (three rounds) on the
+    first calls for a parameter list, then keeps the fastest: 12 calls on one
+    list run every candidate and the chosen one, each bit-exact with the
+    oracle."""
+    rng = np.random.default_rng(606)
+    numels = [int(x) for x in rng.integers(1, 70000, 40)] + [4096 * 300, 17]
+    dtypes = [DTS[int(x)] for x in rng.integers(0, 3, len(numels))]
+    host, dev = make_list(numels, dtypes, seed=606)
+    dts = [TORCH_TO_DT[d] for d in dtypes]
+    plist = zo.ParamList(dev)
+    seed = W.step_seed(606)
+    for call in range(12):
+        a, b = 2 * call + 7, 2 * call + 8
+        zo.perturb2(plist, seed, a, 1e-3, b, -1e-3)
+        oracle.perturb(host, dts, seed, a, 1e-3)
+        oracle.perturb(host, dts, seed, b, -1e-3)
+        torch.cuda.synchronize()
+        assert_storage_equal(dev, host, f"call {call}")
+
+
+def test_fused_step_in_a_cuda_graph():
+    """Every call of a fused step only enqueues work on the current stream and
+    allocates nothing, so a whole step can be captured into a CUDA graph and
+    replayed: the replay matches the oracle's Algorithm 1 order."""
+    K, eps = 4, 1e-3
+    host, dev = make_list(MIXED_NUMELS, MIXED_DTYPES, seed=808)
+    dts = [TORCH_TO_DT[d] for d in MIXED_DTYPES]
+    plist = zo.ParamList(dev)
+    seed = W.step_seed(808)
+    L = torch.tensor(W.synthetic_losses(K, 808), device="cuda")
+    c = torch.empty(K, dtype=torch.float64, device="cuda")
+    st = torch.zeros(1, dtype=torch.int32, device="cuda")
+    scratch = zo.ParamList([t.clone() for t in dev])           # warm-up outside the capture
+    zo.perturb(scratch, seed, 0, eps)
+    zo.perturb2(scratch, seed, 0, eps, 1, eps)
+    zo.precondition(L, eps, out=(c, st))
+    zo.update(scratch, seed, c, eps, status=st, pre=(K - 1, eps))
+    torch.cuda.synchronize()
+    g = torch.cuda.CUDAGraph()
+    s = torch.cuda.Stream()
+    s.wait_stream(torch.cuda.current_stream())
+    with torch.cuda.stream(s):
+        with torch.cuda.graph(g, stream=s):
+            zo.perturb(plist, seed, 0, eps)
+            for k in range(K):
+                zo.perturb(plist, seed, k, -2 * eps)
+                if k + 1 < K:
+                    zo.perturb2(plist, seed, k, eps, k + 1, eps)
+            zo.precondition(L, eps, out=(c, st))
+            zo.update(plist, seed, c, eps, status=st, pre=(K - 1, eps))
+    torch.cuda.synchronize()
+    assert_storage_equal(dev, host, "capture must not execute")
+    g.replay()
+    torch.cuda.synchronize()
+    for k in range(K):
+        for sc in (eps, -2 * eps, eps):
+            oracle.perturb(host, dts, seed, k, sc)
+    rc, c_o, _, _ = oracle.precondition(W.synthetic_losses(K, 808), eps)
+    assert rc == oracle.OK and int(st.item()) == zo.ZO_OK
+    np.testing.assert_allclose(c.cpu().numpy(), c_o, rtol=1e-12)
+    oracle.update(host, dts, seed, c.cpu().numpy(), eps)
+    for d, h, dt in zip(dev, host, dts):
+        assert_update_close(storage_bits(d), storage_bits(h), dt, c.cpu().numpy(), eps, context="graph replay")
+
+
 @pytest.mark.parametrize("K", [1, 9, 64])
 def test_update_with_leading_perturb(K, packing_mode):
     host, dev = make_list(MIXED_NUMELS, MIXED_DTYPES, seed=K + 5)
