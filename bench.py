@@ -493,10 +493,11 @@ def run_zo(args):
         dom_kernel, dom_ms, dom_launches = "perturb_pair_kernel", pair_ms, K
         traffic = committed_traffic("perturb_pair_kernel", args.config)
     elif n2 > 0 and n2 * perturb2_ms > n1 * perturb_ms:
-        dom_kernel, dom_ms, dom_launches = "perturb_kernel<2>", perturb2_ms, n2
+        dom_kernel, dom_ms, dom_launches = ("perturb_kernel<2, *> (zo_perturb2, configuration tuned per list)",
+                                            perturb2_ms, n2)
         traffic = committed_traffic("perturb2_kernel", args.config)
     else:
-        dom_kernel, dom_ms, dom_launches = "perturb_kernel<1>", perturb_ms, n1
+        dom_kernel, dom_ms, dom_launches = "perturb_kernel<1, 0> (zo_perturb)", perturb_ms, n1
         traffic = committed_traffic("perturb_kernel", args.config)
     dom_bytes = pair_bytes if pair else perturb_bytes
     # algorithmic HBM bytes of one step: every pass reads and writes theta once,
