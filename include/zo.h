@@ -131,6 +131,12 @@ int zo_perturb(const zo_tensor* params, int32_t n_tensors, uint64_t seed, uint32
  * forward pass runs between probe k's restore (+eps) and probe k+1's first
  * perturbation (+eps), so a step can apply them together:
  * zo_perturb2(k, +eps, k + 1, +eps). Errors as zo_perturb.
+ * Launch configuration: the first nine calls on a parameter list (identified
+ * by device, sizes, dtypes and 32-byte alignments) each run one of three
+ * loop / grid configurations between two CUDA events recorded on `stream`;
+ * later calls use the fastest. The results never depend on the
+ * configuration. Calls made while `stream` is being captured into a CUDA
+ * graph use the first configuration and record no event.
  * ------------------------------------------------------------------------- */
 int zo_perturb2(const zo_tensor* params, int32_t n_tensors, uint64_t seed, uint32_t probe_a, float scale_a,
                 uint32_t probe_b, float scale_b, void* stream);
