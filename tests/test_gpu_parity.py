@@ -445,6 +445,58 @@ def test_fused_step_in_a_cuda_graph():
         assert_update_close(storage_bits(d), storage_bits(h), dt, c.cpu().numpy(), eps, context="graph replay")
 
 
+def test_concurrent_host_threads_on_their_own_streams():
+    """Two host threads, each with its own parameter list and stream, call the
+    library at the same time (the binding releases the GIL in every call):
+    the per-thread launch state, the device table and the two-op tuner keep
+    them apart, and each list matches the oracle."""
+    import threading
+    K, eps, iters = 6, 1e-3, 20
+    jobs = []
+    for j in range(2):
+        numels = [4096 * 40 + 16 * j, 333, 70000 + j]
+        dtypes = [torch.bfloat16, torch.float16, torch.float32]
+        host, dev = make_list(numels, dtypes, seed=900 + j)
+        jobs.append({"host": host, "dev": dev, "dts": [TORCH_TO_DT[d] for d in dtypes],
+                     "seed": W.step_seed(900 + j), "stream": torch.cuda.Stream(), "err": None})
+
+    def run(job):
+        try:
+            with torch.cuda.stream(job["stream"]):
+                plist = zo.ParamList(job["dev"])
+                seed = job["seed"]
+                for it in range(iters):
+                    zo.perturb(plist, seed, it, eps)
+                    zo.perturb2(plist, seed, it, -eps, it + 1, 2 * eps)
+                L = torch.tensor(W.synthetic_losses(K, 3), device="cuda")
+                c, st = zo.precondition(L, eps)
+                zo.update(plist, seed, c, eps, status=st, pre=(3, eps))
+                job["c"] = c
+            job["stream"].synchronize()
+        except Exception as e:  # reported by the main thread
+            job["err"] = e
+
+    threads = [threading.Thread(target=run, args=(j,)) for j in jobs]
+    for t in threads:
+        t.start()
+    for t in threads:
+        t.join()
+    for job in jobs:
+        assert job["err"] is None, job["err"]
+        host, dts, seed = job["host"], job["dts"], job["seed"]
+        for it in range(iters):
+            oracle.perturb(host, dts, seed, it, eps)
+            oracle.perturb(host, dts, seed, it, -eps)
+            oracle.perturb(host, dts, seed, it + 1, 2 * eps)
+        oracle.perturb(host, dts, seed, 3, eps)
+        c = job["c"].cpu().numpy()
+        rc, c_o, _, _ = oracle.precondition(W.synthetic_losses(K, 3), eps)
+        np.testing.assert_allclose(c, c_o, rtol=1e-12)
+        oracle.update(host, dts, seed, c, eps)
+        for d, h, dt in zip(job["dev"], host, dts):
+            assert_update_close(storage_bits(d), storage_bits(h), dt, c, eps, context="concurrent threads")
+
+
 @pytest.mark.parametrize("K", [1, 9, 64])
 def test_update_with_leading_perturb(K, packing_mode):
     host, dev = make_list(MIXED_NUMELS, MIXED_DTYPES, seed=K + 5)
