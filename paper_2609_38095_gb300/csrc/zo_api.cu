@@ -336,7 +336,10 @@ int run_perturb(const zo_tensor* params, int32_t n, PerturbParams& pp, DeviceInf
     int64_t nb = 0;
     t0 = fill_table(pp.tab, params, t0, n, blk, &nb);
     if (nb > 0) {
-      cudaError_t e = zo::launch_perturb(pp, grid_for(nb, d->sms, bps), loop, s);
+      bool f32v = false;  // aligned fp32 tensors in this launch: pipelined fp32 path (single-op kernel)
+      for (int i = 0; i < pp.tab.n && !f32v; ++i)
+        f32v = (pp.tab.flags[i] & zo::kVec32) && (pp.tab.flags[i] & zo::kDtypeMask) == zo::kF32;
+      cudaError_t e = zo::launch_perturb(pp, grid_for(nb, d->sms, bps), loop, f32v, s);
       if (e != cudaSuccess) return cuda_fail(e, "perturb_kernel");
     }
     blk += nb;

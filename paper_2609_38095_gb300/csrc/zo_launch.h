@@ -16,7 +16,8 @@ constexpr int kMaxLossPartials = 2048;
 constexpr int kStaticLossPartials = 4096;   // fixed scratch of the allocation-free loss (32 KB)
 constexpr int64_t kStaticLossSlice = 2048;  // elements per partial in that variant
 
-cudaError_t launch_perturb(const PerturbParams& p, int grid, int loop, cudaStream_t stream);
+// f32v: the launch holds 32-byte aligned fp32 tensors (single-op kernel only).
+cudaError_t launch_perturb(const PerturbParams& p, int grid, int loop, bool f32v, cudaStream_t stream);
 cudaError_t launch_perturb_pair(const PairParams& p, int grid, cudaStream_t stream);
 cudaError_t launch_update(const UpdateParams& p, int grid, cudaStream_t stream);
 size_t update_smem_bytes(int groups);

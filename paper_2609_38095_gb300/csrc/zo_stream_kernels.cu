@@ -71,7 +71,8 @@ struct Cursor {
   int t;           // tensor index
   uint32_t tb;     // first launch block of tensor t
   uint32_t te;     // one past its last block
-  uint32_t tfe;    // one past its last full block when it takes the pipelined path, else tb
+  uint32_t tfe;    // one past its last full block when it takes the pipelined 16-bit path, else tb
+  uint32_t tfe32;  // the same for the pipelined fp32 path of the single-op loop
   uint16_t* tp;    // base pointer
   uint8_t dt;      // storage dtype
 };
@@ -83,14 +84,16 @@ __device__ __forceinline__ void cursor_seek(const TensorTable& tab, Cursor& c, u
   const uint8_t fl = tab.flags[c.t];
   c.dt = fl & kDtypeMask;
   // pipelined path: full, 32-byte aligned blocks of a 16-bit tensor
-  c.tfe = ((fl & kVec32) && c.dt != kF32) ? c.tb + static_cast<uint32_t>(tab.numel[c.t] / 16) : c.tb;
+  const uint32_t full = c.tb + static_cast<uint32_t>(tab.numel[c.t] / 16);
+  c.tfe = ((fl & kVec32) && c.dt != kF32) ? full : c.tb;
+  c.tfe32 = ((fl & kVec32) && c.dt == kF32) ? full : c.tb;
   c.tp = reinterpret_cast<uint16_t*>(tab.ptr[c.t]);
 }
 
 // Any other block: fp32, a partial last block, or an unaligned tensor. One
-// instantiation per calling loop (LOOP): ptxas 13.0 crashes when two kernels
+// instantiation per calling kernel (TAG): ptxas 13.0 crashes when two kernels
 // share this non-inlined function.
-template <int NOPS, int LOOP>
+template <int NOPS, int TAG>
 __device__ __noinline__ void perturb_block_other(const TensorTable& tab, int t, uint32_t b, uint4 x0, uint4 x1,
                                                  PerturbOp op0, PerturbOp op1) {
   const int64_t e0 = static_cast<int64_t>(b - tensor_blk_begin(tab, t)) * 16;
@@ -152,8 +155,25 @@ __device__ __forceinline__ void perturb_run16(uint16_t* p, uint32_t n, size_t ps
 // Grid-stride over the launch's blocks, one block per iteration: the load of
 // the thread's next block (through the cursor, in whatever tensor it lies) is
 // issued before the current block is computed and stored. Every lane of a
-// warp runs the same number of iterations, whatever the tensor sizes.
-template <int NOPS>
+// warp runs the same number of iterations, whatever the tensor sizes. With
+// F32V (single-op launches that contain aligned fp32 tensors) full fp32
+// blocks are pipelined too, as two 256-bit halves; otherwise they go to
+// perturb_block_other, and the 16-bit path keeps its smaller register set.
+enum : int { kBlockOther = 0, kBlock16 = 1, kBlock32 = 2 };
+
+template <bool F32V>
+__device__ __forceinline__ int block_kind(const Cursor& c, uint32_t b) {
+  if (b < c.tfe) return kBlock16;
+  if (F32V && b < c.tfe32) return kBlock32;
+  return kBlockOther;
+}
+
+__device__ __forceinline__ void* block_addr(const Cursor& c, uint32_t b, int kind) {
+  const size_t bytes = kind == kBlock32 ? 64 : 32;
+  return reinterpret_cast<char*>(c.tp) + static_cast<size_t>(b - c.tb) * bytes;
+}
+
+template <int NOPS, bool F32V>
 __device__ __forceinline__ void perturb_blocks(const PerturbParams& P, const PerturbOp (&op)[2], bool same_ctr) {
   const TensorTable& tab = P.tab;
   const uint32_t blk_total = tab.blk_total;
@@ -165,39 +185,56 @@ __device__ __forceinline__ void perturb_blocks(const PerturbParams& P, const Per
   cursor_seek(tab, c, b);
   int t = c.t;  // tensor and dtype of the current block
   uint8_t dt = c.dt;
-  uint16_t* p = b < c.tfe ? c.tp + static_cast<size_t>(b - c.tb) * 16 : nullptr;
-  uint32_t v[8];
-  if (p != nullptr) ld256(p, v);
+  int kind = block_kind<F32V>(c, b);
+  void* p = block_addr(c, b, kind);
+  uint32_t v[8], w[8];  // the block (16-bit), or its two halves (fp32)
+  if (kind != kBlockOther) ld256(p, v);
+  if (kind == kBlock32) ld256(static_cast<char*>(p) + 32, w);
   while (true) {
     const uint32_t bn = b + stride;
-    uint16_t* pn = nullptr;
-    uint32_t vn[8];
+    int kindn = kBlockOther;
+    void* pn = nullptr;
+    uint32_t vn[8], wn[8];
     if (bn < blk_total) {
       if (bn >= c.te) cursor_seek(tab, c, bn);
-      pn = bn < c.tfe ? c.tp + static_cast<size_t>(bn - c.tb) * 16 : nullptr;
-      if (pn != nullptr) ld256(pn, vn);
+      kindn = block_kind<F32V>(c, bn);
+      pn = block_addr(c, bn, kindn);
+      if (kindn != kBlockOther) ld256(pn, vn);
+      if (kindn == kBlock32) ld256(static_cast<char*>(pn) + 32, wn);
     }
     const int64_t vb = tab.blk_base + b;  // virtual block: the Philox counter
     uint4 x[2];
     x[0] = block_bits(vb, op[0].ctr2, P.keys);
     x[1] = x[0];
     if (NOPS == 2 && !same_ctr) x[1] = block_bits(vb, op[1].ctr2, P.keys);
-    if (p != nullptr) {
+    if (kind == kBlock16) {
       if (dt == kBF16)
         perturb_regs16<kBF16, NOPS>(v, x, op);
       else
         perturb_regs16<kF16, NOPS>(v, x, op);
       st256(p, v);
+    } else if (F32V && kind == kBlock32) {
+#pragma unroll
+      for (int r = 0; r < 8; ++r) {
+        v[r] = __float_as_uint(add_signed_mul(__uint_as_float(v[r]), x[0], r, op[0]));
+        w[r] = __float_as_uint(add_signed_mul(__uint_as_float(w[r]), x[0], 8 + r, op[0]));
+      }
+      st256(p, v);
+      st256(static_cast<char*>(p) + 32, w);
     } else {
-      perturb_block_other<NOPS, kLoopBlocks>(tab, t, b, x[0], x[1], op[0], op[1]);
+      perturb_block_other<NOPS, F32V ? 2 : kLoopBlocks>(tab, t, b, x[0], x[1], op[0], op[1]);
     }
     if (bn >= blk_total) break;
     b = bn;
     t = c.t;
     dt = c.dt;
+    kind = kindn;
     p = pn;
 #pragma unroll
-    for (int r = 0; r < 8; ++r) v[r] = vn[r];
+    for (int r = 0; r < 8; ++r) {
+      v[r] = vn[r];
+      w[r] = wn[r];
+    }
   }
 }
 
@@ -250,7 +287,7 @@ __device__ __forceinline__ void perturb_runs(const PerturbParams& P, const Pertu
 // (OPT-30B-shaped: runs with 3 blocks per SM 18.54 ms, per block with 4
 // 18.72 ms; Qwen3-8B-shaped: 5.96 ms against 5.27 ms), so the host times the
 // candidates on the caller's own list; all give the same bits.
-template <int NOPS, int LOOP>
+template <int NOPS, int LOOP, bool F32V = false>
 __global__ void __launch_bounds__(256) perturb_kernel(const __grid_constant__ PerturbParams P) {
   if (P.status != nullptr && *P.status != 0) return;
   PerturbOp op[2] = {P.op[0], P.op[1]};
@@ -258,7 +295,7 @@ __global__ void __launch_bounds__(256) perturb_kernel(const __grid_constant__ Pe
     op[0].nscale_bits = __float_as_uint(__double2float_rn(P.coef_mul * P.coef[P.probe])) ^ 0x80000000u;
   const bool same_ctr = op[1].ctr2 == op[0].ctr2;
   if (LOOP == kLoopBlocks)
-    perturb_blocks<NOPS>(P, op, same_ctr);
+    perturb_blocks<NOPS, F32V>(P, op, same_ctr);
   else
     perturb_runs<NOPS>(P, op, same_ctr);
 }
@@ -631,8 +668,10 @@ __global__ void probe_signs_kernel(RoundKeys keys, uint32_t q, uint32_t j, int64
 
 namespace zo {
 
-cudaError_t launch_perturb(const PerturbParams& p, int grid, int loop, cudaStream_t stream) {
-  if (p.nops == 1)
+cudaError_t launch_perturb(const PerturbParams& p, int grid, int loop, bool f32v, cudaStream_t stream) {
+  if (p.nops == 1 && f32v)
+    perturb_kernel<1, kLoopBlocks, true><<<grid, kThreads, 0, stream>>>(p);
+  else if (p.nops == 1)
     perturb_kernel<1, kLoopBlocks><<<grid, kThreads, 0, stream>>>(p);
   else if (loop == kLoopRuns)
     perturb_kernel<2, kLoopRuns><<<grid, kThreads, 0, stream>>>(p);
