@@ -115,6 +115,17 @@ __device__ __noinline__ void perturb_block_other(const TensorTable& tab, int t, 
       }
       st256(p + 8 * half, v);
     }
+  } else if (cnt == 16 && dt != kF32) {  // a full block of an unaligned 16-bit tensor
+    uint16_t* p = static_cast<uint16_t*>(base) + e0;
+    uint32_t v[8];
+    ld16x16(p, v);
+    const uint4 x[2] = {x0, x1};
+    const PerturbOp op[2] = {op0, op1};
+    if (dt == kBF16)
+      perturb_regs16<kBF16, NOPS>(v, x, op);
+    else
+      perturb_regs16<kF16, NOPS>(v, x, op);
+    st16x16(p, v);
   } else {
     for (int i = 0; i < cnt; ++i) {
       float th = add_signed(load_elem(base, dt, e0 + i), x0, i, op0);
@@ -327,6 +338,17 @@ __device__ __noinline__ void pair_block_other(const PairTable& tab, int t, uint3
   const void* src = reinterpret_cast<const void*>(tab.src[t]);
   void* pl = reinterpret_cast<void*>(tab.plus[t]);
   void* mi = reinterpret_cast<void*>(tab.minus[t]);
+  if (cnt == 16 && dt != kF32) {  // a full block with an unaligned pointer among the three
+    uint32_t v[8], m[8];
+    ld16x16(static_cast<const uint16_t*>(src) + e0, v);
+    if (dt == kBF16)
+      pair_regs16<kBF16>(v, x, op, v, m);
+    else
+      pair_regs16<kF16>(v, x, op, v, m);
+    st16x16(static_cast<uint16_t*>(pl) + e0, v);
+    st16x16(static_cast<uint16_t*>(mi) + e0, m);
+    return;
+  }
   for (int i = 0; i < cnt; ++i) {
     const float th = load_elem(src, dt, e0 + i);
     const float d = __uint_as_float(op.nscale_bits ^ sign_bit(x, i, op.bit));
@@ -508,10 +530,12 @@ __device__ __forceinline__ uint32_t pre_regs16(uint32_t v, const uint4& xp, int 
   return pack2<DT>(add_signed(f.x, xp, 2 * r, op), add_signed(f.y, xp, 2 * r + 1, op));
 }
 
-// One full, 32-byte aligned block: theta (16-bit) is loaded before the probe
-// loop so the load overlaps the arithmetic; the leading perturbation, when
-// present, is applied and rounded to storage before the probe sum is added.
-template <int PACK, uint8_t DT>
+// One full block: theta (16-bit) is loaded before the probe loop so the load
+// overlaps the arithmetic; the leading perturbation, when present, is applied
+// and rounded to storage before the probe sum is added. ALIGNED: the block is
+// 32-byte aligned (256-bit accesses), else only 2-byte aligned (16-bit
+// storage only).
+template <int PACK, uint8_t DT, bool ALIGNED = true>
 __device__ __forceinline__ void update_block_vec(void* base, int64_t e0, int64_t b, const UpdateParams& P,
                                                  uint32_t lut_base, bool do_sum) {
   float acc[16];
@@ -538,7 +562,10 @@ __device__ __forceinline__ void update_block_vec(void* base, int64_t e0, int64_t
   } else {
     uint16_t* p = static_cast<uint16_t*>(base) + e0;
     uint32_t v[8];
-    ld256(p, v);
+    if (ALIGNED)
+      ld256(p, v);
+    else
+      ld16x16(p, v);
     if (do_sum) accumulate_any<PACK>(acc, b, P, lut_base);
     uint4 xp = make_uint4(0u, 0u, 0u, 0u);
     if (P.has_pre) xp = block_bits(b, P.pre.ctr2, P.keys);
@@ -550,7 +577,10 @@ __device__ __forceinline__ void update_block_vec(void* base, int64_t e0, int64_t
         v[r] = pack2<DT>(__fadd_rn(f.x, acc[2 * r]), __fadd_rn(f.y, acc[2 * r + 1]));
       }
     }
-    st256(p, v);
+    if (ALIGNED)
+      st256(p, v);
+    else
+      st16x16(p, v);
   }
 }
 
@@ -598,6 +628,10 @@ __global__ void __launch_bounds__(256) update_kernel(const __grid_constant__ Upd
         update_block_vec<PACK, kF16>(base, e0, b, P, lut_base, do_sum);
       else
         update_block_vec<PACK, kF32>(base, e0, b, P, lut_base, do_sum);
+    } else if (cnt == 16 && dt == kBF16) {  // full blocks of unaligned 16-bit tensors
+      update_block_vec<PACK, kBF16, false>(base, e0, b, P, lut_base, do_sum);
+    } else if (cnt == 16 && dt == kF16) {
+      update_block_vec<PACK, kF16, false>(base, e0, b, P, lut_base, do_sum);
     } else {
       float acc[16];
 #pragma unroll

@@ -110,6 +110,30 @@ def test_perturb_unaligned_views(dtype, offset):
     np.testing.assert_array_equal(after[offset + n:], base_host[offset + n:])
 
 
+@pytest.mark.parametrize("dtype", [torch.bfloat16, torch.float16])
+@pytest.mark.parametrize("offset", [1, 2, 8])
+def test_update_unaligned_views(dtype, offset):
+    """Fused update (with a leading perturbation) on views 2-, 4- and
+    16-byte aligned: within the update tolerance of the oracle, nothing
+    outside the view written."""
+    rng = np.random.default_rng(40 + offset)
+    n = 4096 * 3 + 21
+    dt = TORCH_TO_DT[dtype]
+    base_host = W.random_storage(rng, n + offset + 40, dt)
+    base = to_torch(base_host, dtype)
+    view = base[offset:offset + n]
+    host = [base_host[offset:offset + n].copy()]
+    K, seed, lr = 24, W.step_seed(41), 1e-3
+    c_np = rng.normal(0, 20, K)
+    zo.update([view], seed, torch.tensor(c_np, device="cuda"), lr, pre=(K - 1, 1e-3))
+    oracle.perturb(host, [dt], seed, K - 1, 1e-3)
+    oracle.update(host, [dt], seed, c_np, lr)
+    assert_update_close(storage_bits(view), storage_bits(host[0]), dt, c_np, lr, context=f"offset {offset}")
+    after = storage_np(base)
+    np.testing.assert_array_equal(after[:offset], base_host[:offset])
+    np.testing.assert_array_equal(after[offset + n:], base_host[offset + n:])
+
+
 def test_perturb_many_tensors_split_launches(packing_mode):
     """More tensors than one launch's table holds (1024)."""
     rng = np.random.default_rng(12)
