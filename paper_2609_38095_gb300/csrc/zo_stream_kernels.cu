@@ -530,12 +530,10 @@ __device__ __forceinline__ uint32_t pre_regs16(uint32_t v, const uint4& xp, int 
   return pack2<DT>(add_signed(f.x, xp, 2 * r, op), add_signed(f.y, xp, 2 * r + 1, op));
 }
 
-// One full block: theta (16-bit) is loaded before the probe loop so the load
-// overlaps the arithmetic; the leading perturbation, when present, is applied
-// and rounded to storage before the probe sum is added. ALIGNED: the block is
-// 32-byte aligned (256-bit accesses), else only 2-byte aligned (16-bit
-// storage only).
-template <int PACK, uint8_t DT, bool ALIGNED = true>
+// One full, 32-byte aligned block: theta (16-bit) is loaded before the probe
+// loop so the load overlaps the arithmetic; the leading perturbation, when
+// present, is applied and rounded to storage before the probe sum is added.
+template <int PACK, uint8_t DT>
 __device__ __forceinline__ void update_block_vec(void* base, int64_t e0, int64_t b, const UpdateParams& P,
                                                  uint32_t lut_base, bool do_sum) {
   float acc[16];
@@ -562,10 +560,7 @@ __device__ __forceinline__ void update_block_vec(void* base, int64_t e0, int64_t
   } else {
     uint16_t* p = static_cast<uint16_t*>(base) + e0;
     uint32_t v[8];
-    if (ALIGNED)
-      ld256(p, v);
-    else
-      ld16x16(p, v);
+    ld256(p, v);
     if (do_sum) accumulate_any<PACK>(acc, b, P, lut_base);
     uint4 xp = make_uint4(0u, 0u, 0u, 0u);
     if (P.has_pre) xp = block_bits(b, P.pre.ctr2, P.keys);
@@ -577,10 +572,7 @@ __device__ __forceinline__ void update_block_vec(void* base, int64_t e0, int64_t
         v[r] = pack2<DT>(__fadd_rn(f.x, acc[2 * r]), __fadd_rn(f.y, acc[2 * r + 1]));
       }
     }
-    if (ALIGNED)
-      st256(p, v);
-    else
-      st16x16(p, v);
+    st256(p, v);
   }
 }
 
@@ -628,10 +620,6 @@ __global__ void __launch_bounds__(256) update_kernel(const __grid_constant__ Upd
         update_block_vec<PACK, kF16>(base, e0, b, P, lut_base, do_sum);
       else
         update_block_vec<PACK, kF32>(base, e0, b, P, lut_base, do_sum);
-    } else if (cnt == 16 && dt == kBF16) {  // full blocks of unaligned 16-bit tensors
-      update_block_vec<PACK, kBF16, false>(base, e0, b, P, lut_base, do_sum);
-    } else if (cnt == 16 && dt == kF16) {
-      update_block_vec<PACK, kF16, false>(base, e0, b, P, lut_base, do_sum);
     } else {
       float acc[16];
 #pragma unroll
