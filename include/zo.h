@@ -17,8 +17,11 @@
  * ---------------------------------------
  * Memory. Every array argument is DEVICE memory of the current CUDA device,
  * owned by the caller, except the zo_tensor descriptor array itself (host
- * memory, read during the call only). The library allocates nothing: the
- * tensor table travels inside the kernel launch parameters.
+ * memory, read during the call only). The library allocates no device
+ * memory: the tensor table travels inside the kernel launch parameters. Its
+ * only CUDA objects are the timing events of zo_perturb2's launch
+ * configuration choice (18 per parameter list, at most 64 lists, kept until
+ * the process exits).
  *
  * Streams. `stream` is a cudaStream_t (NULL = legacy default stream). Every
  * call only enqueues work on it and returns; results are visible to later
