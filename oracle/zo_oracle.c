@@ -19,11 +19,15 @@
  *                        uniformity / independence statistics.
  *   probe_bit/bytes      pinned: brute force unpack rule (Appendix F layout),
  *                        statistics.
- *   dtype conversions    pinned: numpy float16 and torch bfloat16 casts.
+ *   dtype conversions    pinned: numpy float16 and torch bfloat16 casts, on
+ *                        edge cases and (property tests) arbitrary fp32 bits.
  *   perturb              pinned: brute force, exact-grid restore identity,
- *                        restore drift bound.
+ *                        restore drift bound, numpy fp32 addition (property).
  *   precondition         pinned: worked value of Sec. 6 (|c|=1e8, alpha=0.1),
- *                        alpha=0 / alpha=1 special cases, quadratic closed form.
+ *                        alpha=0 / alpha=1 special cases, quadratic closed form,
+ *                        invariants on arbitrary triples (property); relative
+ *                        curvature: alpha=1 closed form, equal magnitudes,
+ *                        scale invariance, degenerate cases.
  *   update               pinned: K=1 equals perturb, fp64 brute force sum,
  *                        update(c) then update(-c), quadratic gradient identity.
  *   update_sequential    pinned: equals K perturb passes.
