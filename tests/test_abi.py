@@ -173,3 +173,34 @@ def test_tensor_block_limit(L):
     big = (1 << 31) * 16
     assert L.zo_perturb(tensors((FAKE, big, 1)), 1, 1, 0, 1e-3, None) == zo.ZO_ERR_ARG
     assert L.zo_perturb(tensors((FAKE, big - 16 + 1, 1)), 1, 1, 0, 1e-3, None) == zo.ZO_ERR_ARG
+
+
+def test_header_is_plain_c_and_links_from_c(tmp_path, L):
+    """include/zo.h compiles as C99 with warnings as errors, and a C program
+    links against libzo.so and calls it (host-only entry points: no GPU)."""
+    import shutil
+    import subprocess
+    gcc = shutil.which("gcc")
+    if gcc is None:
+        pytest.skip("gcc not available")
+    src = tmp_path / "use_zo.c"
+    src.write_text(
+        "#include <stdio.h>\n#include <string.h>\n#include \"zo.h\"\n"
+        "int main(void) {\n"
+        "  zo_tensor t = {0, 0, ZO_BF16, 0};\n"
+        "  if (zo_version() != 10300) return 1;\n"
+        "  if (strncmp(zo_status_string(ZO_ERR_ARG), \"ZO_ERR_ARG\", 10) != 0) return 2;\n"
+        "  if (zo_perturb(&t, -1, 1, 0, 1e-3f, NULL) != ZO_ERR_ARG) return 3;\n"
+        "  if (zo_set_packing(3) != ZO_ERR_ARG) return 4;\n"
+        "  if (zo_quadratic_loss_workspace_size(1 << 20) <= 0) return 5;\n"
+        "  puts(\"ok\");\n  return 0;\n}\n")
+    lib = zo.LIB_PATH
+    exe = tmp_path / "use_zo"
+    inc = os.path.join(ROOT, "include")
+    cmd = [gcc, "-std=c99", "-Wall", "-Wextra", "-Werror", "-I", inc, str(src), "-o", str(exe),
+           "-L", os.path.dirname(lib), "-l:" + os.path.basename(lib), "-Wl,-rpath," + os.path.dirname(lib)]
+    r = subprocess.run(cmd, capture_output=True, text=True)
+    assert r.returncode == 0, r.stderr
+    r = subprocess.run([str(exe)], capture_output=True, text=True, timeout=60)
+    assert r.returncode == 0 and r.stdout.strip() == "ok", (r.returncode, r.stdout, r.stderr)
+
