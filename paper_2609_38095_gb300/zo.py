@@ -231,6 +231,8 @@ def precondition(losses, eps: float, alpha: float = 0.1, lambda_reg: float = 1.0
         status = torch.empty(1, dtype=torch.int32, device=dev)
     else:
         c, status = out
+        if c.numel() < K or status.numel() < 1:
+            raise ValueError("out must be (c with at least K elements, status with at least one)")
     w = curv = None
     if with_weights:
         w = torch.empty(K, dtype=torch.float64, device=dev)
@@ -301,10 +303,12 @@ def quadratic_loss(theta, a, out=None, workspace=None):
         out = torch.empty(1, dtype=torch.float64, device=dev)
     if workspace is None:
         workspace = torch.empty(quadratic_loss_workspace_size(n), dtype=torch.uint8, device=dev)
+    if out.numel() < 1:
+        raise ValueError("out must hold one float64")
     with torch.cuda.device(dev):
         rc = _lib().zo_quadratic_loss(_dev_ptr(theta, torch.float32, "theta"), _dev_ptr(a, torch.float32, "a"), n,
-                                      ctypes.c_void_p(out.data_ptr()), ctypes.c_void_p(workspace.data_ptr()),
-                                      workspace.numel(), _stream(dev))
+                                      _dev_ptr(out, torch.float64, "out"), _dev_ptr(workspace, what="workspace"),
+                                      workspace.numel() * workspace.element_size(), _stream(dev))
     _check("zo_quadratic_loss", rc)
     return out
 
@@ -319,8 +323,10 @@ def quadratic_loss_static(theta, a, out=None):
     dev = theta.device
     if out is None:
         out = torch.empty(1, dtype=torch.float64, device=dev)
+    if out.numel() < 1:
+        raise ValueError("out must hold one float64")
     with torch.cuda.device(dev):
         rc = _lib().zo_quadratic_loss_static(_dev_ptr(theta, torch.float32, "theta"), _dev_ptr(a, torch.float32, "a"),
-                                             n, ctypes.c_void_p(out.data_ptr()), _stream(dev))
+                                             n, _dev_ptr(out, torch.float64, "out"), _stream(dev))
     _check("zo_quadratic_loss_static", rc)
     return out

@@ -610,3 +610,22 @@ def test_fused_calls_on_split_launches_and_unaligned_views(packing_mode):
     zo.update(dev2, seed, c, 1e-3)
     for x, y in zip(dev, dev2):
         assert torch.equal(x.view(torch.uint8), y.view(torch.uint8)) if x.numel() else True
+
+
+def test_binding_rejects_bad_output_buffers():
+    """The binding checks what the library will write: the coefficient and
+    status buffers' sizes and dtypes, the loss output's dtype."""
+    L = torch.tensor(W.synthetic_losses(8, 0), device="cuda")
+    with pytest.raises(ValueError):
+        zo.precondition(L, 1e-3, out=(torch.empty(7, dtype=torch.float64, device="cuda"),
+                                      torch.empty(1, dtype=torch.int32, device="cuda")))
+    with pytest.raises(TypeError):
+        zo.precondition(L, 1e-3, out=(torch.empty(8, dtype=torch.float32, device="cuda"),
+                                      torch.empty(1, dtype=torch.int32, device="cuda")))
+    th = torch.zeros(100, device="cuda")
+    with pytest.raises(TypeError):
+        zo.quadratic_loss(th, th, out=torch.empty(1, dtype=torch.float32, device="cuda"))
+    with pytest.raises(ValueError):
+        zo.quadratic_loss_static(th, th, out=torch.empty(0, dtype=torch.float64, device="cuda"))
+    with pytest.raises(TypeError):
+        zo.update([th], 1, torch.zeros(4, dtype=torch.float32, device="cuda"), 1e-3)
