@@ -299,15 +299,15 @@ class TwoOpTuner {
 };
 TwoOpTuner g_two_op_tuner;
 
-// FNV-1a over what decides the two-op pass's speed: device, sizes, dtypes,
-// 32-byte alignment.
+// Hash of what decides the two-op pass's speed: device, sizes, dtypes,
+// 32-byte alignment (an FNV-style multiply-xor per 64-bit word, then a final
+// avalanche; a collision only shares a tuning decision).
 uint64_t list_key(const zo_tensor* params, int32_t n) {
   uint64_t h = 0xcbf29ce484222325ull;
   auto mix = [&h](uint64_t v) {
-    for (int i = 0; i < 8; ++i) {
-      h ^= (v >> (8 * i)) & 0xFFu;
-      h *= 0x100000001b3ull;
-    }
+    h ^= v;
+    h *= 0x100000001b3ull;
+    h ^= h >> 29;
   };
   int dev = 0;
   cudaGetDevice(&dev);
@@ -317,6 +317,9 @@ uint64_t list_key(const zo_tensor* params, int32_t n) {
     mix(static_cast<uint64_t>(params[t].numel));
     mix(static_cast<uint64_t>(params[t].dtype) | (reinterpret_cast<uintptr_t>(params[t].ptr) % 32 == 0 ? 0x100u : 0u));
   }
+  h ^= h >> 33;
+  h *= 0xff51afd7ed558ccdull;
+  h ^= h >> 33;
   return h;
 }
 
