@@ -38,9 +38,11 @@
  * same order and with the same sizes, must be given to every call of a step:
  * the probe is a function of the position of each element in that list.
  * Tensors may mix dtypes. numel may be 0 and at most 16 * (2^31 - 1) - 1
- * (ZO_ERR_ARG beyond). ptr must be aligned to its element size; 32-byte
- * alignment selects the vectorised path, anything else the element-wise path
- * (same results).
+ * (ZO_ERR_ARG beyond). ptr must be aligned to its element size. Any such
+ * alignment gives the same results; a tensor whose ptr is not 32-byte aligned
+ * is streamed in 32-byte aligned chunks by a second kernel of the same call
+ * (zo_perturb, zo_perturb2, zo_update_sequential) or with narrower accesses
+ * (zo_perturb_pair, zo_update).
  *
  * Probes. z_k is Rademacher, one bit per parameter per probe (Sec. 2, Sec. 4.3
  * "Bit-Packed perturbations"; unpack rule of Appendix F: bit 1 -> +1, bit 0 ->

@@ -90,6 +90,7 @@ struct DeviceInfo {
   int perturb_bps = 0;                    // single-op perturb blocks per SM
   int two_op_bps[kTwoOpCandidates] = {};  // two-op perturb blocks per SM, by candidate
   int pair_bps = 0;                       // perturb_pair blocks per SM
+  int shift_bps[2][3] = {};               // perturb_shift blocks per SM, by operation count and dtype
   int update_bps[2][zo::kMaxGroups + 1] = {};  // by packing (1, 8) and probe-group count
 };
 constexpr int kMaxDevices = 64;
@@ -119,6 +120,13 @@ int device_info(DeviceInfo** out) {
     e = zo::pair_blocks_per_sm(&bps);
     if (e != cudaSuccess) return cuda_fail(e, "occupancy(perturb_pair)");
     d.pair_bps = bps < 1 ? 1 : (bps < kPairBlocksPerSm ? bps : kPairBlocksPerSm);
+    for (int nops = 1; nops <= 2; ++nops) {
+      for (uint8_t dt = 0; dt < 3; ++dt) {
+        e = zo::shift_blocks_per_sm(nops, dt, &bps);
+        if (e != cudaSuccess) return cuda_fail(e, "occupancy(perturb_shift)");
+        d.shift_bps[nops - 1][dt] = bps < 1 ? 1 : bps;
+      }
+    }
     d.sms = sms;
   }
   *out = &d;
@@ -324,6 +332,43 @@ uint64_t list_key(const zo_tensor* params, int32_t n) {
 }
 
 // Enqueue perturb launches over the whole parameter list.
+// Tensors of a perturb launch that are not 32-byte aligned go to
+// perturb_shift_kernel: flag them (kShift). Returns a bit mask of their
+// storage types; *main_work tells whether any other tensor has elements.
+unsigned mark_shift(zo::TensorTable& tab, bool* main_work) {
+  unsigned types = 0;
+  *main_work = false;
+  for (int i = 0; i < tab.n; ++i) {
+    if (tab.numel[i] == 0) continue;
+    if (tab.flags[i] & zo::kVec32) {
+      *main_work = true;
+    } else {
+      tab.flags[i] |= zo::kShift;
+      types |= 1u << (tab.flags[i] & zo::kDtypeMask);
+    }
+  }
+  return types;
+}
+
+// grp_end over the flagged tensors of storage type dt (the others own no
+// group). Returns the number of groups.
+uint32_t shift_groups(const zo::TensorTable& tab, uint8_t dt, uint32_t* grp_end) {
+  uint32_t groups = 0;
+  for (int i = 0; i < tab.n; ++i) {
+    const uint8_t fl = tab.flags[i];
+    if ((fl & zo::kShift) && (fl & zo::kDtypeMask) == dt) {
+      const uint32_t esz = dt == zo::kF32 ? 4 : 2;
+      const int64_t a = static_cast<int64_t>(tab.ptr[i] % 32) / esz;  // 1..15: pointers are element-aligned
+      const int64_t chunks = (tab.numel[i] + a + 15) / 16;
+      groups += static_cast<uint32_t>((chunks + zo::kShiftGroup - 1) / zo::kShiftGroup);
+    }
+    grp_end[i] = groups;
+  }
+  return groups;
+}
+
+thread_local zo::ShiftParams tl_shift;
+
 int run_perturb(const zo_tensor* params, int32_t n, PerturbParams& pp, DeviceInfo* d, cudaStream_t s) {
   int loop = zo::kLoopBlocks, bps = d->perturb_bps, slot = -1;
   uint64_t key = 0;
@@ -339,11 +384,25 @@ int run_perturb(const zo_tensor* params, int32_t n, PerturbParams& pp, DeviceInf
     int64_t nb = 0;
     t0 = fill_table(pp.tab, params, t0, n, blk, &nb);
     if (nb > 0) {
+      bool main_work = false;
+      const unsigned shift_types = mark_shift(pp.tab, &main_work);
       bool f32v = false;  // aligned fp32 tensors in this launch: pipelined fp32 path (single-op kernel)
       for (int i = 0; i < pp.tab.n && !f32v; ++i)
         f32v = (pp.tab.flags[i] & zo::kVec32) && (pp.tab.flags[i] & zo::kDtypeMask) == zo::kF32;
-      cudaError_t e = zo::launch_perturb(pp, grid_for(nb, d->sms, bps), loop, f32v, s);
-      if (e != cudaSuccess) return cuda_fail(e, "perturb_kernel");
+      if (main_work) {
+        cudaError_t e = zo::launch_perturb(pp, grid_for(nb, d->sms, bps), loop, f32v, s);
+        if (e != cudaSuccess) return cuda_fail(e, "perturb_kernel");
+      }
+      if (shift_types) tl_shift.p = pp;
+      for (uint8_t dt = 0; dt < 3; ++dt) {
+        if (!(shift_types & (1u << dt))) continue;
+        const uint32_t groups = shift_groups(pp.tab, dt, tl_shift.grp_end);
+        tl_shift.grp_total = groups;
+        const int64_t want = (static_cast<int64_t>(groups) * 32 + zo::kThreads - 1) / zo::kThreads;
+        const int64_t cap = static_cast<int64_t>(d->sms) * d->shift_bps[pp.nops - 1][dt];
+        cudaError_t e = zo::launch_perturb_shift(tl_shift, dt, static_cast<int>(want < cap ? want : cap), s);
+        if (e != cudaSuccess) return cuda_fail(e, "perturb_shift_kernel");
+      }
     }
     blk += nb;
   }

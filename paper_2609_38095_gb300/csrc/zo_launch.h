@@ -18,10 +18,13 @@ constexpr int64_t kStaticLossSlice = 2048;  // elements per partial in that vari
 
 // f32v: the launch holds 32-byte aligned fp32 tensors (single-op kernel only).
 cudaError_t launch_perturb(const PerturbParams& p, int grid, int loop, bool f32v, cudaStream_t stream);
+// dt: the storage type of the tensors grp_end counts (one launch per type).
+cudaError_t launch_perturb_shift(const ShiftParams& p, uint8_t dt, int grid, cudaStream_t stream);
 cudaError_t launch_perturb_pair(const PairParams& p, int grid, cudaStream_t stream);
 cudaError_t launch_update(const UpdateParams& p, int grid, cudaStream_t stream);
 size_t update_smem_bytes(int groups);
 cudaError_t perturb_blocks_per_sm(int nops, int loop, int* out);
+cudaError_t shift_blocks_per_sm(int nops, uint8_t dt, int* out);
 cudaError_t pair_blocks_per_sm(int* out);
 cudaError_t update_blocks_per_sm(int groups, int packing, int* out);
 cudaError_t launch_probe_bytes(const RoundKeys& keys, uint32_t ctr2, uint32_t bit, int64_t first, int64_t n,

@@ -6,8 +6,11 @@
 // Work unit: one thread owns one 16-element Philox block at a time (grid-
 // stride over the virtual block space of the launch's tensor table). A block
 // of a 16-bit tensor is 32 bytes: one 256-bit load and one 256-bit store when
-// the tensor is 32-byte aligned, element-wise access otherwise or for a
-// tensor's last, partial block.
+// the tensor is 32-byte aligned, element-wise access for a tensor's last,
+// partial block. The perturbation passes hand tensors that are not 32-byte
+// aligned to perturb_shift_kernel, which works on aligned 32-byte chunks
+// straddling two blocks; the pair and update kernels take narrower accesses
+// for them.
 #include "zo_device.cuh"
 
 namespace zo {
@@ -92,13 +95,16 @@ __device__ __forceinline__ void cursor_seek(const TensorTable& tab, Cursor& c, u
 
 // Any other block: fp32, a partial last block, or an unaligned tensor. One
 // instantiation per calling kernel (TAG): ptxas 13.0 crashes when two kernels
-// share this non-inlined function.
+// share this non-inlined function. Blocks of tensors flagged kShift are
+// perturb_shift_kernel's and left alone (the loops above stay exactly as
+// they are for the aligned tensors).
 template <int NOPS, int TAG>
 __device__ __noinline__ void perturb_block_other(const TensorTable& tab, int t, uint32_t b, uint4 x0, uint4 x1,
                                                  PerturbOp op0, PerturbOp op1) {
+  const uint8_t fl = tab.flags[t];
+  if (fl & kShift) return;
   const int64_t e0 = static_cast<int64_t>(b - tensor_blk_begin(tab, t)) * 16;
   const int64_t cnt = min(static_cast<int64_t>(16), tab.numel[t] - e0);
-  const uint8_t fl = tab.flags[t];
   const uint8_t dt = fl & kDtypeMask;
   void* base = reinterpret_cast<void*>(tab.ptr[t]);
   if (cnt == 16 && (fl & kVec32) && dt == kF32) {
@@ -309,6 +315,148 @@ __global__ void __launch_bounds__(256) perturb_kernel(const __grid_constant__ Pe
     perturb_blocks<NOPS, F32V>(P, op, same_ctr);
   else
     perturb_runs<NOPS>(P, op, same_ctr);
+}
+
+// ---------------------------------------------------------------------------
+// Unaligned tensors (kShift): the same perturbation over 32-byte aligned
+// chunks instead of Philox blocks, so every full chunk moves with 256-bit
+// accesses whatever the tensor's offset. Chunk c (elements 16c - a ..
+// 16c - a + 15) draws its signs from bytes 16 - a .. 31 - a of the 32 bytes
+// Philox(c - 1) ++ Philox(c). In a warp, lane l generates block
+// c0 - 1 + l and works on chunk c0 - 1 + l with the block below taken from
+// lane l - 1 by a shuffle: 32 Philox calls per 31 chunks, lane 0 only
+// generates. Chunks that cross the tensor's ends go element by element.
+// ---------------------------------------------------------------------------
+// Bytes b .. b + 15 (b = 0..15) of the 32-byte string lo ++ hi.
+__device__ __forceinline__ uint4 window16(const uint4& lo, const uint4& hi, uint32_t b) {
+  const uint32_t w[8] = {lo.x, lo.y, lo.z, lo.w, hi.x, hi.y, hi.z, hi.w};
+  uint32_t e[6], d[5];
+#pragma unroll
+  for (int i = 0; i < 6; ++i) e[i] = (b & 8u) ? w[i + 2] : w[i];  // move by two words
+#pragma unroll
+  for (int i = 0; i < 5; ++i) d[i] = (b & 4u) ? e[i + 1] : e[i];  // and by one
+  const uint32_t sh = 8u * (b & 3u);
+  return make_uint4(__funnelshift_r(d[0], d[1], sh), __funnelshift_r(d[1], d[2], sh),
+                    __funnelshift_r(d[2], d[3], sh), __funnelshift_r(d[3], d[4], sh));
+}
+
+__device__ __forceinline__ uint4 shfl_up4(const uint4& x) {
+  return make_uint4(__shfl_up_sync(0xffffffffu, x.x, 1), __shfl_up_sync(0xffffffffu, x.y, 1),
+                    __shfl_up_sync(0xffffffffu, x.z, 1), __shfl_up_sync(0xffffffffu, x.w, 1));
+}
+
+// A chunk across an end of the tensor, element by element (not inlined: it
+// is rare and would otherwise hold registers in the vector path).
+template <int NOPS, uint8_t DT>
+__device__ __noinline__ void shift_chunk_elements(void* base, int64_t n, int64_t e0, uint4 y0, uint4 y1,
+                                                  PerturbOp op0, PerturbOp op1) {
+  for (int p = 0; p < 16; ++p) {
+    const int64_t e = e0 + p;
+    if (e < 0 || e >= n) continue;
+    float th = add_signed(load_elem(base, DT, e), y0, p, op0);
+    if (NOPS == 2) th = add_signed(round_to_storage(DT, th), y1, p, op1);
+    store_elem(base, DT, e, th);
+  }
+}
+
+// One group of kShiftGroup chunks of tensor t (all lanes of the warp), as
+// kShiftSub rounds of 31 chunks. 16-bit chunks are software-pipelined: the
+// load of the lane's next chunk is issued before the current one is
+// computed (two 32-byte loads in flight per lane, as for fp32's two halves).
+template <int NOPS, uint8_t DT>
+__device__ __forceinline__ bool shift_full(int lane, int64_t c, uint32_t a, int64_t n) {
+  return lane > 0 && c >= 1 && 16 * c - a + 16 <= n;
+}
+
+template <int NOPS, uint8_t DT>
+__device__ __forceinline__ void shift_group(const PerturbParams& P, const PerturbOp (&op)[2], bool same_ctr, int t,
+                                            int64_t c_first) {
+  constexpr int kElem = DT == kF32 ? 4 : 2;
+  constexpr bool kAhead = DT != kF32;
+  constexpr int kWords = 16 * kElem / 4;  // 32-bit words per chunk: 8 (16-bit) or 16 (fp32)
+  const TensorTable& tab = P.tab;
+  const uintptr_t ptr = tab.ptr[t];
+  const int64_t n = tab.numel[t];
+  const uint32_t a = static_cast<uint32_t>(ptr & 31u) / kElem;  // 1..15 (16-bit) or 1..7 (fp32)
+  char* chunk0 = reinterpret_cast<char*>(ptr - (ptr & 31u));     // 32-byte aligned, a elements before the tensor
+  const int64_t nchunks = (n + a + 15) / 16;
+  const int64_t vb0 = tab.blk_base + tensor_blk_begin(tab, t);  // virtual block of element 0
+  const int lane = static_cast<int>(threadIdx.x & 31u);
+  int64_t c = c_first + lane - 1;  // lane 0: the block below lane 1's chunk, no chunk of its own
+  bool full = shift_full<NOPS, DT>(lane, c, a, n);
+  uint32_t v[kWords];
+  if (kAhead && full) ld256(chunk0 + c * (16 * kElem), *reinterpret_cast<uint32_t(*)[8]>(&v[0]));
+#pragma unroll 1
+  for (int s = 0; s < kShiftSub; ++s) {
+    const int64_t cn = c + kShiftLanes;
+    bool fulln = false;
+    uint32_t vn[kWords];
+    if (kAhead && s + 1 < kShiftSub) {
+      fulln = shift_full<NOPS, DT>(lane, cn, a, n);
+      if (fulln) ld256(chunk0 + cn * (16 * kElem), *reinterpret_cast<uint32_t(*)[8]>(&vn[0]));
+    }
+    char* q = chunk0 + c * (16 * kElem);
+    if (!kAhead && full) {
+      ld256(q, *reinterpret_cast<uint32_t(*)[8]>(&v[0]));
+      ld256(q + 32, *reinterpret_cast<uint32_t(*)[8]>(&v[kWords - 8]));
+    }
+    const int64_t vb = vb0 + c;
+    uint4 x[2], y[2];
+    x[0] = block_bits(vb, op[0].ctr2, P.keys);
+    x[1] = x[0];
+    if (NOPS == 2 && !same_ctr) x[1] = block_bits(vb, op[1].ctr2, P.keys);
+    y[0] = window16(shfl_up4(x[0]), x[0], 16u - a);
+    y[1] = y[0];
+    if (NOPS == 2 && !same_ctr) y[1] = window16(shfl_up4(x[1]), x[1], 16u - a);
+    if (full) {
+      if constexpr (DT == kF32) {
+#pragma unroll
+        for (int i = 0; i < 16; ++i) {
+          float th = add_signed_mul(__uint_as_float(v[i]), y[0], i, op[0]);
+          if (NOPS == 2) th = add_signed_mul(th, y[1], i, op[1]);
+          v[i] = __float_as_uint(th);
+        }
+        st256(q, *reinterpret_cast<uint32_t(*)[8]>(&v[0]));
+        st256(q + 32, *reinterpret_cast<uint32_t(*)[8]>(&v[kWords - 8]));
+      } else {
+        perturb_regs16<DT, NOPS>(*reinterpret_cast<uint32_t(*)[8]>(&v[0]), y, op);
+        st256(q, *reinterpret_cast<uint32_t(*)[8]>(&v[0]));
+      }
+    } else if (lane > 0 && c >= 0 && c < nchunks) {
+      shift_chunk_elements<NOPS, DT>(reinterpret_cast<void*>(ptr), n, 16 * c - a, y[0], y[1], op[0], op[1]);
+    }
+    c = cn;
+    if (kAhead) {
+      full = fulln;
+#pragma unroll
+      for (int r = 0; r < kWords; ++r) v[r] = vn[r];
+    } else {
+      full = shift_full<NOPS, DT>(lane, c, a, n);
+    }
+  }
+}
+
+// One kernel per storage type (a shared one would hold the registers of all
+// three paths): the host launches it for each type its unaligned tensors
+// have, with grp_end counting only that type's tensors. Four blocks per SM
+// (64 registers, no spills): measured faster than three (80 registers) for
+// both the single- and the two-op pass.
+template <int NOPS, uint8_t DT>
+__global__ void __launch_bounds__(256, 4) perturb_shift_kernel(const __grid_constant__ ShiftParams S) {
+  const PerturbParams& P = S.p;
+  if (P.status != nullptr && *P.status != 0) return;
+  PerturbOp op[2] = {P.op[0], P.op[1]};
+  if (P.coef != nullptr)
+    op[0].nscale_bits = __float_as_uint(__double2float_rn(P.coef_mul * P.coef[P.probe])) ^ 0x80000000u;
+  const bool same_ctr = op[1].ctr2 == op[0].ctr2;
+  const uint32_t warp = (blockIdx.x * blockDim.x + threadIdx.x) >> 5;
+  const uint32_t nwarps = (gridDim.x * blockDim.x) >> 5;
+  int t = 0;
+  for (uint32_t g = warp; g < S.grp_total; g += nwarps) {  // the same g on every lane of the warp
+    while (g >= S.grp_end[t]) ++t;
+    const int64_t c_first = static_cast<int64_t>(g - (t == 0 ? 0u : S.grp_end[t - 1])) * kShiftGroup;
+    shift_group<NOPS, DT>(P, op, same_ctr, t, c_first);
+  }
 }
 
 // ---------------------------------------------------------------------------
@@ -703,8 +851,27 @@ cudaError_t launch_perturb(const PerturbParams& p, int grid, int loop, bool f32v
 }
 
 static_assert(sizeof(PairParams) <= 32764, "pair table exceeds the kernel parameter space");
+static_assert(sizeof(ShiftParams) <= 32764, "shift table exceeds the kernel parameter space");
 static_assert(sizeof(PerturbParams) <= 32764 && sizeof(UpdateParams) <= 32764,
               "tensor table exceeds the kernel parameter space");
+
+template <int NOPS>
+void launch_shift_nops(const ShiftParams& p, uint8_t dt, int grid, cudaStream_t stream) {
+  if (dt == kBF16)
+    perturb_shift_kernel<NOPS, kBF16><<<grid, kThreads, 0, stream>>>(p);
+  else if (dt == kF16)
+    perturb_shift_kernel<NOPS, kF16><<<grid, kThreads, 0, stream>>>(p);
+  else
+    perturb_shift_kernel<NOPS, kF32><<<grid, kThreads, 0, stream>>>(p);
+}
+
+cudaError_t launch_perturb_shift(const ShiftParams& p, uint8_t dt, int grid, cudaStream_t stream) {
+  if (p.p.nops == 2)
+    launch_shift_nops<2>(p, dt, grid, stream);
+  else
+    launch_shift_nops<1>(p, dt, grid, stream);
+  return cudaGetLastError();
+}
 
 cudaError_t launch_perturb_pair(const PairParams& p, int grid, cudaStream_t stream) {
   perturb_pair_kernel<<<grid, kThreads, 0, stream>>>(p);
@@ -728,6 +895,19 @@ cudaError_t perturb_blocks_per_sm(int nops, int loop, int* out) {
   if (loop == kLoopRuns)
     return cudaOccupancyMaxActiveBlocksPerMultiprocessor(out, perturb_kernel<2, kLoopRuns>, kThreads, 0);
   return cudaOccupancyMaxActiveBlocksPerMultiprocessor(out, perturb_kernel<2, kLoopBlocks>, kThreads, 0);
+}
+
+template <int NOPS>
+cudaError_t shift_bps_nops(uint8_t dt, int* out) {
+  if (dt == kBF16)
+    return cudaOccupancyMaxActiveBlocksPerMultiprocessor(out, perturb_shift_kernel<NOPS, kBF16>, kThreads, 0);
+  if (dt == kF16)
+    return cudaOccupancyMaxActiveBlocksPerMultiprocessor(out, perturb_shift_kernel<NOPS, kF16>, kThreads, 0);
+  return cudaOccupancyMaxActiveBlocksPerMultiprocessor(out, perturb_shift_kernel<NOPS, kF32>, kThreads, 0);
+}
+
+cudaError_t shift_blocks_per_sm(int nops, uint8_t dt, int* out) {
+  return nops == 2 ? shift_bps_nops<2>(dt, out) : shift_bps_nops<1>(dt, out);
 }
 
 cudaError_t pair_blocks_per_sm(int* out) {

@@ -94,7 +94,7 @@ def test_perturb_bit_exact_scales(scale):
 @pytest.mark.parametrize("offset", [1, 2, 4, 8, 16])
 def test_perturb_unaligned_views(dtype, offset):
     """Views at element offsets that break 32-byte alignment take the
-    element-wise path; results are identical."""
+    aligned-chunk path; results are identical."""
     rng = np.random.default_rng(offset)
     n = 4096 + 37
     base_host = W.random_storage(rng, n + offset + 64, TORCH_TO_DT[dtype])
@@ -108,6 +108,79 @@ def test_perturb_unaligned_views(dtype, offset):
     after = storage_np(base)
     np.testing.assert_array_equal(after[:offset], base_host[:offset])
     np.testing.assert_array_equal(after[offset + n:], base_host[offset + n:])
+
+
+SHIFT_SIZES = [1, 3, 14, 15, 16, 17, 31, 100, 4096 + 37, 20011]
+
+
+def unaligned_list(dtype, seed, prefix=0):
+    """A view at every element offset that breaks 32-byte alignment (sizes
+    from under one 16-element chunk to several chunk groups), each in its own
+    allocation with guard elements around it, an aligned tensor after each,
+    optionally after `prefix` small aligned tensors (pushing the views into a
+    later launch)."""
+    per = 32 // torch.tensor([], dtype=dtype).element_size()
+    rng = np.random.default_rng(seed)
+    dt = TORCH_TO_DT[dtype]
+    bases, views, host = [], [], []
+    for _ in range(prefix):
+        h = W.random_storage(rng, int(rng.integers(0, 40)), dt)
+        views.append(to_torch(h, dtype))
+        host.append(h.copy())
+    for off in range(1, per):
+        n = SHIFT_SIZES[off % len(SHIFT_SIZES)]
+        bh = W.random_storage(rng, off + n + 40, dt)
+        b = to_torch(bh, dtype)
+        bases.append((bh, b, off, n))
+        views.append(b[off:off + n])
+        host.append(bh[off:off + n].copy())
+        ah = W.random_storage(rng, 16 * off + 5, dt)
+        views.append(to_torch(ah, dtype))
+        host.append(ah.copy())
+    return bases, views, host
+
+
+def assert_guards(bases):
+    for bh, b, off, n in bases:
+        after = storage_np(b)
+        np.testing.assert_array_equal(after[:off], bh[:off], err_msg=f"before the view at offset {off}")
+        np.testing.assert_array_equal(after[off + n:], bh[off + n:], err_msg=f"after the view at offset {off}")
+
+
+@pytest.mark.parametrize("dtype", DTS)
+@pytest.mark.parametrize("ops", ["one", "two_same_group", "two_groups"])
+@pytest.mark.parametrize("prefix", [0, 1030])
+def test_perturb_every_unaligned_offset(dtype, ops, prefix, packing_mode):
+    """Unaligned views are perturbed in 32-byte aligned chunks that straddle
+    two Philox blocks: every offset, every size class, one and two
+    operations (probes in one sign group and in two), in the first and in a
+    later launch: bit for bit the oracle, nothing outside the views written."""
+    bases, views, host = unaligned_list(dtype, seed=60 + prefix, prefix=prefix)
+    dts = [TORCH_TO_DT[dtype]] * len(views)
+    seed = W.step_seed(21)
+    if ops == "one":
+        zo.perturb(views, seed, 13, 1e-3)
+        oracle.perturb(host, dts, seed, 13, 1e-3)
+    else:
+        k2 = 14 if ops == "two_same_group" else 22
+        zo.perturb2(views, seed, 13, 1e-3, k2, -2e-3)
+        oracle.perturb(host, dts, seed, 13, 1e-3)
+        oracle.perturb(host, dts, seed, k2, -2e-3)
+    assert_storage_equal(views, host, ops)
+    assert_guards(bases)
+
+
+@pytest.mark.parametrize("dtype", DTS)
+def test_update_sequential_unaligned_views(dtype, packing_mode):
+    """The comparator's per-probe passes read their scale from the device
+    coefficients in the unaligned-chunk kernel too."""
+    bases, views, host = unaligned_list(dtype, seed=70)
+    dts = [TORCH_TO_DT[dtype]] * len(views)
+    c_np = np.random.default_rng(71).normal(0, 25, 9)
+    zo.update_sequential(views, W.step_seed(5), torch.tensor(c_np, device="cuda"), 2e-3)
+    oracle.update_sequential(host, dts, W.step_seed(5), c_np, 2e-3)
+    assert_storage_equal(views, host)
+    assert_guards(bases)
 
 
 @pytest.mark.parametrize("dtype", [torch.bfloat16, torch.float16])
@@ -591,7 +664,7 @@ def test_fused_schedule_matches_algorithm1(packing_mode):
 
 def test_fused_calls_on_split_launches_and_unaligned_views(packing_mode):
     """zo_perturb2 and zo_update_ex on 2500 tensors of odd sizes and mixed
-    dtypes (several launches) plus unaligned views (element-wise path): bit
+    dtypes (several launches) plus unaligned views (aligned-chunk path): bit
     for bit the unfused calls."""
     rng = np.random.default_rng(77)
     numels = [int(x) for x in rng.integers(0, 200, 2500)]
