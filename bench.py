@@ -66,6 +66,9 @@ def parse_args():
                     help="skip the extra measurement of the out-of-place pair schedule")
     ap.add_argument("--sequential", action="store_true",
                     help="also time Algorithm 1's K sequential passes against the fused update")
+    ap.add_argument("--view-offset", type=int, default=0,
+                    help="every parameter a view this many elements into its own allocation (e.g. 1: off the "
+                         "32-byte grid, the perturbation passes run the aligned-chunk kernel)")
     return ap.parse_args()
 
 
@@ -309,8 +312,10 @@ def run_zo(args):
 
     ps = param_set(args)
     K, eps, d = ps.K, ps.eps, ps.d
-    params = W.allocate_params(ps, device=dev)
+    params = W.allocate_params(ps, device=dev, view_offset=args.view_offset)
     plist = zo.ParamList(params)
+    shifted = any(t.data_ptr() % 32 for t in params)   # the perturbation passes use perturb_shift_kernel
+    traffic_key = args.config + (f"+view{args.view_offset}" if args.view_offset else "")
     n_steps_total = args.warmup + args.steps + (0 if args.no_e2e else args.steps)
     losses_host = [W.synthetic_losses(K, s) for s in range(n_steps_total)]
     losses_dev = [torch.tensor(L, device=dev) for L in losses_host]
@@ -491,14 +496,17 @@ def run_zo(args):
     n1, n2 = (K + 1, K - 1) if fused else ((0, 0) if pair else (3 * K, 0))
     if pair:
         dom_kernel, dom_ms, dom_launches = "perturb_pair_kernel", pair_ms, K
-        traffic = committed_traffic("perturb_pair_kernel", args.config)
+        traffic = committed_traffic("perturb_pair_kernel", traffic_key)
     elif n2 > 0 and n2 * perturb2_ms > n1 * perturb_ms:
-        dom_kernel, dom_ms, dom_launches = ("perturb_kernel<2, *> (zo_perturb2, configuration tuned per list)",
+        dom_kernel, dom_ms, dom_launches = ("perturb_shift_kernel<2, *> (zo_perturb2, tensors off the 32-byte grid)"
+                                            if shifted else
+                                            "perturb_kernel<2, *> (zo_perturb2, configuration tuned per list)",
                                             perturb2_ms, n2)
-        traffic = committed_traffic("perturb2_kernel", args.config)
+        traffic = committed_traffic("perturb2_kernel", traffic_key)
     else:
-        dom_kernel, dom_ms, dom_launches = "perturb_kernel<1, 0> (zo_perturb)", perturb_ms, n1
-        traffic = committed_traffic("perturb_kernel", args.config)
+        dom_kernel, dom_ms, dom_launches = ("perturb_shift_kernel<1, *> (zo_perturb, tensors off the 32-byte grid)"
+                                            if shifted else "perturb_kernel<1, 0> (zo_perturb)", perturb_ms, n1)
+        traffic = committed_traffic("perturb_kernel", traffic_key)
     dom_bytes = pair_bytes if pair else perturb_bytes
     # algorithmic HBM bytes of one step: every pass reads and writes theta once,
     # except the pair passes (read theta, write two copies)
@@ -525,6 +533,7 @@ def run_zo(args):
                    "storage": "fp16" if
                    ps.dtype == W.DT_F16 else ("bf16" if ps.dtype == W.DT_BF16 else "fp32"),
                    "eps": eps, "lr": eps, "parallelism": f"replicas{world}",
+                   **({"view_offset": args.view_offset} if args.view_offset else {}),
                    "l2": "inputs larger than L2 (every pass streams the whole parameter set)"},
         "roofline": {"bound": "hbm", "kernel": dom_kernel, "achieved": dom_achieved, "peak": hbm_peak,
                      "unit": "GB/s", "frac": dom_achieved / hbm_peak, "traffic": traffic,

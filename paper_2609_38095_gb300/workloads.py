@@ -136,14 +136,20 @@ def torch_dtype(dtype: int):
     return {DT_F32: torch.float32, DT_BF16: torch.bfloat16, DT_F16: torch.float16}[dtype]
 
 
-def allocate_params(ps: ParamSet, device="cuda", seed_base=1234):
+def allocate_params(ps: ParamSet, device="cuda", seed_base=1234, view_offset=0):
     """Separate device tensors shaped like `ps`, each ~ N(0, 0.02^2) drawn on
-    the device from its own torch generator (seed_base + tensor index)."""
+    the device from its own torch generator (seed_base + tensor index). With
+    view_offset > 0 every tensor is a view that many elements into its own
+    allocation (off the 32-byte grid unless the offset is a multiple of 32
+    bytes)."""
     import torch
     out = []
     tdt = torch_dtype(ps.dtype)
     for i, (_, n) in enumerate(ps.shapes):
-        t = torch.empty(n, dtype=tdt, device=device)
+        if view_offset:
+            t = torch.empty(n + view_offset, dtype=tdt, device=device)[view_offset:]
+        else:
+            t = torch.empty(n, dtype=tdt, device=device)
         g = torch.Generator(device=device)
         g.manual_seed(seed_base + i)
         t.normal_(0.0, 0.02, generator=g)
