@@ -368,6 +368,7 @@ uint32_t shift_groups(const zo::TensorTable& tab, uint8_t dt, uint32_t* grp_end)
 }
 
 thread_local zo::ShiftParams tl_shift;
+thread_local zo::UpdateShiftParams tl_update_shift;
 
 int run_perturb(const zo_tensor* params, int32_t n, PerturbParams& pp, DeviceInfo* d, cudaStream_t s) {
   int loop = zo::kLoopBlocks, bps = d->perturb_bps, slot = -1;
@@ -584,8 +585,25 @@ int zo_update_ex(const zo_tensor* params, int32_t n_tensors, uint64_t seed, cons
     int64_t nb = 0;
     t0 = fill_table(up.tab, params, t0, n_tensors, blk, &nb);
     if (nb > 0) {
-      cudaError_t e = zo::launch_update(up, grid_for(nb, d->sms, bps * kUpdateWaves), s);
-      if (e != cudaSuccess) return cuda_fail(e, "update_kernel");
+      bool main_work = false;
+      const unsigned shift_types = mark_shift(up.tab, &main_work);
+      if (main_work) {
+        cudaError_t e = zo::launch_update(up, grid_for(nb, d->sms, bps * kUpdateWaves), s);
+        if (e != cudaSuccess) return cuda_fail(e, "update_kernel");
+      }
+      if (shift_types) tl_update_shift.u = up;
+      for (uint8_t dt = 0; dt < 3; ++dt) {
+        if (!(shift_types & (1u << dt))) continue;
+        const uint32_t groups = shift_groups(up.tab, dt, tl_update_shift.grp_end);
+        tl_update_shift.grp_total = groups;
+        int sbps = 1;
+        cudaError_t e = zo::update_shift_blocks_per_sm(up.groups, up.packing, dt, &sbps);
+        if (e != cudaSuccess) return cuda_fail(e, "occupancy(update_shift)");
+        const int64_t want = (static_cast<int64_t>(groups) * 32 + zo::kThreads - 1) / zo::kThreads;
+        const int64_t cap = static_cast<int64_t>(d->sms) * (sbps > 0 ? sbps : 1) * kUpdateWaves;
+        e = zo::launch_update_shift(tl_update_shift, dt, static_cast<int>(want < cap ? want : cap), s);
+        if (e != cudaSuccess) return cuda_fail(e, "update_shift_kernel");
+      }
     }
     blk += nb;
   }

@@ -22,6 +22,8 @@ cudaError_t launch_perturb(const PerturbParams& p, int grid, int loop, bool f32v
 cudaError_t launch_perturb_shift(const ShiftParams& p, uint8_t dt, int grid, cudaStream_t stream);
 cudaError_t launch_perturb_pair(const PairParams& p, int grid, cudaStream_t stream);
 cudaError_t launch_update(const UpdateParams& p, int grid, cudaStream_t stream);
+cudaError_t launch_update_shift(const UpdateShiftParams& p, uint8_t dt, int grid, cudaStream_t stream);
+cudaError_t update_shift_blocks_per_sm(int groups, int packing, uint8_t dt, int* out);
 size_t update_smem_bytes(int groups);
 cudaError_t perturb_blocks_per_sm(int nops, int loop, int* out);
 cudaError_t shift_blocks_per_sm(int nops, uint8_t dt, int* out);

@@ -7,10 +7,10 @@
 // stride over the virtual block space of the launch's tensor table). A block
 // of a 16-bit tensor is 32 bytes: one 256-bit load and one 256-bit store when
 // the tensor is 32-byte aligned, element-wise access for a tensor's last,
-// partial block. The perturbation passes hand tensors that are not 32-byte
-// aligned to perturb_shift_kernel, which works on aligned 32-byte chunks
-// straddling two blocks; the pair and update kernels take narrower accesses
-// for them.
+// partial block. The perturbation passes and the update hand tensors that
+// are not 32-byte aligned to perturb_shift_kernel / update_shift_kernel,
+// which work on aligned 32-byte chunks straddling two blocks; the pair
+// kernel takes narrower accesses for them.
 #include "zo_device.cuh"
 
 namespace zo {
@@ -724,21 +724,24 @@ __device__ __forceinline__ void update_block_vec(void* base, int64_t e0, int64_t
   }
 }
 
-template <int PACK>
-__global__ void __launch_bounds__(256) update_kernel(const __grid_constant__ UpdateParams P) {
-  extern __shared__ __align__(16) unsigned char smem[];
+// Per-CTA prologue of the update kernels: a_k = fp32(coef_mul * c_k) for the
+// K probes (zero-padded to 8 * groups) and the per-quad partial-sum tables in
+// their frames. Returns false when the block has nothing to do (a failed
+// preconditioner and no leading perturbation); do_sum is false when only the
+// leading perturbation applies.
+__device__ __forceinline__ bool update_prologue(const UpdateParams& P, unsigned char* smem, int& skip,
+                                                uint32_t& lut_base, bool& do_sum) {
   float* a_s = reinterpret_cast<float*>(smem);  // 8 * groups coefficients (zero padded)
   const uint32_t smem_sh = static_cast<uint32_t>(__cvta_generic_to_shared(smem));
-  const uint32_t lut_base = (smem_sh + 32u * P.groups + kFrameBytes - 1) & ~(kFrameBytes - 1);
+  lut_base = (smem_sh + 32u * P.groups + kFrameBytes - 1) & ~(kFrameBytes - 1);
   float* lut = reinterpret_cast<float*>(smem + (lut_base - smem_sh));  // generic view of the frames
-  __shared__ int skip;
   if (threadIdx.x == 0) skip = (P.status != nullptr && *P.status != 0);
   const int npad = 8 * P.groups;
   for (int k = threadIdx.x; k < npad; k += blockDim.x)
     a_s[k] = k < P.K ? __double2float_rn(P.coef_mul * P.coef[k]) : 0.0f;
   __syncthreads();
-  if (skip && !P.has_pre) return;
-  const bool do_sum = !skip;  // a failed preconditioner still gets the leading perturbation
+  if (skip && !P.has_pre) return false;
+  do_sum = !skip;  // a failed preconditioner still gets the leading perturbation
   for (int e = threadIdx.x; e < 32 * P.groups; e += blockDim.x) {
     const int h = e >> 4, n = e & 15;
     const float* a = a_s + 4 * h;
@@ -749,6 +752,16 @@ __global__ void __launch_bounds__(256) update_kernel(const __grid_constant__ Upd
     lut[(h >> 1) * (kFrameBytes / 4) + (h & 1) * 16 + n] = s;
   }
   __syncthreads();
+  return true;
+}
+
+template <int PACK>
+__global__ void __launch_bounds__(256) update_kernel(const __grid_constant__ UpdateParams P) {
+  extern __shared__ __align__(16) unsigned char smem[];
+  __shared__ int skip;
+  uint32_t lut_base;
+  bool do_sum;
+  if (!update_prologue(P, smem, skip, lut_base, do_sum)) return;
 
   const TensorTable& tab = P.tab;
   const uint32_t stride = gridDim.x * blockDim.x;
@@ -768,7 +781,7 @@ __global__ void __launch_bounds__(256) update_kernel(const __grid_constant__ Upd
         update_block_vec<PACK, kF16>(base, e0, b, P, lut_base, do_sum);
       else
         update_block_vec<PACK, kF32>(base, e0, b, P, lut_base, do_sum);
-    } else {
+    } else if (!(fl & kShift)) {  // kShift: an unaligned tensor, update_shift_kernel's
       float acc[16];
 #pragma unroll
       for (int m = 0; m < 16; ++m) acc[m] = 0.0f;
@@ -785,6 +798,122 @@ __global__ void __launch_bounds__(256) update_kernel(const __grid_constant__ Upd
         }
       }
     }
+  }
+}
+
+// ---------------------------------------------------------------------------
+// Fused update of unaligned tensors (kShift), in the 32-byte aligned chunks of
+// perturb_shift_kernel. Lane l sums the probes of block c = c0 - 1 + l (in
+// block order, exactly as update_kernel does) and takes the sums of block
+// c - 1 from lane l - 1; chunk c's sixteen sums are elements 16 - a .. 31 - a
+// of the two blocks' sums, so every element gets the same fp32 value as in
+// update_kernel.
+// ---------------------------------------------------------------------------
+// out[p] = (lo ++ hi)[s + p] for p = 0..15, s = 0..15: four stages of selects.
+__device__ __forceinline__ void window16f(const float (&lo)[16], const float (&hi)[16], uint32_t s,
+                                          float (&out)[16]) {
+  float t8[24], t4[20], t2[18];
+#pragma unroll
+  for (int i = 0; i < 24; ++i) {
+    const float a = i < 16 ? lo[i] : hi[i - 16];
+    const float b = i + 8 < 16 ? lo[i + 8] : hi[i - 8];
+    t8[i] = (s & 8u) ? b : a;
+  }
+#pragma unroll
+  for (int i = 0; i < 20; ++i) t4[i] = (s & 4u) ? t8[i + 4] : t8[i];
+#pragma unroll
+  for (int i = 0; i < 18; ++i) t2[i] = (s & 2u) ? t4[i + 2] : t4[i];
+#pragma unroll
+  for (int i = 0; i < 16; ++i) out[i] = (s & 1u) ? t2[i + 1] : t2[i];
+}
+
+template <int PACK, uint8_t DT>
+__device__ __forceinline__ void update_shift_group(const UpdateParams& P, uint32_t lut_base, bool do_sum, int t,
+                                                   int64_t c_first) {
+  constexpr int kElem = DT == kF32 ? 4 : 2;
+  constexpr int kWords = 16 * kElem / 4;
+  const TensorTable& tab = P.tab;
+  const uintptr_t ptr = tab.ptr[t];
+  const int64_t n = tab.numel[t];
+  const uint32_t a = static_cast<uint32_t>(ptr & 31u) / kElem;
+  char* chunk0 = reinterpret_cast<char*>(ptr - (ptr & 31u));
+  const int64_t nchunks = (n + a + 15) / 16;
+  const int64_t vb0 = tab.blk_base + tensor_blk_begin(tab, t);
+  const int lane = static_cast<int>(threadIdx.x & 31u);
+#pragma unroll 1
+  for (int s = 0; s < kShiftSub; ++s) {
+    const int64_t c = c_first + s * kShiftLanes + lane - 1;
+    const bool full = shift_full<1, DT>(lane, c, a, n);
+    char* q = chunk0 + c * (16 * kElem);
+    uint32_t v[kWords];
+    if (full) {  // issued before the probe sums, which hide its latency
+      ld256(q, *reinterpret_cast<uint32_t(*)[8]>(&v[0]));
+      if constexpr (DT == kF32) ld256(q + 32, *reinterpret_cast<uint32_t(*)[8]>(&v[8]));
+    }
+    float own[16], below[16], sum[16];
+#pragma unroll
+    for (int m = 0; m < 16; ++m) own[m] = 0.0f;
+    if (do_sum) accumulate_any<PACK>(own, vb0 + c, P, lut_base);
+#pragma unroll
+    for (int m = 0; m < 16; ++m) below[m] = __shfl_up_sync(0xffffffffu, own[m], 1);
+    window16f(below, own, 16u - a, sum);
+    uint4 y = make_uint4(0u, 0u, 0u, 0u);
+    if (P.has_pre) {
+      const uint4 xp = block_bits(vb0 + c, P.pre.ctr2, P.keys);
+      y = window16(shfl_up4(xp), xp, 16u - a);
+    }
+    if (full) {
+      if constexpr (DT == kF32) {
+#pragma unroll
+        for (int i = 0; i < 16; ++i) {
+          float th = __uint_as_float(v[i]);
+          if (P.has_pre) th = add_signed(th, y, i, P.pre);
+          if (do_sum) th = __fadd_rn(th, sum[i]);
+          v[i] = __float_as_uint(th);
+        }
+        st256(q, *reinterpret_cast<uint32_t(*)[8]>(&v[0]));
+        st256(q + 32, *reinterpret_cast<uint32_t(*)[8]>(&v[8]));
+      } else {
+#pragma unroll
+        for (int r = 0; r < 8; ++r) {
+          if (P.has_pre) v[r] = pre_regs16<DT>(v[r], y, r, P.pre);
+          if (do_sum) {
+            const float2 f = unpack2<DT>(v[r]);
+            v[r] = pack2<DT>(__fadd_rn(f.x, sum[2 * r]), __fadd_rn(f.y, sum[2 * r + 1]));
+          }
+        }
+        st256(q, *reinterpret_cast<uint32_t(*)[8]>(&v[0]));
+      }
+    } else if (lane > 0 && c >= 0 && c < nchunks) {  // a chunk across an end of the tensor
+      void* base = reinterpret_cast<void*>(ptr);
+#pragma unroll
+      for (int p = 0; p < 16; ++p) {
+        const int64_t e = 16 * c - a + p;
+        if (e < 0 || e >= n) continue;
+        float th = load_elem(base, DT, e);
+        if (P.has_pre) th = round_to_storage(DT, add_signed(th, y, p, P.pre));
+        if (do_sum) th = __fadd_rn(th, sum[p]);
+        store_elem(base, DT, e, th);
+      }
+    }
+  }
+}
+
+template <int PACK, uint8_t DT>
+__global__ void __launch_bounds__(256) update_shift_kernel(const __grid_constant__ UpdateShiftParams S) {
+  const UpdateParams& P = S.u;
+  extern __shared__ __align__(16) unsigned char smem[];
+  __shared__ int skip;
+  uint32_t lut_base;
+  bool do_sum;
+  if (!update_prologue(P, smem, skip, lut_base, do_sum)) return;
+  const uint32_t warp = (blockIdx.x * blockDim.x + threadIdx.x) >> 5;
+  const uint32_t nwarps = (gridDim.x * blockDim.x) >> 5;
+  int t = 0;
+  for (uint32_t g = warp; g < S.grp_total; g += nwarps) {  // the same g on every lane of the warp
+    while (g >= S.grp_end[t]) ++t;
+    const int64_t c_first = static_cast<int64_t>(g - (t == 0 ? 0u : S.grp_end[t - 1])) * kShiftGroup;
+    update_shift_group<PACK, DT>(P, lut_base, do_sum, t, c_first);
   }
 }
 
@@ -851,7 +980,8 @@ cudaError_t launch_perturb(const PerturbParams& p, int grid, int loop, bool f32v
 }
 
 static_assert(sizeof(PairParams) <= 32764, "pair table exceeds the kernel parameter space");
-static_assert(sizeof(ShiftParams) <= 32764, "shift table exceeds the kernel parameter space");
+static_assert(sizeof(ShiftParams) <= 32764 && sizeof(UpdateShiftParams) <= 32764,
+              "shift table exceeds the kernel parameter space");
 static_assert(sizeof(PerturbParams) <= 32764 && sizeof(UpdateParams) <= 32764,
               "tensor table exceeds the kernel parameter space");
 
@@ -871,6 +1001,40 @@ cudaError_t launch_perturb_shift(const ShiftParams& p, uint8_t dt, int grid, cud
   else
     launch_shift_nops<1>(p, dt, grid, stream);
   return cudaGetLastError();
+}
+
+template <int PACK>
+void launch_update_shift_pack(const UpdateShiftParams& p, uint8_t dt, int grid, size_t smem, cudaStream_t stream) {
+  if (dt == kBF16)
+    update_shift_kernel<PACK, kBF16><<<grid, kThreads, smem, stream>>>(p);
+  else if (dt == kF16)
+    update_shift_kernel<PACK, kF16><<<grid, kThreads, smem, stream>>>(p);
+  else
+    update_shift_kernel<PACK, kF32><<<grid, kThreads, smem, stream>>>(p);
+}
+
+cudaError_t launch_update_shift(const UpdateShiftParams& p, uint8_t dt, int grid, cudaStream_t stream) {
+  const size_t smem = update_smem_bytes(p.u.groups);
+  if (p.u.packing == kPacking8)
+    launch_update_shift_pack<kPacking8>(p, dt, grid, smem, stream);
+  else
+    launch_update_shift_pack<kPacking1>(p, dt, grid, smem, stream);
+  return cudaGetLastError();
+}
+
+template <int PACK>
+cudaError_t update_shift_bps_pack(int groups, uint8_t dt, int* out) {
+  const size_t smem = update_smem_bytes(groups);
+  if (dt == kBF16)
+    return cudaOccupancyMaxActiveBlocksPerMultiprocessor(out, update_shift_kernel<PACK, kBF16>, kThreads, smem);
+  if (dt == kF16)
+    return cudaOccupancyMaxActiveBlocksPerMultiprocessor(out, update_shift_kernel<PACK, kF16>, kThreads, smem);
+  return cudaOccupancyMaxActiveBlocksPerMultiprocessor(out, update_shift_kernel<PACK, kF32>, kThreads, smem);
+}
+
+cudaError_t update_shift_blocks_per_sm(int groups, int packing, uint8_t dt, int* out) {
+  return packing == kPacking8 ? update_shift_bps_pack<kPacking8>(groups, dt, out)
+                              : update_shift_bps_pack<kPacking1>(groups, dt, out);
 }
 
 cudaError_t launch_perturb_pair(const PairParams& p, int grid, cudaStream_t stream) {

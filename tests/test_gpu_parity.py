@@ -171,6 +171,49 @@ def test_perturb_every_unaligned_offset(dtype, ops, prefix, packing_mode):
 
 
 @pytest.mark.parametrize("dtype", DTS)
+@pytest.mark.parametrize("K", [5, 16, 64])
+@pytest.mark.parametrize("pre", [False, True])
+def test_update_every_unaligned_offset(dtype, K, pre, packing_mode):
+    """The fused update of unaligned views (aligned chunks, probe sums taken
+    from the neighbouring lane) gives bit for bit what update_kernel gives
+    for the same values in aligned tensors, is within the derived bound of
+    the oracle, and writes nothing outside the views."""
+    bases, views, host = unaligned_list(dtype, seed=80 + K)
+    dts = [TORCH_TO_DT[dtype]] * len(views)
+    aligned = [to_torch(h.copy(), dtype) for h in host]
+    c_np = np.random.default_rng(81 + K).normal(0, 25, K)
+    c = torch.tensor(c_np, device="cuda")
+    seed, lr = W.step_seed(6), 1e-3
+    p = (K - 1, 1e-3) if pre else None
+    zo.update(views, seed, c, lr, pre=p)
+    zo.update(aligned, seed, c, lr, pre=p)
+    for i, (x, y) in enumerate(zip(views, aligned)):
+        assert torch.equal(x.contiguous().view(torch.uint8), y.view(torch.uint8)), f"tensor {i}"
+    if pre:
+        oracle.perturb(host, dts, seed, K - 1, 1e-3)
+    oracle.update(host, dts, seed, c_np, lr)
+    for i, (d, h) in enumerate(zip(views, host)):
+        assert_update_close(storage_bits(d), storage_bits(h), TORCH_TO_DT[dtype], c_np, lr, context=f"tensor {i}")
+    assert_guards(bases)
+
+
+def test_update_unaligned_failed_preconditioner():
+    """status != 0: the update kernels of unaligned views apply only the
+    leading perturbation (or nothing without one)."""
+    bases, views, host = unaligned_list(torch.bfloat16, seed=90)
+    dts = [W.DT_BF16] * len(views)
+    st = torch.tensor([zo.ZO_ERR_NONFINITE], dtype=torch.int32, device="cuda")
+    c = torch.ones(8, dtype=torch.float64, device="cuda")
+    seed = W.step_seed(8)
+    zo.update(views, seed, c, 1e-3, status=st)
+    assert_storage_equal(views, host, "no pre, failed status: untouched")
+    zo.update(views, seed, c, 1e-3, status=st, pre=(3, 2e-3))
+    oracle.perturb(host, dts, seed, 3, 2e-3)
+    assert_storage_equal(views, host, "failed status: only the leading perturbation")
+    assert_guards(bases)
+
+
+@pytest.mark.parametrize("dtype", DTS)
 def test_update_sequential_unaligned_views(dtype, packing_mode):
     """The comparator's per-probe passes read their scale from the device
     coefficients in the unaligned-chunk kernel too."""
