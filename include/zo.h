@@ -41,8 +41,9 @@
  * (ZO_ERR_ARG beyond). ptr must be aligned to its element size. Any such
  * alignment gives the same results; a tensor whose ptr is not 32-byte aligned
  * is streamed in 32-byte aligned chunks by a second kernel of the same call
- * (zo_perturb, zo_perturb2, zo_update, zo_update_ex, zo_update_sequential),
- * or with narrower accesses (zo_perturb_pair).
+ * (zo_perturb, zo_perturb2, zo_update, zo_update_ex, zo_update_sequential;
+ * zo_perturb_pair when theta, plus and minus share the offset), otherwise
+ * with narrower accesses.
  *
  * Probes. z_k is Rademacher, one bit per parameter per probe (Sec. 2, Sec. 4.3
  * "Bit-Packed perturbations"; unpack rule of Appendix F: bit 1 -> +1, bit 0 ->

@@ -76,6 +76,7 @@ zo::PerturbOp make_op(uint32_t k, float scale, int packing) {
 // configurations, timed on the caller's list (TwoOpTuner below).
 constexpr int kPerturbBlocksPerSm = 4;
 constexpr int kPairBlocksPerSm = 3;
+constexpr int kShiftBlocksPerSm = 4;   // pair_shift_kernel: 256 threads, at most 64 registers
 constexpr int kTwoOpCandidates = 3;
 constexpr int kTwoOpLoop[kTwoOpCandidates] = {zo::kLoopRuns, zo::kLoopRuns, zo::kLoopBlocks};
 constexpr int kTwoOpBlocksPerSm[kTwoOpCandidates] = {3, 4, 4};
@@ -438,6 +439,68 @@ int32_t fill_pair_table(zo::PairTable& tab, const zo_tensor* theta, const zo_ten
   return t;
 }
 
+// Tensors of a pair launch for pair_shift_kernel: fp32 tensors, and 16-bit
+// tensors not all 32-byte aligned, when the three pointers share their offset
+// from the 32-byte grid (the others keep perturb_pair_kernel's paths).
+// Returns a bit mask of their storage types.
+unsigned mark_pair_shift(zo::PairTable& tab, bool* main_work) {
+  unsigned types = 0;
+  *main_work = false;
+  for (int i = 0; i < tab.n; ++i) {
+    const uint32_t begin = i == 0 ? 0u : tab.blk_end[i - 1];
+    if (tab.blk_end[i] == begin) continue;  // empty
+    const uint8_t dt = tab.flags[i] & zo::kDtypeMask;
+    const bool same = tab.src[i] % 32 == tab.plus[i] % 32 && tab.src[i] % 32 == tab.minus[i] % 32;
+    if (same && (dt == zo::kF32 || !(tab.flags[i] & zo::kVec32))) {
+      tab.flags[i] |= zo::kShift;
+      types |= 1u << dt;
+    } else {
+      *main_work = true;
+    }
+  }
+  return types;
+}
+
+thread_local zo::PairShiftParams tl_pair_shift;
+
+// Launch pair_shift_kernel over the flagged tensors of type dt (in batches of
+// kMaxPairShift entries).
+int run_pair_shift(const zo::PairParams& pp, uint8_t dt, DeviceInfo* d, cudaStream_t s) {
+  zo::PairShiftParams& S = tl_pair_shift;
+  S.keys = pp.keys;
+  S.op = pp.op;
+  const zo::PairTable& tab = pp.tab;
+  const uint32_t esz = dt == zo::kF32 ? 4 : 2;
+  int i = 0;
+  while (i < tab.n) {
+    S.n = 0;
+    uint32_t groups = 0;
+    for (; i < tab.n && S.n < zo::kMaxPairShift; ++i) {
+      const uint8_t fl = tab.flags[i];
+      if (!(fl & zo::kShift) || (fl & zo::kDtypeMask) != dt) continue;
+      const uint32_t begin = i == 0 ? 0u : tab.blk_end[i - 1];
+      const int64_t numel = static_cast<int64_t>(tab.blk_end[i] - begin - 1) * 16 + tab.last[i];
+      const int64_t a = static_cast<int64_t>(tab.src[i] % 32) / esz;
+      const int64_t chunks = (numel + a + 15) / 16;
+      const int j = S.n++;
+      S.src[j] = tab.src[i];
+      S.plus[j] = tab.plus[i];
+      S.minus[j] = tab.minus[i];
+      S.numel[j] = numel;
+      S.vb0[j] = tab.blk_base + begin;
+      groups += static_cast<uint32_t>((chunks + zo::kShiftGroup - 1) / zo::kShiftGroup);
+      S.grp_end[j] = groups;
+    }
+    if (S.n == 0) break;
+    S.grp_total = groups;
+    const int64_t want = (static_cast<int64_t>(groups) * 32 + zo::kThreads - 1) / zo::kThreads;
+    const int64_t cap = static_cast<int64_t>(d->sms) * kShiftBlocksPerSm;
+    cudaError_t e = zo::launch_pair_shift(S, dt, static_cast<int>(want < cap ? want : cap), s);
+    if (e != cudaSuccess) return cuda_fail(e, "pair_shift_kernel");
+  }
+  return ZO_OK;
+}
+
 thread_local PerturbParams tl_perturb;
 thread_local zo::PairParams tl_pair;
 thread_local UpdateParams tl_update;
@@ -536,9 +599,17 @@ int zo_perturb_pair(const zo_tensor* theta, const zo_tensor* plus, const zo_tens
     int64_t nb = 0;
     t0 = fill_pair_table(pp.tab, theta, plus, minus, t0, n_tensors, blk, &nb);
     if (nb > 0) {
-      cudaError_t e = zo::launch_perturb_pair(pp, grid_for(nb, d->sms, d->pair_bps),
-                                              static_cast<cudaStream_t>(stream));
-      if (e != cudaSuccess) return cuda_fail(e, "perturb_pair_kernel");
+      bool main_work = false;
+      const unsigned shift_types = mark_pair_shift(pp.tab, &main_work);
+      if (main_work) {
+        cudaError_t e = zo::launch_perturb_pair(pp, grid_for(nb, d->sms, d->pair_bps),
+                                                static_cast<cudaStream_t>(stream));
+        if (e != cudaSuccess) return cuda_fail(e, "perturb_pair_kernel");
+      }
+      for (uint8_t dt = 0; dt < 3; ++dt) {
+        if (!(shift_types & (1u << dt))) continue;
+        if ((rc = run_pair_shift(pp, dt, d, static_cast<cudaStream_t>(stream))) != ZO_OK) return rc;
+      }
     }
     blk += nb;
   }

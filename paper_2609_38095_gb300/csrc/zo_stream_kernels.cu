@@ -9,8 +9,9 @@
 // the tensor is 32-byte aligned, element-wise access for a tensor's last,
 // partial block. The perturbation passes and the update hand tensors that
 // are not 32-byte aligned to perturb_shift_kernel / update_shift_kernel,
-// which work on aligned 32-byte chunks straddling two blocks; the pair
-// kernel takes narrower accesses for them.
+// which work on aligned 32-byte chunks straddling two blocks; the pair pass
+// hands them (and fp32 tensors) to pair_shift_kernel when its three pointers
+// share the offset, and takes narrower accesses otherwise.
 #include "zo_device.cuh"
 
 namespace zo {
@@ -359,15 +360,15 @@ __device__ __noinline__ void shift_chunk_elements(void* base, int64_t n, int64_t
   }
 }
 
-// One group of kShiftGroup chunks of tensor t (all lanes of the warp), as
-// kShiftSub rounds of 31 chunks. 16-bit chunks are software-pipelined: the
-// load of the lane's next chunk is issued before the current one is
-// computed (two 32-byte loads in flight per lane, as for fp32's two halves).
-template <int NOPS, uint8_t DT>
+// Chunk c is the lane's own (lane > 0) and lies wholly inside the tensor.
 __device__ __forceinline__ bool shift_full(int lane, int64_t c, uint32_t a, int64_t n) {
   return lane > 0 && c >= 1 && 16 * c - a + 16 <= n;
 }
 
+// One group of kShiftGroup chunks of tensor t (all lanes of the warp), as
+// kShiftSub rounds of 31 chunks. 16-bit chunks are software-pipelined: the
+// load of the lane's next chunk is issued before the current one is
+// computed (two 32-byte loads in flight per lane, as for fp32's two halves).
 template <int NOPS, uint8_t DT>
 __device__ __forceinline__ void shift_group(const PerturbParams& P, const PerturbOp (&op)[2], bool same_ctr, int t,
                                             int64_t c_first) {
@@ -383,7 +384,7 @@ __device__ __forceinline__ void shift_group(const PerturbParams& P, const Pertur
   const int64_t vb0 = tab.blk_base + tensor_blk_begin(tab, t);  // virtual block of element 0
   const int lane = static_cast<int>(threadIdx.x & 31u);
   int64_t c = c_first + lane - 1;  // lane 0: the block below lane 1's chunk, no chunk of its own
-  bool full = shift_full<NOPS, DT>(lane, c, a, n);
+  bool full = shift_full(lane, c, a, n);
   uint32_t v[kWords];
   if (kAhead && full) ld256(chunk0 + c * (16 * kElem), *reinterpret_cast<uint32_t(*)[8]>(&v[0]));
 #pragma unroll 1
@@ -392,7 +393,7 @@ __device__ __forceinline__ void shift_group(const PerturbParams& P, const Pertur
     bool fulln = false;
     uint32_t vn[kWords];
     if (kAhead && s + 1 < kShiftSub) {
-      fulln = shift_full<NOPS, DT>(lane, cn, a, n);
+      fulln = shift_full(lane, cn, a, n);
       if (fulln) ld256(chunk0 + cn * (16 * kElem), *reinterpret_cast<uint32_t(*)[8]>(&vn[0]));
     }
     char* q = chunk0 + c * (16 * kElem);
@@ -431,7 +432,7 @@ __device__ __forceinline__ void shift_group(const PerturbParams& P, const Pertur
 #pragma unroll
       for (int r = 0; r < kWords; ++r) v[r] = vn[r];
     } else {
-      full = shift_full<NOPS, DT>(lane, c, a, n);
+      full = shift_full(lane, c, a, n);
     }
   }
 }
@@ -479,6 +480,7 @@ __device__ __forceinline__ void pair_regs16(const uint32_t (&v)[8], const uint4&
 }
 
 __device__ __noinline__ void pair_block_other(const PairTable& tab, int t, uint32_t b, uint4 x, PerturbOp op) {
+  if (tab.flags[t] & kShift) return;  // pair_shift_kernel's
   const uint32_t tb = t == 0 ? 0u : tab.blk_end[t - 1];
   const int64_t e0 = static_cast<int64_t>(b - tb) * 16;
   const int cnt = b + 1 == tab.blk_end[t] ? tab.last[t] : 16;
@@ -569,6 +571,108 @@ __global__ void __launch_bounds__(256) perturb_pair_kernel(const __grid_constant
     vec = vecn;
 #pragma unroll
     for (int r = 0; r < 8; ++r) v[r] = vn[r];
+  }
+}
+
+// ---------------------------------------------------------------------------
+// The pair of perturbations in 32-byte aligned chunks (as perturb_shift_kernel;
+// a = 0 for aligned fp32 tensors, whose chunks are the blocks themselves).
+// ---------------------------------------------------------------------------
+template <uint8_t DT>
+__device__ __noinline__ void pair_chunk_elements(const void* src, void* pl, void* mi, int64_t n, int64_t e0, uint4 y,
+                                                 PerturbOp op) {
+  for (int p = 0; p < 16; ++p) {
+    const int64_t e = e0 + p;
+    if (e < 0 || e >= n) continue;
+    const float th = load_elem(src, DT, e);
+    const float d = __uint_as_float(op.nscale_bits ^ sign_bit(y, p, op.bit));
+    store_elem(pl, DT, e, __fadd_rn(th, d));
+    store_elem(mi, DT, e, __fsub_rn(th, d));
+  }
+}
+
+template <uint8_t DT>
+__device__ __forceinline__ void pair_shift_group(const PairShiftParams& S, int t, int64_t c_first) {
+  constexpr int kElem = DT == kF32 ? 4 : 2;
+  constexpr bool kAhead = DT != kF32;
+  constexpr int kWords = 16 * kElem / 4;
+  const PerturbOp& op = S.op;
+  const uintptr_t src = S.src[t];
+  const uint32_t off = static_cast<uint32_t>(src & 31u);  // the same for plus and minus
+  const uint32_t a = off / kElem;                        // 0..15 (16-bit) or 0..7 (fp32)
+  const char* s0 = reinterpret_cast<const char*>(src - off);
+  char* p0 = reinterpret_cast<char*>(S.plus[t] - off);
+  char* m0 = reinterpret_cast<char*>(S.minus[t] - off);
+  const int64_t n = S.numel[t];
+  const int64_t nchunks = (n + a + 15) / 16;
+  const int lane = static_cast<int>(threadIdx.x & 31u);
+  auto full_at = [&](int64_t c) { return lane > 0 && 16 * c >= a && 16 * c - a + 16 <= n; };
+  int64_t c = c_first + lane - 1;
+  bool full = full_at(c);
+  uint32_t v[kWords];
+  if (kAhead && full) ld256(s0 + c * (16 * kElem), *reinterpret_cast<uint32_t(*)[8]>(&v[0]));
+#pragma unroll 1
+  for (int s = 0; s < kShiftSub; ++s) {
+    const int64_t cn = c + kShiftLanes;
+    bool fulln = false;
+    uint32_t vn[kWords];
+    if (kAhead && s + 1 < kShiftSub) {
+      fulln = full_at(cn);
+      if (fulln) ld256(s0 + cn * (16 * kElem), *reinterpret_cast<uint32_t(*)[8]>(&vn[0]));
+    }
+    const int64_t cb = c * (16 * kElem);
+    if (!kAhead && full) {
+      ld256(s0 + cb, *reinterpret_cast<uint32_t(*)[8]>(&v[0]));
+      ld256(s0 + cb + 32, *reinterpret_cast<uint32_t(*)[8]>(&v[kWords - 8]));
+    }
+    const uint4 x = block_bits(S.vb0[t] + c, op.ctr2, S.keys);
+    const uint4 below = shfl_up4(x);
+    const uint4 y = a == 0 ? x : window16(below, x, 16u - a);
+    if (full) {
+      if constexpr (DT == kF32) {
+        uint32_t m[16];
+#pragma unroll
+        for (int i = 0; i < 16; ++i) {
+          const float th = __uint_as_float(v[i]);
+          const float d = __uint_as_float(op.nscale_bits ^ sign_bit_mul(y, i, op));
+          v[i] = __float_as_uint(__fadd_rn(th, d));
+          m[i] = __float_as_uint(__fsub_rn(th, d));
+        }
+        st256(p0 + cb, *reinterpret_cast<uint32_t(*)[8]>(&v[0]));
+        st256(p0 + cb + 32, *reinterpret_cast<uint32_t(*)[8]>(&v[8]));
+        st256(m0 + cb, *reinterpret_cast<uint32_t(*)[8]>(&m[0]));
+        st256(m0 + cb + 32, *reinterpret_cast<uint32_t(*)[8]>(&m[8]));
+      } else {
+        uint32_t m[8];
+        pair_regs16<DT>(*reinterpret_cast<uint32_t(*)[8]>(&v[0]), y, op, *reinterpret_cast<uint32_t(*)[8]>(&v[0]),
+                        m);
+        st256(p0 + cb, *reinterpret_cast<uint32_t(*)[8]>(&v[0]));
+        st256(m0 + cb, m);
+      }
+    } else if (lane > 0 && c >= 0 && c < nchunks) {  // a chunk across an end of the tensor
+      pair_chunk_elements<DT>(reinterpret_cast<const void*>(src), reinterpret_cast<void*>(S.plus[t]),
+                              reinterpret_cast<void*>(S.minus[t]), n, 16 * c - a, y, op);
+    }
+    c = cn;
+    if (kAhead) {
+      full = fulln;
+#pragma unroll
+      for (int r = 0; r < kWords; ++r) v[r] = vn[r];
+    } else {
+      full = full_at(c);
+    }
+  }
+}
+
+template <uint8_t DT>
+__global__ void __launch_bounds__(256, 4) pair_shift_kernel(const __grid_constant__ PairShiftParams S) {
+  const uint32_t warp = (blockIdx.x * blockDim.x + threadIdx.x) >> 5;
+  const uint32_t nwarps = (gridDim.x * blockDim.x) >> 5;
+  int t = 0;
+  for (uint32_t g = warp; g < S.grp_total; g += nwarps) {  // the same g on every lane of the warp
+    while (g >= S.grp_end[t]) ++t;
+    const int64_t c_first = static_cast<int64_t>(g - (t == 0 ? 0u : S.grp_end[t - 1])) * kShiftGroup;
+    pair_shift_group<DT>(S, t, c_first);
   }
 }
 
@@ -843,7 +947,7 @@ __device__ __forceinline__ void update_shift_group(const UpdateParams& P, uint32
 #pragma unroll 1
   for (int s = 0; s < kShiftSub; ++s) {
     const int64_t c = c_first + s * kShiftLanes + lane - 1;
-    const bool full = shift_full<1, DT>(lane, c, a, n);
+    const bool full = shift_full(lane, c, a, n);
     char* q = chunk0 + c * (16 * kElem);
     uint32_t v[kWords];
     if (full) {  // issued before the probe sums, which hide its latency
@@ -980,7 +1084,7 @@ cudaError_t launch_perturb(const PerturbParams& p, int grid, int loop, bool f32v
 }
 
 static_assert(sizeof(PairParams) <= 32764, "pair table exceeds the kernel parameter space");
-static_assert(sizeof(ShiftParams) <= 32764 && sizeof(UpdateShiftParams) <= 32764,
+static_assert(sizeof(ShiftParams) <= 32764 && sizeof(UpdateShiftParams) <= 32764 && sizeof(PairShiftParams) <= 32764,
               "shift table exceeds the kernel parameter space");
 static_assert(sizeof(PerturbParams) <= 32764 && sizeof(UpdateParams) <= 32764,
               "tensor table exceeds the kernel parameter space");
@@ -1000,6 +1104,16 @@ cudaError_t launch_perturb_shift(const ShiftParams& p, uint8_t dt, int grid, cud
     launch_shift_nops<2>(p, dt, grid, stream);
   else
     launch_shift_nops<1>(p, dt, grid, stream);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_pair_shift(const PairShiftParams& p, uint8_t dt, int grid, cudaStream_t stream) {
+  if (dt == kBF16)
+    pair_shift_kernel<kBF16><<<grid, kThreads, 0, stream>>>(p);
+  else if (dt == kF16)
+    pair_shift_kernel<kF16><<<grid, kThreads, 0, stream>>>(p);
+  else
+    pair_shift_kernel<kF32><<<grid, kThreads, 0, stream>>>(p);
   return cudaGetLastError();
 }
 

@@ -85,9 +85,10 @@ def test_pair_bit_exact_mixed(k, scale, packing_mode):
 @pytest.mark.parametrize("offset", [1, 8, 16])
 @pytest.mark.parametrize("dtype", [torch.bfloat16, torch.float16, torch.float32])
 def test_pair_unaligned(which, offset, dtype):
-    """Any one of the three pointers off the 32-byte grid sends the tensor to
-    the element-wise path; results are identical and nothing outside the views
-    is written."""
+    """One of the three pointers off the 32-byte grid (the others aligned)
+    sends the tensor to the per-block path with the widest accesses each
+    address allows; results are identical and nothing outside the views is
+    written."""
     n = 4096 + 37
     dt = TORCH_TO_DT[dtype]
     rng = np.random.default_rng(offset)
@@ -109,6 +110,53 @@ def test_pair_unaligned(which, offset, dtype):
         after = storage_np(d)
         np.testing.assert_array_equal(after[:off], h[:off])
         np.testing.assert_array_equal(after[off + n:], h[off + n:])
+
+
+@pytest.mark.parametrize("dtype", DTS)
+def test_pair_every_shared_offset(dtype, packing_mode):
+    """theta, plus and minus all views at the same element offset (every
+    offset off the 32-byte grid; fp32 also at offset 0): the aligned-chunk
+    pair kernel, bit for bit the oracle, nothing outside the views written."""
+    per = 32 // torch.tensor([], dtype=dtype).element_size()
+    offsets = list(range(1, per)) + ([0] if dtype == torch.float32 else [])
+    sizes = [1, 3, 15, 16, 17, 100, 4096 + 37, 20011]
+    dt = TORCH_TO_DT[dtype]
+    rng = np.random.default_rng(per)
+    theta, plus, minus, host, guards = [], [], [], [], []
+    for i, off in enumerate(offsets):
+        n = sizes[i % len(sizes)]
+        for lst in (theta, plus, minus):
+            h = W.random_storage(rng, off + n + 40, dt)
+            b = to_torch(h, dtype)
+            guards.append((h, b, off, n))
+            lst.append(b[off:off + n])
+        host.append(storage_np(theta[-1]).copy())
+    seed = W.step_seed(12)
+    zo.perturb_pair(theta, plus, minus, seed, 29, 1e-3)
+    want_p, want_m = expect(host, [dt] * len(host), seed, 29, 1e-3)
+    assert_equal(plus, want_p, "plus")
+    assert_equal(minus, want_m, "minus")
+    assert_equal(theta, host, "theta untouched")
+    for h, b, off, n in guards[0::3]:                   # theta's allocations: untouched entirely
+        np.testing.assert_array_equal(storage_np(b), h)
+    for h, b, off, n in guards[1::3] + guards[2::3]:    # outputs: nothing outside the views
+        after = storage_np(b)
+        np.testing.assert_array_equal(after[:off], h[:off])
+        np.testing.assert_array_equal(after[off + n:], h[off + n:])
+
+
+def test_pair_many_fp32_tensors(packing_mode):
+    """More fp32 tensors in one launch than one chunk-kernel launch takes
+    (512): the host splits them."""
+    rng = np.random.default_rng(41)
+    numels = [int(x) for x in rng.integers(0, 90, 1000)]
+    host, dev = make(numels, [torch.float32] * len(numels), seed=41)
+    plus, minus = like(dev, 11), like(dev, 12)
+    seed = W.step_seed(13)
+    zo.perturb_pair(dev, plus, minus, seed, 5, 2e-3)
+    want_p, want_m = expect(host, [W.DT_F32] * len(host), seed, 5, 2e-3)
+    assert_equal(plus, want_p, "plus")
+    assert_equal(minus, want_m, "minus")
 
 
 def test_pair_split_launches(packing_mode):
