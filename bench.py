@@ -315,6 +315,12 @@ def run_zo(args):
     params = W.allocate_params(ps, device=dev, view_offset=args.view_offset)
     plist = zo.ParamList(params)
     shifted = any(t.data_ptr() % 32 for t in params)   # the perturbation passes use perturb_shift_kernel
+
+    def like_param(t):
+        """A buffer for theta +- eps z_k laid out like t (same offset into its own allocation)."""
+        if not args.view_offset:
+            return torch.empty_like(t)
+        return torch.empty(t.numel() + args.view_offset, dtype=t.dtype, device=t.device)[args.view_offset:]
     traffic_key = args.config + (f"+view{args.view_offset}" if args.view_offset else "")
     n_steps_total = args.warmup + args.steps + (0 if args.no_e2e else args.steps)
     losses_host = [W.synthetic_losses(K, s) for s in range(n_steps_total)]
@@ -325,8 +331,8 @@ def run_zo(args):
     chunks = (len(params) + 1023) // 1024
     pair = args.schedule == "pair"
     if pair:
-        plus = zo.ParamList([torch.empty_like(t) for t in params])
-        minus = zo.ParamList([torch.empty_like(t) for t in params])
+        plus = zo.ParamList([like_param(t) for t in params])
+        minus = zo.ParamList([like_param(t) for t in params])
 
     timing = {"perturb": [], "perturb2": [], "pair": [], "update": [], "precondition": []}
     fused = args.schedule == "fused"
@@ -430,8 +436,8 @@ def run_zo(args):
     if not pair and not args.no_pair:
         free, _ = torch.cuda.mem_get_info(dev)
         if free > 2.05 * d * ps.bytes_per_elem:
-            plus_a = zo.ParamList([torch.empty_like(t) for t in params])
-            minus_a = zo.ParamList([torch.empty_like(t) for t in params])
+            plus_a = zo.ParamList([like_param(t) for t in params])
+            minus_a = zo.ParamList([like_param(t) for t in params])
             ev = []
 
             def pair_step(s, record):
@@ -495,7 +501,8 @@ def run_zo(args):
     # the roofline is reported for the kernel with the largest share of the step
     n1, n2 = (K + 1, K - 1) if fused else ((0, 0) if pair else (3 * K, 0))
     if pair:
-        dom_kernel, dom_ms, dom_launches = "perturb_pair_kernel", pair_ms, K
+        dom_kernel, dom_ms, dom_launches = ("pair_shift_kernel<*> (tensors off the 32-byte grid)" if shifted
+                                            else "perturb_pair_kernel"), pair_ms, K
         traffic = committed_traffic("perturb_pair_kernel", traffic_key)
     elif n2 > 0 and n2 * perturb2_ms > n1 * perturb_ms:
         dom_kernel, dom_ms, dom_launches = ("perturb_shift_kernel<2, *> (zo_perturb2, tensors off the 32-byte grid)"
