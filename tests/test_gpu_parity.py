@@ -543,16 +543,30 @@ def test_perturb2_every_tuned_configuration():
 def test_fused_step_in_a_cuda_graph():
     """Every call of a fused step only enqueues work on the current stream and
     allocates nothing, so a whole step can be captured into a CUDA graph and
-    replayed: the replay matches the oracle's Algorithm 1 order."""
+    replayed (aligned tensors and views off the 32-byte grid): the replay
+    matches the oracle's Algorithm 1 order."""
     K, eps = 4, 1e-3
     host, dev = make_list(MIXED_NUMELS, MIXED_DTYPES, seed=808)
     dts = [TORCH_TO_DT[d] for d in MIXED_DTYPES]
+    rng = np.random.default_rng(809)
+    for dtype, off, n in ((torch.bfloat16, 3, 5000), (torch.float32, 1, 777), (torch.float16, 5, 40)):
+        h = W.random_storage(rng, n, TORCH_TO_DT[dtype])       # views off the 32-byte grid: the chunk kernels
+        v = torch.empty(n + off, dtype=dtype, device="cuda")[off:]
+        v.copy_(to_torch(h, dtype))
+        host.append(h.copy())
+        dev.append(v)
+        dts.append(TORCH_TO_DT[dtype])
+
+    def same_layout(t):
+        off = (t.data_ptr() % 32) // t.element_size()
+        return torch.empty(t.numel() + off, dtype=t.dtype, device="cuda")[off:].copy_(t)
+
     plist = zo.ParamList(dev)
     seed = W.step_seed(808)
     L = torch.tensor(W.synthetic_losses(K, 808), device="cuda")
     c = torch.empty(K, dtype=torch.float64, device="cuda")
     st = torch.zeros(1, dtype=torch.int32, device="cuda")
-    scratch = zo.ParamList([t.clone() for t in dev])           # warm-up outside the capture
+    scratch = zo.ParamList([same_layout(t) for t in dev])      # warm-up outside the capture
     zo.perturb(scratch, seed, 0, eps)
     zo.perturb2(scratch, seed, 0, eps, 1, eps)
     zo.precondition(L, eps, out=(c, st))
