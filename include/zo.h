@@ -42,8 +42,8 @@
  * alignment gives the same results; a tensor whose ptr is not 32-byte aligned
  * is streamed in 32-byte aligned chunks by a second kernel of the same call
  * (zo_perturb, zo_perturb2, zo_update, zo_update_ex, zo_update_sequential;
- * zo_perturb_pair when theta, plus and minus share the offset), otherwise
- * with narrower accesses.
+ * zo_perturb_pair when plus and minus share their offset), otherwise with
+ * narrower accesses.
  *
  * Probes. z_k is Rademacher, one bit per parameter per probe (Sec. 2, Sec. 4.3
  * "Bit-Packed perturbations"; unpack rule of Appendix F: bit 1 -> +1, bit 0 ->

@@ -439,33 +439,39 @@ int32_t fill_pair_table(zo::PairTable& tab, const zo_tensor* theta, const zo_ten
   return t;
 }
 
-// Tensors of a pair launch for pair_shift_kernel: fp32 tensors, and 16-bit
-// tensors not all 32-byte aligned, when the three pointers share their offset
-// from the 32-byte grid (the others keep perturb_pair_kernel's paths).
-// Returns a bit mask of their storage types.
+// Tensors of a pair launch for pair_shift_kernel: fp32 tensors whose three
+// pointers share their offset from the 32-byte grid, and 16-bit tensors not
+// all 32-byte aligned whose plus and minus share theirs (theta may sit at
+// another, the "moved" kernel); the others keep perturb_pair_kernel's paths.
+// Returns a bit mask of (storage type, moved) classes: bit dt + 3 * moved.
+bool pair_moved(const zo::PairTable& tab, int i) { return tab.src[i] % 32 != tab.plus[i] % 32; }
+
 unsigned mark_pair_shift(zo::PairTable& tab, bool* main_work) {
-  unsigned types = 0;
+  unsigned classes = 0;
   *main_work = false;
   for (int i = 0; i < tab.n; ++i) {
     const uint32_t begin = i == 0 ? 0u : tab.blk_end[i - 1];
     if (tab.blk_end[i] == begin) continue;  // empty
     const uint8_t dt = tab.flags[i] & zo::kDtypeMask;
-    const bool same = tab.src[i] % 32 == tab.plus[i] % 32 && tab.src[i] % 32 == tab.minus[i] % 32;
-    if (same && (dt == zo::kF32 || !(tab.flags[i] & zo::kVec32))) {
+    const bool outs = tab.plus[i] % 32 == tab.minus[i] % 32;
+    const bool moved = pair_moved(tab, i);
+    const bool take = dt == zo::kF32 ? (outs && !moved) : (outs && !(tab.flags[i] & zo::kVec32));
+    if (take) {
       tab.flags[i] |= zo::kShift;
-      types |= 1u << dt;
+      classes |= 1u << (dt + 3 * (moved ? 1 : 0));
     } else {
       *main_work = true;
     }
   }
-  return types;
+  return classes;
 }
 
 thread_local zo::PairShiftParams tl_pair_shift;
 
-// Launch pair_shift_kernel over the flagged tensors of type dt (in batches of
-// kMaxPairShift entries).
-int run_pair_shift(const zo::PairParams& pp, uint8_t dt, DeviceInfo* d, cudaStream_t s) {
+// Launch pair_shift_kernel over the flagged tensors of type dt whose theta
+// is (moved) or is not at another offset than the outputs, in batches of
+// kMaxPairShift entries.
+int run_pair_shift(const zo::PairParams& pp, uint8_t dt, bool moved, DeviceInfo* d, cudaStream_t s) {
   zo::PairShiftParams& S = tl_pair_shift;
   S.keys = pp.keys;
   S.op = pp.op;
@@ -477,10 +483,10 @@ int run_pair_shift(const zo::PairParams& pp, uint8_t dt, DeviceInfo* d, cudaStre
     uint32_t groups = 0;
     for (; i < tab.n && S.n < zo::kMaxPairShift; ++i) {
       const uint8_t fl = tab.flags[i];
-      if (!(fl & zo::kShift) || (fl & zo::kDtypeMask) != dt) continue;
+      if (!(fl & zo::kShift) || (fl & zo::kDtypeMask) != dt || pair_moved(tab, i) != moved) continue;
       const uint32_t begin = i == 0 ? 0u : tab.blk_end[i - 1];
       const int64_t numel = static_cast<int64_t>(tab.blk_end[i] - begin - 1) * 16 + tab.last[i];
-      const int64_t a = static_cast<int64_t>(tab.src[i] % 32) / esz;
+      const int64_t a = static_cast<int64_t>(tab.plus[i] % 32) / esz;  // chunks follow the outputs
       const int64_t chunks = (numel + a + 15) / 16;
       const int j = S.n++;
       S.src[j] = tab.src[i];
@@ -495,7 +501,7 @@ int run_pair_shift(const zo::PairParams& pp, uint8_t dt, DeviceInfo* d, cudaStre
     S.grp_total = groups;
     const int64_t want = (static_cast<int64_t>(groups) * 32 + zo::kThreads - 1) / zo::kThreads;
     const int64_t cap = static_cast<int64_t>(d->sms) * kShiftBlocksPerSm;
-    cudaError_t e = zo::launch_pair_shift(S, dt, static_cast<int>(want < cap ? want : cap), s);
+    cudaError_t e = zo::launch_pair_shift(S, dt, moved, static_cast<int>(want < cap ? want : cap), s);
     if (e != cudaSuccess) return cuda_fail(e, "pair_shift_kernel");
   }
   return ZO_OK;
@@ -606,9 +612,10 @@ int zo_perturb_pair(const zo_tensor* theta, const zo_tensor* plus, const zo_tens
                                                 static_cast<cudaStream_t>(stream));
         if (e != cudaSuccess) return cuda_fail(e, "perturb_pair_kernel");
       }
-      for (uint8_t dt = 0; dt < 3; ++dt) {
-        if (!(shift_types & (1u << dt))) continue;
-        if ((rc = run_pair_shift(pp, dt, d, static_cast<cudaStream_t>(stream))) != ZO_OK) return rc;
+      for (unsigned cls = 0; cls < 6; ++cls) {
+        if (!(shift_types & (1u << cls))) continue;
+        const uint8_t dt = static_cast<uint8_t>(cls % 3);
+        if ((rc = run_pair_shift(pp, dt, cls >= 3, d, static_cast<cudaStream_t>(stream))) != ZO_OK) return rc;
       }
     }
     blk += nb;

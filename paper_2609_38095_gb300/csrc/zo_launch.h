@@ -21,7 +21,8 @@ cudaError_t launch_perturb(const PerturbParams& p, int grid, int loop, bool f32v
 // dt: the storage type of the tensors grp_end counts (one launch per type).
 cudaError_t launch_perturb_shift(const ShiftParams& p, uint8_t dt, int grid, cudaStream_t stream);
 cudaError_t launch_perturb_pair(const PairParams& p, int grid, cudaStream_t stream);
-cudaError_t launch_pair_shift(const PairShiftParams& p, uint8_t dt, int grid, cudaStream_t stream);
+// moved: theta at another offset from the 32-byte grid than plus and minus (16-bit only).
+cudaError_t launch_pair_shift(const PairShiftParams& p, uint8_t dt, bool moved, int grid, cudaStream_t stream);
 cudaError_t launch_update(const UpdateParams& p, int grid, cudaStream_t stream);
 cudaError_t launch_update_shift(const UpdateShiftParams& p, uint8_t dt, int grid, cudaStream_t stream);
 cudaError_t update_shift_blocks_per_sm(int groups, int packing, uint8_t dt, int* out);

@@ -10,8 +10,8 @@
 // partial block. The perturbation passes and the update hand tensors that
 // are not 32-byte aligned to perturb_shift_kernel / update_shift_kernel,
 // which work on aligned 32-byte chunks straddling two blocks; the pair pass
-// hands them (and fp32 tensors) to pair_shift_kernel when its three pointers
-// share the offset, and takes narrower accesses otherwise.
+// hands them (and fp32 tensors) to pair_shift_kernel when plus and minus
+// share their offset, and takes narrower accesses otherwise.
 #include "zo_device.cuh"
 
 namespace zo {
@@ -664,7 +664,79 @@ __device__ __forceinline__ void pair_shift_group(const PairShiftParams& S, int t
   }
 }
 
+// Bytes bo .. bo + 31 (bo even, 0..30) of the 64-byte string lo ++ hi.
+__device__ __forceinline__ void window32(const uint32_t (&lo)[8], const uint32_t (&hi)[8], uint32_t bo,
+                                         uint32_t (&out)[8]) {
+  const uint32_t q = bo >> 2, sh = 8u * (bo & 3u);
+  uint32_t e4[12], e2[10], e1[9];
+#pragma unroll
+  for (int i = 0; i < 12; ++i) {
+    const uint32_t a = i < 8 ? lo[i] : hi[i - 8];
+    const uint32_t b = i + 4 < 8 ? lo[i + 4] : hi[i - 4];
+    e4[i] = (q & 4u) ? b : a;
+  }
+#pragma unroll
+  for (int i = 0; i < 10; ++i) e2[i] = (q & 2u) ? e4[i + 2] : e4[i];
+#pragma unroll
+  for (int i = 0; i < 9; ++i) e1[i] = (q & 1u) ? e2[i + 1] : e2[i];
+#pragma unroll
+  for (int i = 0; i < 8; ++i) out[i] = __funnelshift_r(e1[i], e1[i + 1], sh);
+}
+
+// 16-bit tensors whose theta sits at another offset from the 32-byte grid
+// than plus and minus: chunks follow the outputs, and theta's sixteen
+// elements of chunk c are taken from the aligned 32-byte segments of theta
+// that hold them (two, each also read by a neighbouring lane, whose second
+// read hits L1; one when they fill a segment exactly).
 template <uint8_t DT>
+__device__ __forceinline__ void pair_shift_group_moved(const PairShiftParams& S, int t, int64_t c_first) {
+  const PerturbOp& op = S.op;
+  const uintptr_t src = S.src[t];
+  const uint32_t off = static_cast<uint32_t>(S.plus[t] & 31u);  // the outputs' offset, shared by plus and minus
+  const uint32_t a = off / 2, a_src = static_cast<uint32_t>(src & 31u) / 2;
+  // theta element 16c - a sits at position d of theta's aligned segment c + dc
+  const uint32_t d = (a_src + 16u - a) & 15u;
+  const int64_t dc = a_src >= a ? 0 : -1;
+  const char* s0 = reinterpret_cast<const char*>(src - (src & 31u));
+  char* p0 = reinterpret_cast<char*>(S.plus[t] - off);
+  char* m0 = reinterpret_cast<char*>(S.minus[t] - off);
+  const int64_t n = S.numel[t];
+  const int64_t nchunks = (n + a + 15) / 16;
+  const int lane = static_cast<int>(threadIdx.x & 31u);
+#pragma unroll 1
+  for (int s = 0; s < kShiftSub; ++s) {
+    const int64_t c = c_first + s * kShiftLanes + lane - 1;
+    const bool full = lane > 0 && 16 * c >= a && 16 * c - a + 16 <= n;
+    uint32_t lo[8], hi[8];
+    if (full) {  // the second segment only when the sixteen elements reach into it (d > 0)
+      const char* q = s0 + (c + dc) * 32;
+      ld256(q, lo);
+      if (d != 0) {
+        ld256(q + 32, hi);
+      } else {
+#pragma unroll
+        for (int r = 0; r < 8; ++r) hi[r] = lo[r];
+      }
+    }
+    const uint4 x = block_bits(S.vb0[t] + c, op.ctr2, S.keys);
+    const uint4 below = shfl_up4(x);
+    const uint4 y = a == 0 ? x : window16(below, x, 16u - a);
+    if (full) {
+      uint32_t v[8], m[8];
+      window32(lo, hi, 2u * d, v);
+      pair_regs16<DT>(v, y, op, v, m);
+      st256(p0 + c * 32, v);
+      st256(m0 + c * 32, m);
+    } else if (lane > 0 && c >= 0 && c < nchunks) {  // a chunk across an end of the tensor
+      pair_chunk_elements<DT>(reinterpret_cast<const void*>(src), reinterpret_cast<void*>(S.plus[t]),
+                              reinterpret_cast<void*>(S.minus[t]), n, 16 * c - a, y, op);
+    }
+  }
+}
+
+// MOVED: every tensor of the launch has theta at another offset than plus
+// and minus (16-bit only); otherwise all three share it.
+template <uint8_t DT, bool MOVED>
 __global__ void __launch_bounds__(256, 4) pair_shift_kernel(const __grid_constant__ PairShiftParams S) {
   const uint32_t warp = (blockIdx.x * blockDim.x + threadIdx.x) >> 5;
   const uint32_t nwarps = (gridDim.x * blockDim.x) >> 5;
@@ -672,7 +744,10 @@ __global__ void __launch_bounds__(256, 4) pair_shift_kernel(const __grid_constan
   for (uint32_t g = warp; g < S.grp_total; g += nwarps) {  // the same g on every lane of the warp
     while (g >= S.grp_end[t]) ++t;
     const int64_t c_first = static_cast<int64_t>(g - (t == 0 ? 0u : S.grp_end[t - 1])) * kShiftGroup;
-    pair_shift_group<DT>(S, t, c_first);
+    if constexpr (MOVED)
+      pair_shift_group_moved<DT>(S, t, c_first);
+    else
+      pair_shift_group<DT>(S, t, c_first);
   }
 }
 
@@ -1107,13 +1182,17 @@ cudaError_t launch_perturb_shift(const ShiftParams& p, uint8_t dt, int grid, cud
   return cudaGetLastError();
 }
 
-cudaError_t launch_pair_shift(const PairShiftParams& p, uint8_t dt, int grid, cudaStream_t stream) {
-  if (dt == kBF16)
-    pair_shift_kernel<kBF16><<<grid, kThreads, 0, stream>>>(p);
+cudaError_t launch_pair_shift(const PairShiftParams& p, uint8_t dt, bool moved, int grid, cudaStream_t stream) {
+  if (dt == kBF16 && moved)
+    pair_shift_kernel<kBF16, true><<<grid, kThreads, 0, stream>>>(p);
+  else if (dt == kF16 && moved)
+    pair_shift_kernel<kF16, true><<<grid, kThreads, 0, stream>>>(p);
+  else if (dt == kBF16)
+    pair_shift_kernel<kBF16, false><<<grid, kThreads, 0, stream>>>(p);
   else if (dt == kF16)
-    pair_shift_kernel<kF16><<<grid, kThreads, 0, stream>>>(p);
+    pair_shift_kernel<kF16, false><<<grid, kThreads, 0, stream>>>(p);
   else
-    pair_shift_kernel<kF32><<<grid, kThreads, 0, stream>>>(p);
+    pair_shift_kernel<kF32, false><<<grid, kThreads, 0, stream>>>(p);
   return cudaGetLastError();
 }
 

@@ -85,9 +85,10 @@ def test_pair_bit_exact_mixed(k, scale, packing_mode):
 @pytest.mark.parametrize("offset", [1, 8, 16])
 @pytest.mark.parametrize("dtype", [torch.bfloat16, torch.float16, torch.float32])
 def test_pair_unaligned(which, offset, dtype):
-    """One of the three pointers off the 32-byte grid (the others aligned)
-    sends the tensor to the per-block path with the widest accesses each
-    address allows; results are identical and nothing outside the views is
+    """One of the three pointers off the 32-byte grid, the others aligned:
+    theta -> the aligned-chunk kernel with theta read from its segments;
+    plus or minus -> the per-block path with the widest accesses each
+    address allows. Results are identical and nothing outside the views is
     written."""
     n = 4096 + 37
     dt = TORCH_TO_DT[dtype]
@@ -140,6 +141,38 @@ def test_pair_every_shared_offset(dtype, packing_mode):
     for h, b, off, n in guards[0::3]:                   # theta's allocations: untouched entirely
         np.testing.assert_array_equal(storage_np(b), h)
     for h, b, off, n in guards[1::3] + guards[2::3]:    # outputs: nothing outside the views
+        after = storage_np(b)
+        np.testing.assert_array_equal(after[:off], h[:off])
+        np.testing.assert_array_equal(after[off + n:], h[off + n:])
+
+
+@pytest.mark.parametrize("dtype", [torch.bfloat16, torch.float16])
+@pytest.mark.parametrize("out_off", [0, 5])
+def test_pair_theta_at_another_offset(dtype, out_off, packing_mode):
+    """theta at every element offset, plus and minus sharing another one (0:
+    fresh allocations): chunks follow the outputs and theta is read from the
+    aligned segments that hold each chunk's elements; bit for bit the oracle,
+    nothing outside the views written."""
+    sizes = [1, 3, 15, 16, 17, 100, 4096 + 37, 20011]
+    dt = TORCH_TO_DT[dtype]
+    rng = np.random.default_rng(60 + out_off)
+    theta, plus, minus, host, guards = [], [], [], [], []
+    for i, off in enumerate(o for o in range(16) if o != out_off):
+        n = sizes[i % len(sizes)]
+        for lst, o in ((theta, off), (plus, out_off), (minus, out_off)):
+            h = W.random_storage(rng, o + n + 40, dt)
+            b = to_torch(h, dtype)
+            guards.append((h, b, o, n))
+            lst.append(b[o:o + n])
+        host.append(storage_np(theta[-1]).copy())
+    seed = W.step_seed(14)
+    zo.perturb_pair(theta, plus, minus, seed, 30, -1e-3)
+    want_p, want_m = expect(host, [dt] * len(host), seed, 30, -1e-3)
+    assert_equal(plus, want_p, "plus")
+    assert_equal(minus, want_m, "minus")
+    for h, b, off, n in guards[0::3]:
+        np.testing.assert_array_equal(storage_np(b), h)
+    for h, b, off, n in guards[1::3] + guards[2::3]:
         after = storage_np(b)
         np.testing.assert_array_equal(after[:off], h[:off])
         np.testing.assert_array_equal(after[off + n:], h[off + n:])
