@@ -93,6 +93,7 @@ struct DeviceInfo {
   int pair_bps = 0;                       // perturb_pair blocks per SM
   int shift_bps[2][3] = {};               // perturb_shift blocks per SM, by operation count and dtype
   int update_bps[2][zo::kMaxGroups + 1] = {};  // by packing (1, 8) and probe-group count
+  int update_shift_bps[2][3][zo::kMaxGroups + 1] = {};  // update_shift_kernel: packing, dtype, group count
 };
 constexpr int kMaxDevices = 64;
 DeviceInfo g_dev[kMaxDevices];
@@ -131,6 +132,19 @@ int device_info(DeviceInfo** out) {
     d.sms = sms;
   }
   *out = &d;
+  return ZO_OK;
+}
+
+int update_shift_blocks_per_sm(DeviceInfo* d, int groups, int packing, uint8_t dt, int* out) {
+  std::lock_guard<std::mutex> lock(g_dev_mu);
+  int& slot = d->update_shift_bps[packing == zo::kPacking8 ? 1 : 0][dt][groups];
+  if (slot == 0) {
+    int bps = 0;
+    cudaError_t e = zo::update_shift_blocks_per_sm(groups, packing, dt, &bps);
+    if (e != cudaSuccess) return cuda_fail(e, "occupancy(update_shift)");
+    slot = bps > 0 ? bps : 1;
+  }
+  *out = slot;
   return ZO_OK;
 }
 
@@ -675,11 +689,10 @@ int zo_update_ex(const zo_tensor* params, int32_t n_tensors, uint64_t seed, cons
         const uint32_t groups = shift_groups(up.tab, dt, tl_update_shift.grp_end);
         tl_update_shift.grp_total = groups;
         int sbps = 1;
-        cudaError_t e = zo::update_shift_blocks_per_sm(up.groups, up.packing, dt, &sbps);
-        if (e != cudaSuccess) return cuda_fail(e, "occupancy(update_shift)");
+        if ((rc = update_shift_blocks_per_sm(d, up.groups, up.packing, dt, &sbps)) != ZO_OK) return rc;
         const int64_t want = (static_cast<int64_t>(groups) * 32 + zo::kThreads - 1) / zo::kThreads;
-        const int64_t cap = static_cast<int64_t>(d->sms) * (sbps > 0 ? sbps : 1) * kUpdateWaves;
-        e = zo::launch_update_shift(tl_update_shift, dt, static_cast<int>(want < cap ? want : cap), s);
+        const int64_t cap = static_cast<int64_t>(d->sms) * sbps * kUpdateWaves;
+        cudaError_t e = zo::launch_update_shift(tl_update_shift, dt, static_cast<int>(want < cap ? want : cap), s);
         if (e != cudaSuccess) return cuda_fail(e, "update_shift_kernel");
       }
     }
