@@ -160,7 +160,10 @@ int zo_perturb2(const zo_tensor* params, int32_t n_tensors, uint64_t seed, uint3
  * length with the same numel and dtype per entry. plus[t] may be theta[t]
  * itself (then theta becomes theta + scale z) and so may minus[t]; plus[t]
  * and minus[t] must be different, and any other overlap is undefined.
- * The vectorised path needs all three pointers of a tensor 32-byte aligned.
+ * Access paths (same results): 256-bit blocks when all three pointers of a
+ * 16-bit tensor are 32-byte aligned; 32-byte aligned chunks when plus and
+ * minus share their offset from that grid (theta at any offset) and for fp32
+ * tensors whose three pointers share it; narrower accesses otherwise.
  * Errors: ZO_ERR_ARG (also for mismatched lists or plus[t] == minus[t]),
  * ZO_ERR_DTYPE, ZO_ERR_ALIGN, ZO_ERR_CUDA. No counterpart in the paper as a
  * kernel: it trades device memory for HBM traffic. */
