@@ -21,7 +21,8 @@
  * memory: the tensor table travels inside the kernel launch parameters. Its
  * only CUDA objects are the timing events of zo_perturb2's launch
  * configuration choice (18 per parameter list, at most 64 lists, kept until
- * the process exits).
+ * the process exits). Host side, each calling thread keeps its launch
+ * parameter blocks (about 150 KB of thread-local storage).
  *
  * Streams. `stream` is a cudaStream_t (NULL = legacy default stream). Every
  * call only enqueues work on it and returns; results are visible to later
