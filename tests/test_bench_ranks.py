@@ -61,3 +61,21 @@ def test_reference_arm_runs_on_rank0_only(capsys, monkeypatch):
     monkeypatch.setattr(sys, "argv", ["bench.py", "--impl", "reference", "--gpus", "2"])
     bench.run_reference(bench.parse_args())
     assert capsys.readouterr().out == ""
+
+
+def test_reference_arm_line_on_cpu(capsys, monkeypatch):
+    """Rank 0's reference arm (the oracle on the host cores) prints one JSON
+    line with the contract's keys, on a machine without a GPU."""
+    import json
+    monkeypatch.delenv("RANK", raising=False)
+    monkeypatch.setattr(sys, "argv", ["bench.py", "--impl", "reference", "--config", "opt-1.3b", "--steps", "1",
+                                      "--warmup", "1", "--cpu-seconds", "0.4", "--cpu-workers", "2"])
+    bench.run_reference(bench.parse_args())
+    lines = [ln for ln in capsys.readouterr().out.splitlines() if ln.strip()]
+    assert len(lines) == 1
+    d = json.loads(lines[0])
+    assert d["impl"] == "reference" and d["value"] > 0 and d["higher_is_better"] is True
+    for key in ("metric", "unit", "n_gpus", "steps", "warmup", "ms_per_step", "scaling", "dtype", "data", "config"):
+        assert key in d, key
+    assert d["cpu_baseline"]["kind"] == "oracle" and d["cpu_baseline"]["value"] == d["value"]
+    assert d["e2e"] == {"value": d["value"], "unit": d["unit"], "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}
