@@ -20,7 +20,9 @@
  *   probe_bit/bytes      pinned: brute force unpack rule (Appendix F layout),
  *                        statistics.
  *   dtype conversions    pinned: numpy float16 and torch bfloat16 casts, on
- *                        edge cases and (property tests) arbitrary fp32 bits.
+ *                        edge cases and (property tests) arbitrary fp32 bits;
+ *                        NaN results in the one encoding read above (NaN-ness
+ *                        pinned against numpy, the encoding is a reading).
  *   perturb              pinned: brute force, exact-grid restore identity,
  *                        restore drift bound, numpy fp32 addition (property).
  *   precondition         pinned: worked value of Sec. 6 (|c|=1e8, alpha=0.1),
@@ -214,11 +216,21 @@ static float f32_from_bits(uint32_t u) {
   return f;
 }
 
+/* NaN results. The paper says nothing about NaN weights, and IEEE 754 leaves
+ * the sign and payload of an arithmetic result that is NaN to the
+ * implementation. Reading taken here: a NaN result is stored as the positive
+ * quiet NaN with every payload bit set, in each storage format. */
+#define ORC_NAN_F32 0x7FFFFFFFu
+#define ORC_NAN_16 0x7FFFu
+
+/* Storage bits of an fp32 result (fp32 storage). */
+static uint32_t f32_result_bits(float f) { return isnan(f) ? ORC_NAN_F32 : f32_bits(f); }
+
 /* bfloat16 is the upper half of an fp32 bit pattern. */
 float oracle_bf16_to_f32(uint16_t h) { return f32_from_bits((uint32_t)h << 16); }
 
 uint16_t oracle_f32_to_bf16(float f) {
-  if (isnan(f)) return (uint16_t)((f32_bits(f) >> 16) | 0x0040u); /* quiet NaN */
+  if (isnan(f)) return (uint16_t)ORC_NAN_16;
   /* 8 significand bits, fp32's exponent range; max = (2 - 2^-7) * 2^127 */
   double r = round_to_format((double)f, 8, -126, ldexp(2.0 - ldexp(1.0, -7), 127));
   /* r is exactly representable in fp32 (or infinite), so this cast is exact */
@@ -240,8 +252,8 @@ float oracle_f16_to_f32(uint16_t h) {
 }
 
 uint16_t oracle_f32_to_f16(float f) {
+  if (isnan(f)) return (uint16_t)ORC_NAN_16;
   uint16_t sign = (uint16_t)((f32_bits(f) >> 16) & 0x8000u);
-  if (isnan(f)) return (uint16_t)(sign | 0x7E00u);
   double r = round_to_format((double)f, 11, -14, 65504.0);
   double ar = fabs(r);
   if (isinf(r)) return (uint16_t)(sign | 0x7C00u);
@@ -265,7 +277,7 @@ static float load_f32(const void* base, int32_t dtype, int64_t i) {
 /* Store fp32 value v into element i, rounding once to the storage format. */
 static void store_f32(void* base, int32_t dtype, int64_t i, float v) {
   if (dtype == ORC_F32)
-    ((float*)base)[i] = v;
+    ((uint32_t*)base)[i] = f32_result_bits(v);
   else if (dtype == ORC_BF16)
     ((uint16_t*)base)[i] = oracle_f32_to_bf16(v);
   else
@@ -275,17 +287,17 @@ static void store_f32(void* base, int32_t dtype, int64_t i, float v) {
 /* Round a double result straight to the storage format (one rounding). */
 static void store_f64(void* base, int32_t dtype, int64_t i, double v) {
   if (dtype == ORC_F32) {
-    ((float*)base)[i] = (float)v;
+    ((uint32_t*)base)[i] = f32_result_bits((float)v);
   } else if (dtype == ORC_BF16) {
     if (isnan(v)) {
-      ((uint16_t*)base)[i] = 0x7FC0u;
+      ((uint16_t*)base)[i] = (uint16_t)ORC_NAN_16;
       return;
     }
     double r = round_to_format(v, 8, -126, ldexp(2.0 - ldexp(1.0, -7), 127));
     ((uint16_t*)base)[i] = (uint16_t)(f32_bits((float)r) >> 16);
   } else {
     if (isnan(v)) {
-      ((uint16_t*)base)[i] = 0x7E00u;
+      ((uint16_t*)base)[i] = (uint16_t)ORC_NAN_16;
       return;
     }
     double r = round_to_format(v, 11, -14, 65504.0);
@@ -328,7 +340,7 @@ int oracle_perturb_elements(int32_t dtype, int64_t n, const uint64_t* g, const f
     float z = (float)oracle_probe_sign(seed, k, g[j]);
     float r = theta[j] + scale * z;
     if (dtype == ORC_F32)
-      out_bits[j] = f32_bits(r);
+      out_bits[j] = f32_result_bits(r);
     else if (dtype == ORC_BF16)
       out_bits[j] = oracle_f32_to_bf16(r);
     else
@@ -450,7 +462,7 @@ int oracle_update_elements(int32_t dtype, int64_t n, const uint64_t* g, const fl
     for (int32_t k = 0; k < K; ++k) acc += (double)a[k] * (double)oracle_probe_sign(seed, (uint32_t)k, g[j]);
     double v = (double)theta[j] + acc;
     if (dtype == ORC_F32) {
-      out_bits[j] = f32_bits((float)v);
+      out_bits[j] = f32_result_bits((float)v);
     } else {
       uint16_t h;
       store_f64(&h, dtype, 0, v);

@@ -68,38 +68,70 @@ def ulp_storage(x, dt) -> np.ndarray:
     return 2.0 ** (e - 7)
 
 
-def update_bound(got, want, dt, c, lr):
-    """Largest |gpu - oracle| the arithmetic allows for the fused update.
-
-    Oracle: one rounding of theta + A (A = sum_k a_k z_k, exact).
-    Kernel: acc = A + e with |e| <= (H + 2) u S (4-probe partials of 3 fp32
-    adds, H = 2 ceil(K/8) partials added in order, S = sum |a_k|, u = 2^-24);
-    then fp32(theta + acc) (half an fp32 ulp) and, for 16-bit storage, one
-    more rounding (half a storage ulp). Hence
-      |gpu - oracle| <= ulp_s(gpu)/2 + ulp_s(oracle)/2 + ulp32(gpu)/2 + (H+3) u S
-    which is one storage ulp unless theta + A nearly cancels."""
+def update_error(dt, c, lr, want):
+    """Largest |acc32 - A| + half an fp32 ulp of the result that the kernel's
+    arithmetic allows, per element: A = sum_k a_k z_k (the oracle forms it
+    exactly), acc32 the kernel's fp32 sum. Partials of at most four probes
+    (three fp32 adds each) are combined and added in order, at most
+    H = 2 ceil(K/8) additions to the accumulator, so the recursive summation
+    bound gives |acc32 - A| <= (H + 2) u S with S = sum |a_k| and u = 2^-24;
+    fp32(theta + acc32) adds half an fp32 ulp."""
     K = len(c)
     H = 2 * ((K + 7) // 8)
     S = float(np.abs(update_coeffs(c, lr).astype(np.float64)).sum())
-    b = 0.5 * (ulp_storage(got, dt) + ulp_storage(want, dt)) + (H + 3) * 2.0 ** -24 * S
-    if dt != W.DT_F32:
-        b = b + 0.5 * ulp_f32(got)
-    return 1.0001 * b
+    return (H + 2) * 2.0 ** -24 * S + 0.5 * ulp_f32(want)
 
 
-def assert_update_close(got_bits, want_bits, dt, c, lr, context="", min_one_ulp=0.999):
-    """Every element within the derived bound; for bf16 / fp16 storage also at
-    least `min_one_ulp` of the elements within one ulp of the storage format
-    (fp32 storage has no one-ulp bar: its fp32 accumulation error is of the
-    order of an fp32 ulp of sum |a_k|)."""
-    g = bits_to_f64(got_bits, dt)
-    w = bits_to_f64(want_bits, dt)
+def update_bound(got, want, dt, c, lr):
+    """Largest |gpu - oracle| the arithmetic allows for the fused update.
+
+    Oracle: one rounding of theta + A (A exact). Kernel: fp32(theta + acc32),
+    then, for 16-bit storage, one rounding to storage. Hence
+      |gpu - oracle| <= ulp_s(gpu)/2 + ulp_s(oracle)/2 + update_error
+    (fp32 storage: the storage rounding is the fp32 one already counted)."""
+    e = update_error(dt, c, lr, want)
+    if dt == W.DT_F32:
+        return 1.0001 * (0.5 * ulp_f32(want) + e)
+    return 1.0001 * (0.5 * (ulp_storage(got, dt) + ulp_storage(want, dt)) + e)
+
+
+def assert_update_close(got_bits, want_bits, dt, c, lr, context=""):
+    """Fused-update parity against the oracle, element by element.
+
+    NaN where the oracle has NaN, with the same bits. bf16 / fp16 storage:
+    every element within one ulp of the oracle, except in the cancellation
+    band -- elements where half a storage ulp of the oracle's value is below
+    the fp32 summation error (|theta + A| of the order of 2^p times that
+    error), where no fp32 accumulation can promise one storage ulp -- which
+    must meet the derived bound instead. fp32 storage: the derived bound.
+    Returns counts (elements, bit-equal, largest ulp distance, band elements)."""
+    gb = np.asarray(got_bits, dtype=np.uint32)
+    wb = np.asarray(want_bits, dtype=np.uint32)
+    g = bits_to_f64(gb, dt)
+    w = bits_to_f64(wb, dt)
+    nan_w, nan_g = np.isnan(w), np.isnan(g)
+    bad = np.nonzero(nan_w != nan_g)[0]
+    assert bad.size == 0, (context, "NaN mismatch", [(int(i), hex(int(gb[i])), hex(int(wb[i]))) for i in bad[:5]])
+    bad = np.nonzero(nan_w & (gb != wb))[0]
+    assert bad.size == 0, (context, "NaN encoding", [(int(i), hex(int(gb[i])), hex(int(wb[i]))) for i in bad[:5]])
+    fin = ~nan_w
+    g, w, gb, wb = g[fin], w[fin], gb[fin], wb[fin]
     bound = update_bound(g, w, dt, c, lr)
-    bad = np.nonzero(~(np.abs(g - w) <= bound))[0]
+    if dt == W.DT_F32:
+        band = np.ones(g.size, dtype=bool)
+        ulp = np.zeros(g.size, dtype=np.int64)
+    else:
+        band = 0.5 * ulp_storage(w, dt) < update_error(dt, c, lr, w)
+        ulp = ulp_distance16(gb, wb)
+        far = np.nonzero(~band & (ulp > 1))[0]
+        assert far.size == 0, (context, "more than one ulp outside the cancellation band",
+                               [(int(i), hex(int(gb[i])), hex(int(wb[i])), int(ulp[i])) for i in far[:5]])
+    # in the band (every element for fp32 storage) the derived bound; equal
+    # infinities pass (their difference is NaN)
+    bad = np.nonzero(band & ~((np.abs(g - w) <= bound) | (gb == wb)))[0]
     assert bad.size == 0, (context, [(int(i), g[i], w[i], bound[i]) for i in bad[:5]])
-    if dt != W.DT_F32 and g.size >= 1000:   # the one-ulp bar is stated for bf16 / fp16 storage
-        one = ulp_distance16(got_bits, want_bits) <= 1
-        assert np.mean(one) >= min_one_ulp, (context, float(np.mean(one)))
+    return {"n": int(gb.size + np.sum(nan_w)), "equal": int(np.sum(gb == wb) + np.sum(nan_w)),
+            "max_ulp": int(ulp.max()) if ulp.size else 0, "band": int(np.sum(band)) if dt != W.DT_F32 else 0}
 
 
 def sample_positions(numels, n_random=1 << 16, seed=0):
