@@ -65,7 +65,10 @@
  * key), byte m = g mod 16 as above, z_k[g] = +1 if bit 0 of that byte is 1.
  *
  * Arithmetic. Weights are read as fp32, the operation is done in fp32 and the
- * result is rounded once to the storage dtype (round to nearest even).
+ * result is rounded once to the storage dtype (round to nearest even). A NaN
+ * result is stored as the positive quiet NaN with every payload bit set
+ * (0x7FFFFFFF fp32, 0x7FFF bf16 and fp16); infinities and signed zeros follow
+ * IEEE 754.
  */
 #ifndef ZO_H_
 #define ZO_H_
@@ -214,10 +217,13 @@ int zo_precondition_ex(const double* losses, int32_t K, double eps, double alpha
  * Eq. 6, Delta theta = -eta Z W dl), in one read and one write of theta:
  *   a_k   = fp32( (-(lr / K)) * c_k )    (fp64 product, rounded to fp32)
  *   theta <- rn( fp32(theta) + sum_{k<K} a_k z_k )
- * with the sum accumulated in fp32 in increasing probe order, four probes
- * at a time: each 4-probe partial ((s0 a0 + s1 a1) + s2 a2) + s3 a3 is exact
- * up to fp32 rounding and partials are added in order. With lr = eps this is
- * Algorithm 1's gamma_k = g_k w_k / (2n) step, fused over all probes.
+ * with the sum accumulated in fp32, eight probes at a time in increasing
+ * probe order: the partial of probes 8q..8q+7 is the fp32 sum of the 4-probe
+ * partials ((s0 a0 + s1 a1) + s2 a2) + s3 a3 of probes 8q..8q+3 and of
+ * 8q+4..8q+7 (s_j = z of that probe), and these 8-probe partials are added
+ * to the running sum in increasing q (probes K..8*ceil(K/8)-1 have a = 0).
+ * With lr = eps this is Algorithm 1's gamma_k = g_k w_k / (2n) step, fused
+ * over all probes.
  *   c       device, K fp64 coefficients (normally zo_precondition's output)
  *   K       1 .. ZO_MAX_PROBES; probes 0..K-1 of `seed`
  *   lr      step size (the paper ties it to eps)

@@ -19,7 +19,7 @@ BUILD = os.path.join(HERE, "_build", platform.machine())   # objects of this hos
 LIB = os.path.join(HERE, "libzo.so")
 STAMP = LIB + ".arch"   # architecture the library was linked for
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
-SOURCES = ["zo_api.cu", "zo_stream_kernels.cu", "zo_small_kernels.cu"]
+SOURCES = ["zo_api.cu", "zo_stream_kernels.cu", "zo_update_lut8.cu", "zo_small_kernels.cu"]
 HEADERS = ["zo_device.cuh", "zo_launch.h"]
 
 

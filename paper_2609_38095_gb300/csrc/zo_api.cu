@@ -85,6 +85,16 @@ constexpr int kTwoOpBlocksPerSm[kTwoOpCandidates] = {3, 4, 4};
 // eligible than one persistent wave (measured +3 % at K = 64 and 256).
 constexpr int kUpdateWaves = 4;
 
+// Packing-1 updates with up to 48 probe groups take the 8-probe-table kernel
+// (update_lut8_kernel); larger K and packing 8 take update_kernel. Measured
+// on the OPT-1.3B-shaped bf16 set against update_kernel: K = 8 1.08 vs 1.17
+// ms, K = 16 1.34 vs 1.60, K = 64 3.83 vs 4.21, K = 256 12.9 vs 14.7 (same
+// bits); on the OPT-30B-shaped fp16 set at K = 256 292 vs 332 ms.
+#ifndef ZO_LUT8_MIN_GROUPS
+#define ZO_LUT8_MIN_GROUPS 1
+#endif
+constexpr int kLut8MinGroups = ZO_LUT8_MIN_GROUPS;
+
 // Per-device launch facts, filled once per device.
 struct DeviceInfo {
   int sms = 0;
@@ -94,6 +104,7 @@ struct DeviceInfo {
   int shift_bps[2][3] = {};               // perturb_shift blocks per SM, by operation count and dtype
   int update_bps[2][zo::kMaxGroups + 1] = {};  // by packing (1, 8) and probe-group count
   int update_shift_bps[2][3][zo::kMaxGroups + 1] = {};  // update_shift_kernel: packing, dtype, group count
+  int lut8_bps[zo::kMaxGroups + 1] = {};  // update_lut8_kernel, by group count
 };
 constexpr int kMaxDevices = 64;
 DeviceInfo g_dev[kMaxDevices];
@@ -142,6 +153,21 @@ int update_shift_blocks_per_sm(DeviceInfo* d, int groups, int packing, uint8_t d
     int bps = 0;
     cudaError_t e = zo::update_shift_blocks_per_sm(groups, packing, dt, &bps);
     if (e != cudaSuccess) return cuda_fail(e, "occupancy(update_shift)");
+    slot = bps > 0 ? bps : 1;
+  }
+  *out = slot;
+  return ZO_OK;
+}
+
+// Also raises the kernel's dynamic shared-memory limit (once per device and
+// group count, before the first launch).
+int lut8_blocks_per_sm(DeviceInfo* d, int groups, int* out) {
+  std::lock_guard<std::mutex> lock(g_dev_mu);
+  int& slot = d->lut8_bps[groups];
+  if (slot == 0) {
+    int bps = 0;
+    cudaError_t e = zo::lut8_prepare(groups, &bps);
+    if (e != cudaSuccess) return cuda_fail(e, "occupancy(update_lut8)");
     slot = bps > 0 ? bps : 1;
   }
   *out = slot;
@@ -669,8 +695,13 @@ int zo_update_ex(const zo_tensor* params, int32_t n_tensors, uint64_t seed, cons
   up.has_pre = has_pre != 0;
   up.pre = make_op(pre_probe, has_pre != 0 ? pre_scale : 0.0f, up.packing);
   up.status = status;
+  const bool lut8 = zo::lut8_supported(up.groups, up.packing) && up.groups >= kLut8MinGroups;
   int bps = 1;
-  if ((rc = update_blocks_per_sm(d, up.groups, up.packing, &bps)) != ZO_OK) return rc;
+  if (lut8) {
+    if ((rc = lut8_blocks_per_sm(d, up.groups, &bps)) != ZO_OK) return rc;
+  } else if ((rc = update_blocks_per_sm(d, up.groups, up.packing, &bps)) != ZO_OK) {
+    return rc;
+  }
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   int64_t blk = 0;
   for (int32_t t0 = 0; t0 < n_tensors;) {
@@ -679,7 +710,12 @@ int zo_update_ex(const zo_tensor* params, int32_t n_tensors, uint64_t seed, cons
     if (nb > 0) {
       bool main_work = false;
       const unsigned shift_types = mark_shift(up.tab, &main_work);
-      if (main_work) {
+      if (main_work && lut8) {
+        // one CTA per 1024 blocks (its chunk), at most the resident CTAs
+        const int64_t want = (nb + 1023) / 1024, cap = static_cast<int64_t>(d->sms) * bps;
+        cudaError_t e = zo::launch_update_lut8(up, static_cast<int>(want < cap ? want : cap), s);
+        if (e != cudaSuccess) return cuda_fail(e, "update_lut8_kernel");
+      } else if (main_work) {
         cudaError_t e = zo::launch_update(up, grid_for(nb, d->sms, bps * kUpdateWaves), s);
         if (e != cudaSuccess) return cuda_fail(e, "update_kernel");
       }

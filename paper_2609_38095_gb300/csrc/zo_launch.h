@@ -24,6 +24,12 @@ cudaError_t launch_perturb_pair(const PairParams& p, int grid, cudaStream_t stre
 // moved: theta at another offset from the 32-byte grid than plus and minus (16-bit only).
 cudaError_t launch_pair_shift(const PairShiftParams& p, uint8_t dt, bool moved, int grid, cudaStream_t stream);
 cudaError_t launch_update(const UpdateParams& p, int grid, cudaStream_t stream);
+// Fused update with per-lane 8-probe tables (packing 1, up to 48 probe
+// groups): one CTA of 512 threads per SM, two blocks per thread per chunk.
+size_t lut8_smem_bytes(int groups);
+bool lut8_supported(int groups, int packing);
+cudaError_t lut8_prepare(int groups, int* blocks_per_sm);  // sets the shared-memory limit, occupancy
+cudaError_t launch_update_lut8(const UpdateParams& p, int grid, cudaStream_t stream);
 cudaError_t launch_update_shift(const UpdateShiftParams& p, uint8_t dt, int grid, cudaStream_t stream);
 cudaError_t update_shift_blocks_per_sm(int groups, int packing, uint8_t dt, int* out);
 size_t update_smem_bytes(int groups);

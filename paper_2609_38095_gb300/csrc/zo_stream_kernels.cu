@@ -30,15 +30,6 @@ namespace zo {
 // is rounded to storage after each, exactly as two separate passes would,
 // but theta crosses HBM once.
 // ---------------------------------------------------------------------------
-// Probe bit of element i (0..15) of a block, moved to bit 31.
-__device__ __forceinline__ uint32_t sign_bit(const uint4& x, int i, uint32_t j) {
-  return (word_of(x, i >> 2) << (31u - 8u * static_cast<uint32_t>(i & 3) - j)) & 0x80000000u;
-}
-
-__device__ __forceinline__ float add_signed(float th, const uint4& x, int i, const PerturbOp& op) {
-  return __fadd_rn(th, __uint_as_float(op.nscale_bits ^ sign_bit(x, i, op.bit)));
-}
-
 // The same with the sign moved by a multiply (PerturbOp::mul), in the vector
 // loops: it moves half of the sign injection from the integer ALU, the busiest
 // pipe of these loops, to the multiply-add pipe (measured: single-op pass
@@ -49,10 +40,6 @@ __device__ __forceinline__ uint32_t sign_bit_mul(const uint4& x, int i, const Pe
 
 __device__ __forceinline__ float add_signed_mul(float th, const uint4& x, int i, const PerturbOp& op) {
   return __fadd_rn(th, __uint_as_float(op.nscale_bits ^ sign_bit_mul(x, i, op)));
-}
-
-__device__ __forceinline__ uint4 block_bits(int64_t b, uint32_t ctr2, const RoundKeys& keys) {
-  return philox10(static_cast<uint32_t>(b), static_cast<uint32_t>(static_cast<uint64_t>(b) >> 32), ctr2, 0u, keys);
 }
 
 // Sixteen 16-bit weights in registers (element 2r in the low half of v[r]).
@@ -759,9 +746,11 @@ __global__ void __launch_bounds__(256, 4) pair_shift_kernel(const __grid_constan
 //   T[n] = ((s0 a_{4h} + s1 a_{4h+1}) + s2 a_{4h+2}) + s3 a_{4h+3},
 //   s_j = +1 if bit j of n is set, else -1,
 // for probe quad h = 2q, the high nibble the table of quad 2q + 1. Each
-// element adds the two looked-up partials to its fp32 accumulator, quads in
-// increasing order: one shared-memory load and one add per four probes
-// instead of a select and an add per probe. Probes K..8*groups-1 have a = 0.
+// element adds the two looked-up partials (low quad + high quad: the group's
+// 8-probe partial) to its fp32 accumulator, groups in increasing order: one
+// shared-memory load and one add per four probes instead of a select and an
+// add per probe. Probes K..8*groups-1 have a = 0. update_lut8_kernel adds the
+// same 8-probe partials in the same order, so both give the same bits.
 //
 // Shared-memory layout: probe group q owns a 256-byte frame starting on a
 // 256-byte boundary of the shared window; bytes [0, 64) hold the table of
@@ -800,7 +789,7 @@ __device__ __forceinline__ void accumulate_block(float (&acc)[16], int64_t b, co
         const uint32_t sel = 0x7650u | static_cast<uint32_t>(j);  // byte j of the offsets, bytes 1-3 of the frame
         const float tlo = lds_lo(__byte_perm(lo4, frame, sel));
         const float thi = lds_hi(__byte_perm(hi4, frame, sel));
-        acc[4 * m + j] = __fadd_rn(__fadd_rn(acc[4 * m + j], tlo), thi);
+        acc[4 * m + j] = __fadd_rn(acc[4 * m + j], __fadd_rn(tlo, thi));
       }
     }
   }
@@ -835,7 +824,7 @@ __device__ __forceinline__ void accumulate_block_p8(float (&acc)[16], int64_t b,
         const uint32_t sel = 0x7650u | static_cast<uint32_t>(j);
         const float tlo = lds_lo(__byte_perm(lo4[m], frame, sel));
         const float thi = lds_hi(__byte_perm(hi4[m], frame, sel));
-        acc[4 * m + j] = __fadd_rn(__fadd_rn(acc[4 * m + j], tlo), thi);
+        acc[4 * m + j] = __fadd_rn(acc[4 * m + j], __fadd_rn(tlo, thi));
       }
     }
   }
@@ -848,13 +837,6 @@ __device__ __forceinline__ void accumulate_any(float (&acc)[16], int64_t b, cons
     accumulate_block_p8(acc, b, P, lut_base);
   else
     accumulate_block(acc, b, P, lut_base);
-}
-
-// Leading perturbation of zo_update_ex, rounded to storage (16-bit pairs).
-template <uint8_t DT>
-__device__ __forceinline__ uint32_t pre_regs16(uint32_t v, const uint4& xp, int r, const PerturbOp& op) {
-  const float2 f = unpack2<DT>(v);
-  return pack2<DT>(add_signed(f.x, xp, 2 * r, op), add_signed(f.y, xp, 2 * r + 1, op));
 }
 
 // One full, 32-byte aligned block: theta (16-bit) is loaded before the probe

@@ -1,0 +1,311 @@
+// zo_update_lut8.cu -- the fused K-probe update (Sec. 4.2, Eqs. 5-6) with one
+// table lookup per eight probes.
+//
+// theta <- rn(fp32(theta) + sum_k a_k z_k[g]), a_k = fp32(coef_mul * c_k).
+//
+// Byte m of Philox(b, q) carries the signs of probes 8q..8q+7 of element
+// 16b + m (packing 1). For each probe group q the 256-entry table
+//   T8_q[n] = T_lo[n & 15] + T_hi[n >> 4],
+//   T_lo[i] = ((s0 a_{8q} + s1 a_{8q+1}) + s2 a_{8q+2}) + s3 a_{8q+3}  (s_j = +1 iff bit j of i)
+// and T_hi likewise for probes 8q+4..8q+7, holds the group's fp32 partial sum
+// for every sign byte n. An element adds one looked-up value per group, groups
+// in increasing order: one byte-permute (the address), one shared load and one
+// add per eight probes. update_kernel adds exactly these partials in this
+// order (as two 4-probe lookups), so the two kernels give the same bits.
+//
+// Bank conflicts. 32 lanes looking up random bytes of one 256-entry table
+// would collide on the 32 shared-memory banks, so every lane reads its own
+// copy: row n of the replicated region (256 bytes) holds T8[n] once per lane,
+// lane l in word l of one half of the row (bank l), and another group's table
+// in the other half. The lookup address is then
+//   region + 256 n + 128 h + 4 l,
+// with the region on a 64 KB boundary of the shared window: one byte-permute
+// puts the sign byte n under the region's upper half-word and next to the
+// lane's offset 128 h + 4 l.
+//
+// Loop order. The replicated tables of all groups do not fit in shared memory
+// (32 KB per group), so probe groups are the outer loop: a CTA owns a chunk of
+// THREADS * BPT = 1024 consecutive blocks; each thread accumulates its blocks
+// over all groups in registers and then applies the sums to theta (read once,
+// written once). Two regions of 64 KB each hold a pair of groups (one per
+// half): while the lanes look up groups 2p and 2p+1 in one region, they copy
+// the next pair's tables into the other; one barrier per pair separates the
+// two. With one or two groups the first region holds them for the whole
+// launch and the loop has no barrier.
+#include "zo_device.cuh"
+#include "zo_launch.h"
+
+namespace zo {
+
+constexpr uint32_t kLut8Region = 65536;   // 256 rows x 256 bytes: the tables of two groups
+constexpr int kLut8MaxGroups = 48;        // larger K takes update_kernel
+
+// Shared-memory request: two 64 KB regions starting on a 64 KB boundary of
+// the shared window, plus the coefficients (8 per group) and unreplicated
+// tables (1 KB per group), placed in the slack below the first region when
+// they fit there (the window starts a few bytes in), else after the second:
+// 192 KB covers both cases for up to kLut8MaxGroups groups.
+size_t lut8_smem_bytes(int) { return 3 * static_cast<size_t>(kLut8Region) + 16u; }
+
+__device__ __forceinline__ float lds_f32(uint32_t addr) {
+  float v;
+  asm volatile("ld.shared.f32 %0, [%1];" : "=f"(v) : "r"(addr));
+  return v;
+}
+
+__device__ __forceinline__ void sts_f32x4(uint32_t addr, float v) {
+  asm volatile("st.shared.v4.f32 [%0], {%1, %1, %1, %1};" ::"r"(addr), "f"(v) : "memory");
+}
+
+// One 4-probe partial ((s0 a0 + s1 a1) + s2 a2) + s3 a3 for sign nibble i.
+__device__ __forceinline__ float quad_partial(const float* a, uint32_t i) {
+  float s = (i & 1u) ? a[0] : -a[0];
+  s = __fadd_rn(s, (i & 2u) ? a[1] : -a[1]);
+  s = __fadd_rn(s, (i & 4u) ? a[2] : -a[2]);
+  s = __fadd_rn(s, (i & 8u) ? a[3] : -a[3]);
+  return s;
+}
+
+// Copy the tables of groups q (and q + 1 when `two`) into the two halves of a
+// region. Each thread owns the same 16-byte pieces (four lane copies) of 2048 /
+// THREADS rows in every table: row n = p * THREADS / 8 + tid / 8, piece tid mod
+// 8, so eight consecutive threads fill one half row (each quarter-warp store
+// covers 128 contiguous bytes) and every address is a per-thread base plus a
+// constant. All loads are issued before the first store.
+//   src_t  shared address of t8 + 4 * (tid / 8)
+//   dst_t  region + 256 * (tid / 8) + 16 * (tid mod 8)
+template <int THREADS>
+__device__ __forceinline__ void lut8_replicate(uint32_t src_t, uint32_t dst_t, int q, bool two) {
+  constexpr int S = 2048 / THREADS;                // rows per thread and table
+  constexpr uint32_t kRowStep = THREADS / 8;       // rows between a thread's pieces
+  float v0[S], v1[S];
+  const uint32_t s0 = src_t + static_cast<uint32_t>(q) * 1024u;
+#pragma unroll
+  for (int p = 0; p < S; ++p) v0[p] = lds_f32(s0 + p * kRowStep * 4u);
+  if (two) {
+#pragma unroll
+    for (int p = 0; p < S; ++p) v1[p] = lds_f32(s0 + 1024u + p * kRowStep * 4u);
+  }
+#pragma unroll
+  for (int p = 0; p < S; ++p) sts_f32x4(dst_t + p * kRowStep * 256u, v0[p]);
+  if (two) {
+#pragma unroll
+    for (int p = 0; p < S; ++p) sts_f32x4(dst_t + 128u + p * kRowStep * 256u, v1[p]);
+  }
+}
+
+// Add group q's partial of the 16 elements of a block (Philox output x) to acc.
+// frame: the region's upper half-word, 128 h + 4 l in the low byte.
+__device__ __forceinline__ void lut8_lookup(float (&acc)[16], const uint4& x, uint32_t frame) {
+#pragma unroll
+  for (int m = 0; m < 4; ++m) {
+    const uint32_t w = word_of(x, m);
+#pragma unroll
+    for (int j = 0; j < 4; ++j) {
+      // bytes: frame.b0 (lane offset), w.b_j (sign byte -> row), frame.b2, frame.b3 (region)
+      const uint32_t addr = __byte_perm(w, frame, 0x7604u | (static_cast<uint32_t>(j) << 4));
+      acc[4 * m + j] = __fadd_rn(acc[4 * m + j], lds_f32(addr));
+    }
+  }
+}
+
+// A thread's block of the current chunk.
+struct Lut8Block {
+  int64_t b;       // virtual block (Philox counter)
+  int64_t e0;      // first element inside its tensor
+  void* base;      // tensor base pointer
+  int cnt;         // elements of the block (1..16)
+  uint8_t fl;      // tensor flags
+  bool act;        // a block this kernel updates
+  bool vec16;      // full 32-byte aligned block of a 16-bit tensor (theta already in v)
+};
+
+template <uint8_t DT>
+__device__ __forceinline__ void lut8_apply16(uint32_t (&v)[8], const float (&acc)[16], const uint4& xp,
+                                             const UpdateParams& P, bool do_sum) {
+#pragma unroll
+  for (int r = 0; r < 8; ++r) {
+    if (P.has_pre) v[r] = pre_regs16<DT>(v[r], xp, r, P.pre);
+    if (do_sum) {
+      const float2 f = unpack2<DT>(v[r]);
+      v[r] = pack2<DT>(__fadd_rn(f.x, acc[2 * r]), __fadd_rn(f.y, acc[2 * r + 1]));
+    }
+  }
+}
+
+// Apply the leading perturbation (if any) and the probe sums to a block that
+// is not a full, aligned 16-bit one: fp32 blocks and partial last blocks.
+__device__ __forceinline__ void lut8_apply_other(const Lut8Block& k, const float (&acc)[16], const UpdateParams& P,
+                                              bool do_sum) {
+  uint4 xp = make_uint4(0u, 0u, 0u, 0u);
+  if (P.has_pre) xp = block_bits(k.b, P.pre.ctr2, P.keys);
+  const uint8_t dt = k.fl & kDtypeMask;
+  if (dt == kF32 && k.cnt == 16 && (k.fl & kVec32)) {
+    float* p = static_cast<float*>(k.base) + k.e0;
+#pragma unroll
+    for (int half = 0; half < 2; ++half) {
+      uint32_t v[8];
+      ld256(p + 8 * half, v);
+#pragma unroll
+      for (int r = 0; r < 8; ++r) {
+        float th = __uint_as_float(v[r]);
+        if (P.has_pre) th = add_signed(th, xp, 8 * half + r, P.pre);
+        if (do_sum) th = __fadd_rn(th, acc[8 * half + r]);
+        v[r] = __float_as_uint(th);
+      }
+      st256(p + 8 * half, v);
+    }
+    return;
+  }
+#pragma unroll
+  for (int i = 0; i < 16; ++i) {
+    if (i < k.cnt) {
+      float th = load_elem(k.base, dt, k.e0 + i);
+      if (P.has_pre) th = round_to_storage(dt, add_signed(th, xp, i, P.pre));
+      if (do_sum) th = __fadd_rn(th, acc[i]);
+      store_elem(k.base, dt, k.e0 + i, th);
+    }
+  }
+}
+
+template <int THREADS, int BPT>
+__global__ void __launch_bounds__(THREADS, 1) update_lut8_kernel(const __grid_constant__ UpdateParams P) {
+  extern __shared__ __align__(16) unsigned char smem[];
+  __shared__ int skip_s;
+  const int G = P.groups;
+  const int NP = (G + 1) / 2;  // group pairs: groups 2p, 2p + 1 share one region
+  // Two regions on 64 KB boundaries; the coefficients and unreplicated tables
+  // below the first one when they fit there, else after the second.
+  const uint32_t sbase = static_cast<uint32_t>(__cvta_generic_to_shared(smem));
+  const uint32_t region0 = (sbase + kLut8Region - 1u) & ~(kLut8Region - 1u);
+  const uint32_t hdr_bytes = 32u * G + 1024u * G;
+  const uint32_t hdr = region0 - sbase >= hdr_bytes ? sbase : region0 + 2u * kLut8Region;
+  float* a_s = reinterpret_cast<float*>(smem + (hdr - sbase));  // 8 G coefficients
+  float* t8 = a_s + 8 * G;                                      // 256 G partials
+
+  if (threadIdx.x == 0) skip_s = (P.status != nullptr && *P.status != 0);
+  for (int k = threadIdx.x; k < 8 * G; k += THREADS)
+    a_s[k] = k < P.K ? __double2float_rn(P.coef_mul * P.coef[k]) : 0.0f;
+  __syncthreads();
+  const bool skip = skip_s != 0;
+  if (skip && !P.has_pre) return;
+  const bool do_sum = !skip;  // a failed preconditioner still gets the leading perturbation
+  if (do_sum) {
+    for (int e = threadIdx.x; e < 256 * G; e += THREADS) {
+      const float* a = a_s + 8 * (e >> 8);
+      const uint32_t n = static_cast<uint32_t>(e) & 255u;
+      t8[e] = __fadd_rn(quad_partial(a, n & 15u), quad_partial(a + 4, n >> 4));
+    }
+    __syncthreads();
+  }
+  const uint32_t src_t = hdr + 32u * G + 4u * (threadIdx.x >> 3);  // this thread's rows of t8
+  const uint32_t dst_t = 256u * (threadIdx.x >> 3) + 16u * (threadIdx.x & 7u);
+  if (do_sum) {
+    lut8_replicate<THREADS>(src_t, region0 + dst_t, 0, G > 1);
+    __syncthreads();
+  }
+
+  const TensorTable& tab = P.tab;
+  const uint32_t lane = threadIdx.x & 31u;
+  const uint32_t chunk = static_cast<uint32_t>(THREADS * BPT);
+  const uint32_t per_round = gridDim.x * chunk;
+  const uint32_t rounds = (tab.blk_total + per_round - 1u) / per_round;
+  uint32_t cur = 0;  // region holding the current pair (0 or 1)
+  int t[BPT];
+#pragma unroll
+  for (int j = 0; j < BPT; ++j) t[j] = 0;
+
+  for (uint32_t rnd = 0; rnd < rounds; ++rnd) {
+    Lut8Block blk[BPT];
+    uint32_t v[BPT][8];
+    float acc[BPT][16];
+#pragma unroll
+    for (int j = 0; j < BPT; ++j) {
+      const uint32_t bl = (rnd * gridDim.x + blockIdx.x) * chunk + static_cast<uint32_t>(j * THREADS) + threadIdx.x;
+      Lut8Block& k = blk[j];
+      k.act = bl < tab.blk_total;
+      k.vec16 = false;
+      if (k.act) {
+        t[j] = advance_tensor(tab, t[j], bl);
+        k.fl = tab.flags[t[j]];
+        k.act = !(k.fl & kShift);  // unaligned tensors are update_shift_kernel's
+        k.b = tab.blk_base + bl;
+        k.e0 = static_cast<int64_t>(bl - tensor_blk_begin(tab, t[j])) * 16;
+        k.cnt = static_cast<int>(min(static_cast<int64_t>(16), tab.numel[t[j]] - k.e0));
+        k.base = reinterpret_cast<void*>(tab.ptr[t[j]]);
+        k.vec16 = k.act && k.cnt == 16 && (k.fl & kVec32) && (k.fl & kDtypeMask) != kF32;
+        if (k.vec16) ld256(static_cast<uint16_t*>(k.base) + k.e0, v[j]);
+      }
+#pragma unroll
+      for (int i = 0; i < 16; ++i) acc[j][i] = 0.0f;
+    }
+    if (do_sum) {
+      for (int pr = 0; pr < NP; ++pr) {
+        const uint32_t frame = ((region0 + cur * kLut8Region) & 0xFFFF0000u) | (lane << 2);
+        const int q = 2 * pr;
+#pragma unroll
+        for (int j = 0; j < BPT; ++j) {
+          if (blk[j].act) lut8_lookup(acc[j], block_bits(blk[j].b, static_cast<uint32_t>(q), P.keys), frame);
+        }
+        if (q + 1 < G) {
+#pragma unroll
+          for (int j = 0; j < BPT; ++j) {
+            if (blk[j].act)
+              lut8_lookup(acc[j], block_bits(blk[j].b, static_cast<uint32_t>(q + 1), P.keys), frame | 128u);
+          }
+        }
+        if (NP > 1) {
+          // the next pair (wrapping to pair 0 for the next chunk) into the other region
+          const int qn = pr + 1 < NP ? q + 2 : 0;
+          lut8_replicate<THREADS>(src_t, region0 + (cur ^ 1u) * kLut8Region + dst_t, qn, qn + 1 < G);
+          __syncthreads();
+          cur ^= 1u;
+        }
+      }
+    }
+#pragma unroll
+    for (int j = 0; j < BPT; ++j) {
+      const Lut8Block& k = blk[j];
+      if (!k.act) continue;
+      if (k.vec16) {
+        uint4 xp = make_uint4(0u, 0u, 0u, 0u);
+        if (P.has_pre) xp = block_bits(k.b, P.pre.ctr2, P.keys);
+        if ((k.fl & kDtypeMask) == kBF16)
+          lut8_apply16<kBF16>(v[j], acc[j], xp, P, do_sum);
+        else
+          lut8_apply16<kF16>(v[j], acc[j], xp, P, do_sum);
+        st256(static_cast<uint16_t*>(k.base) + k.e0, v[j]);
+      } else {
+        lut8_apply_other(k, acc[j], P, do_sum);
+      }
+    }
+  }
+}
+
+template <int THREADS, int BPT>
+cudaError_t launch_lut8_cfg(const UpdateParams& p, int grid, cudaStream_t stream) {
+  const size_t smem = lut8_smem_bytes(p.groups);
+  static_assert(2048 % THREADS == 0, "replication assumes THREADS divides 2048");
+  update_lut8_kernel<THREADS, BPT><<<grid, THREADS, smem, stream>>>(p);
+  return cudaGetLastError();
+}
+
+template <int THREADS, int BPT>
+cudaError_t lut8_prepare_cfg(int groups, int* blocks_per_sm) {
+  // the limit covers every group count, so later launches with more groups still fit
+  cudaError_t e = cudaFuncSetAttribute(update_lut8_kernel<THREADS, BPT>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                       static_cast<int>(lut8_smem_bytes(kLut8MaxGroups)));
+  const size_t smem = lut8_smem_bytes(groups);
+  if (e != cudaSuccess) return e;
+  return cudaOccupancyMaxActiveBlocksPerMultiprocessor(blocks_per_sm, update_lut8_kernel<THREADS, BPT>, THREADS, smem);
+}
+
+bool lut8_supported(int groups, int packing) { return packing == kPacking1 && groups >= 1 && groups <= kLut8MaxGroups; }
+
+cudaError_t lut8_prepare(int groups, int* blocks_per_sm) { return lut8_prepare_cfg<512, 2>(groups, blocks_per_sm); }
+
+cudaError_t launch_update_lut8(const UpdateParams& p, int grid, cudaStream_t stream) {
+  return launch_lut8_cfg<512, 2>(p, grid, stream);
+}
+
+}  // namespace zo

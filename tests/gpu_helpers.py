@@ -48,7 +48,8 @@ def ulp_distance16(a_bits, b_bits) -> np.ndarray:
 
 
 def ulp_f32(x) -> np.ndarray:
-    return np.spacing(np.abs(np.asarray(x, dtype=np.float32))).astype(np.float64)
+    with np.errstate(over="ignore", invalid="ignore"):   # infinities have no spacing
+        return np.spacing(np.abs(np.asarray(x, dtype=np.float32))).astype(np.float64)
 
 
 def update_coeffs(c, lr):
@@ -62,7 +63,8 @@ def ulp_storage(x, dt) -> np.ndarray:
     if dt == W.DT_F32:
         return ulp_f32(x)
     if dt == W.DT_F16:
-        return np.spacing(x.astype(np.float16)).astype(np.float64)
+        with np.errstate(over="ignore", invalid="ignore"):
+            return np.spacing(x.astype(np.float16)).astype(np.float64)
     # bf16: 8 significand bits, fp32's exponent range
     e = np.floor(np.log2(np.maximum(x, 2.0 ** -126)))
     return 2.0 ** (e - 7)
@@ -71,11 +73,12 @@ def ulp_storage(x, dt) -> np.ndarray:
 def update_error(dt, c, lr, want):
     """Largest |acc32 - A| + half an fp32 ulp of the result that the kernel's
     arithmetic allows, per element: A = sum_k a_k z_k (the oracle forms it
-    exactly), acc32 the kernel's fp32 sum. Partials of at most four probes
-    (three fp32 adds each) are combined and added in order, at most
-    H = 2 ceil(K/8) additions to the accumulator, so the recursive summation
-    bound gives |acc32 - A| <= (H + 2) u S with S = sum |a_k| and u = 2^-24;
-    fp32(theta + acc32) adds half an fp32 ulp."""
+    exactly), acc32 the kernel's fp32 sum: per probe group of eight, two
+    4-probe partials (three fp32 adds each) and their sum, added to the
+    accumulator in group order (ceil(K/8) additions), so the recursive
+    summation bound gives |acc32 - A| <= (ceil(K/8) + 3) u S <= (H + 2) u S
+    with H = 2 ceil(K/8), S = sum |a_k| and u = 2^-24 (the larger H + 2 is
+    used); fp32(theta + acc32) adds half an fp32 ulp."""
     K = len(c)
     H = 2 * ((K + 7) // 8)
     S = float(np.abs(update_coeffs(c, lr).astype(np.float64)).sum())
