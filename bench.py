@@ -13,6 +13,11 @@ replicas: every rank trains its own copy; nothing is exchanged.
 
 --impl reference times the CPU oracle instead (rank 0 only), on a bounded
 prefix sample of the same workload.
+
+--config tiny times the small workload's full step instead (d = 2^20 fp32,
+quadratic loss, K = 8): the clean loss, per probe the loss at theta + eps z
+and at theta - eps z, the preconditioner and the fused update, the losses
+computed on the device; its oracle baseline runs the same steps in full.
 """
 import argparse
 import dataclasses
@@ -50,6 +55,8 @@ def parse_args():
     ap.add_argument("--K", type=int, default=None, help="override the probes per step of --config")
     ap.add_argument("--cpu-seconds", type=float, default=12.0, help="target CPU time of the oracle sample")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--single-thread-seconds", type=float, default=4.0,
+                    help="target CPU time of the single-threaded oracle sample")
     ap.add_argument("--cpu-workers", type=int, default=None,
                     help="oracle worker processes for the CPU baseline (default: one per host core)")
     ap.add_argument("--no-e2e", action="store_true")
@@ -64,8 +71,8 @@ def parse_args():
                          "copies of the weights (K+1 passes, 3 copies in device memory)")
     ap.add_argument("--no-pair", action="store_true",
                     help="skip the extra measurement of the out-of-place pair schedule")
-    ap.add_argument("--sequential", action="store_true",
-                    help="also time Algorithm 1's K sequential passes against the fused update")
+    ap.add_argument("--no-sequential", action="store_true",
+                    help="skip timing Algorithm 1's K sequential update passes against the fused update")
     ap.add_argument("--view-offset", type=int, default=0,
                     help="every parameter a view this many elements into its own allocation (e.g. 1: off the "
                          "32-byte grid, the perturbation passes run the aligned-chunk kernel)")
@@ -82,24 +89,29 @@ def measured_peaks():
 
 def kernel_source_hash():
     h = hashlib.sha256()
-    for f in ("zo_device.cuh", "zo_stream_kernels.cu"):
+    for f in ("zo_device.cuh", "zo_stream_kernels.cu", "zo_update_lut8.cu"):
         with open(os.path.join(ROOT, "paper_2609_38095_gb300", "csrc", f), "rb") as fh:
             h.update(fh.read())
     return h.hexdigest()[:16]
 
 
 def committed_traffic(kernel, config_key):
-    """DRAM bytes per launch from the committed ncu summary, or None when the
-    summary is missing or was taken on a different kernel source."""
+    """(DRAM bytes per launch, how they were obtained) from the committed ncu
+    summary, or (None, reason) when the summary is missing or was taken on a
+    different kernel source."""
     p = os.path.join(ROOT, "profiles", "ncu_traffic.txt")
     if not os.path.exists(p):
-        return None
+        return None, "no ncu summary committed"
     want = kernel_source_hash()
     for line in open(p):
         parts = line.split()
         if len(parts) >= 4 and parts[0] == kernel and parts[1] == config_key and parts[2] == want:
-            return float(parts[3])
-    return None
+            how = parts[4] if len(parts) > 4 else "measured"
+            if how.startswith("scaled-from-"):
+                how = ("one ncu capture of the same kernel on a smaller parameter set, scaled to this launch by "
+                       "the ratio of weights streamed: " + how)
+            return float(parts[3]), how
+    return None, "kernel source changed since the committed ncu capture"
 
 
 # ----------------------------------------------------------------- clocks
@@ -223,6 +235,24 @@ def oracle_block_step(task):
     return time.perf_counter() - t0
 
 
+def cpu_model():
+    """The host CPU's model name (from /proc/cpuinfo; Arm hosts give the
+    implementer and part codes)."""
+    try:
+        info = open("/proc/cpuinfo").read().splitlines()
+    except OSError:
+        return platform.processor() or platform.machine()
+    fields = {}
+    for line in info:
+        if ":" in line:
+            k, v = line.split(":", 1)
+            fields.setdefault(k.strip(), v.strip())
+    if "model name" in fields:
+        return fields["model name"]
+    arm = [f"{k} {fields[k]}" for k in ("CPU implementer", "CPU part", "CPU variant") if k in fields]
+    return (platform.machine() + " " + " ".join(arm)).strip() if arm else platform.machine()
+
+
 def host_cores():
     try:
         return len(os.sched_getaffinity(0))
@@ -259,8 +289,30 @@ def time_oracle(ps, target_s, steps=1, warmup=0, packing=1, workers=None):
     sample = (f"first {M} weights of the first tensor ({ps.shapes[0][0]}) of the {ps.name} set, K={ps.K}, "
               f"split over {P} worker processes ({per} weights each, one per host core): "
               f"{3 * ps.K} perturb passes + preconditioner + fused update per step, by the oracle's "
-              f"element-list routines; wall time of the slowest worker")
+              f"element-list routines; wall time of the slowest worker; value = sample weights x K / time "
+              f"(extrapolated to the whole set at the same rate)")
     return value, dt, M, P, sample
+
+
+def time_oracle_single(ps, target_s, packing=1):
+    """The oracle's full step on one core: a prefix of the first tensor sized
+    for about target_s seconds. Returns (value, weights)."""
+    import oracle
+    oracle.set_packing(packing)
+    t_cal = oracle_block_step((ps.dtype, 0, 2048, ps.K, ps.eps, 0, packing))
+    n = max(16, min(int(2048 * target_s / max(t_cal, 1e-6)) // 16 * 16, ps.numels[0] // 16 * 16))
+    dt = oracle_block_step((ps.dtype, 0, n, ps.K, ps.eps, 1, packing))
+    return n * ps.K / dt / 1e9, n
+
+
+def cpu_baseline_line(ps, args, v, M, cores, sample):
+    """The cpu_baseline object: all host cores, plus one core, the CPU model
+    and how the value was obtained."""
+    st_v, st_n = time_oracle_single(ps, args.single_thread_seconds, packing=args.packing)
+    return {"value": v, "unit": UNIT, "cores": cores, "kind": "oracle", "sample": sample,
+            "extrapolated": True, "sample_weights": M, "cpu_model": cpu_model(),
+            "single_thread": {"value": st_v, "unit": UNIT, "cores": 1, "sample_weights": st_n,
+                              "sample": f"first {st_n} weights of {ps.shapes[0][0]}, one full step, one process"}}
 
 
 def param_set(args):
@@ -286,6 +338,254 @@ def run_reference(args):
         "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
     }
     print(json.dumps(line), flush=True)
+
+
+# ------------------------------------------------- the small workload
+# d = 2^20 fp32 weights, quadratic loss f = 1/2 sum a_i theta_i^2, K = 8,
+# eps = 1e-3, lr = 1e-2: the full step, losses included, timed as a whole.
+L2_FLUSH_BYTES = 256 << 20        # larger than the 129 MB L2
+
+
+def _tiny_oracle_phase(task):
+    """Worker: the probe phase (kind "probes": K x (+eps, loss, -2 eps, loss,
+    +eps) with the partial losses of this slice) or the update phase of one
+    step on weights [lo, hi) held in shared memory."""
+    kind, shm_th, shm_a, n_all, lo, hi, step, K, eps, lr, c = task
+    from multiprocessing import shared_memory
+
+    import oracle
+    th_m = shared_memory.SharedMemory(name=shm_th)
+    a_m = shared_memory.SharedMemory(name=shm_a)
+    try:
+        th = np.ndarray((n_all,), dtype=np.float32, buffer=th_m.buf)[lo:hi]
+        a = np.ndarray((n_all,), dtype=np.float32, buffer=a_m.buf)[lo:hi]
+        g = np.arange(lo, hi, dtype=np.uint64)
+        seed = W.step_seed(step)
+        if kind == "probes":
+            rows = np.zeros((K, 2))
+            l0 = oracle.quadratic_loss(th, a)
+            for k in range(K):
+                for j, sc in enumerate((eps, -2 * eps)):
+                    th[:] = oracle.perturb_elements(W.DT_F32, g, th, seed, k, sc).view(np.float32)
+                    rows[k, j] = oracle.quadratic_loss(th, a)
+                th[:] = oracle.perturb_elements(W.DT_F32, g, th, seed, k, eps).view(np.float32)
+            return l0, rows
+        th[:] = oracle.update_elements(W.DT_F32, g, th, seed, c, lr).view(np.float32)
+        return None
+    finally:
+        del th, a
+        th_m.close()
+        a_m.close()
+
+
+def time_tiny_oracle(steps, workers, K, eps, lr):
+    """The oracle on the whole small workload, `steps` full steps, split by
+    element range over `workers` processes (1 = the plain single-threaded
+    oracle on the whole vector). Returns seconds per step."""
+    import multiprocessing
+    from multiprocessing import shared_memory
+
+    import oracle
+    oracle.lib()
+    th0, a0 = W.tiny_theta(), W.tiny_curvatures()
+    n = th0.size
+    if workers <= 1:
+        host = [th0.copy()]
+        t0 = time.perf_counter()
+        for s in range(steps):
+            seed = W.step_seed(s)
+            l0 = oracle.quadratic_loss(host[0], a0)
+            rows = []
+            for k in range(K):
+                oracle.perturb(host, [W.DT_F32], seed, k, eps)
+                lp = oracle.quadratic_loss(host[0], a0)
+                oracle.perturb(host, [W.DT_F32], seed, k, -2 * eps)
+                lm = oracle.quadratic_loss(host[0], a0)
+                oracle.perturb(host, [W.DT_F32], seed, k, eps)
+                rows.append([lp, lm, l0])
+            rc, c, _, _ = oracle.precondition(np.array(rows), eps)
+            assert rc == oracle.OK
+            oracle.update(host, [W.DT_F32], seed, c, lr)
+        return (time.perf_counter() - t0) / steps
+    shm_th = shared_memory.SharedMemory(create=True, size=n * 4)
+    shm_a = shared_memory.SharedMemory(create=True, size=n * 4)
+    try:
+        np.ndarray((n,), dtype=np.float32, buffer=shm_th.buf)[:] = th0
+        np.ndarray((n,), dtype=np.float32, buffer=shm_a.buf)[:] = a0
+        bounds = np.linspace(0, n // 16, workers + 1).astype(np.int64) * 16
+        bounds[-1] = n
+        ctx = multiprocessing.get_context("spawn")
+        with ctx.Pool(workers) as pool:
+            pool.map(_tiny_oracle_phase, [("update", shm_th.name, shm_a.name, n, 0, 0, 0, K, eps, lr,
+                                           np.zeros(K))] * workers)          # start the workers
+            t0 = time.perf_counter()
+            for s in range(steps):
+                parts = pool.map(_tiny_oracle_phase, [("probes", shm_th.name, shm_a.name, n, int(lo), int(hi), s,
+                                                       K, eps, lr, None) for lo, hi in zip(bounds[:-1], bounds[1:])])
+                l0 = sum(p[0] for p in parts)
+                rows = np.zeros((K, 3))
+                rows[:, :2] = sum(p[1] for p in parts)
+                rows[:, 2] = l0
+                rc, c, _, _ = oracle.precondition(rows, eps)
+                assert rc == oracle.OK
+                pool.map(_tiny_oracle_phase, [("update", shm_th.name, shm_a.name, n, int(lo), int(hi), s, K, eps,
+                                               lr, c) for lo, hi in zip(bounds[:-1], bounds[1:])])
+            return (time.perf_counter() - t0) / steps
+    finally:
+        shm_th.close()
+        shm_th.unlink()
+        shm_a.close()
+        shm_a.unlink()
+
+
+def tiny_cpu_baseline(args, K, eps, lr, steps):
+    d = 1 << 20
+    cores = max(1, args.cpu_workers or host_cores())
+    st_s = time_tiny_oracle(steps, 1, K, eps, lr)
+    mt_s = time_tiny_oracle(steps, cores, K, eps, lr) if cores > 1 else st_s
+    return {"value": d * K / mt_s / 1e9, "unit": UNIT, "cores": cores, "kind": "oracle", "extrapolated": False,
+            "sample": f"the whole workload, {steps} full steps (every weight), weights split by range over {cores} "
+                      f"worker processes; losses summed from their partial sums", "cpu_model": cpu_model(),
+            "ms_per_step": mt_s * 1e3,
+            "single_thread": {"value": d * K / st_s / 1e9, "unit": UNIT, "cores": 1, "ms_per_step": st_s * 1e3,
+                              "sample": f"the whole workload, {steps} full steps, one process"}}
+
+
+def run_tiny(args):
+    import torch
+    import torch.distributed as dist
+
+    import paper_2609_38095_gb300 as zo
+    from paper_2609_38095_gb300.quadratic import QuadraticStep
+
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    if args.impl == "reference":
+        if rank != 0:
+            return
+        ps = param_set(args)
+        st_s = time_tiny_oracle(args.steps, max(1, args.cpu_workers or host_cores()), ps.K, ps.eps, W.TINY_LR)
+        value = ps.d * ps.K / st_s / 1e9
+        cores = max(1, args.cpu_workers or host_cores())
+        print(json.dumps({
+            "impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": args.gpus,
+            "steps": args.steps, "warmup": 0, "ms_per_step": st_s * 1e3, "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": "f32", "data": "synthetic",
+            "config": {"workload": ps.name, "K": ps.K, "d": ps.d, "lr": W.TINY_LR, "eps": ps.eps},
+            "cpu_baseline": {"value": value, "unit": UNIT, "cores": cores, "kind": "oracle",
+                             "sample": f"the whole workload, {args.steps} full steps", "cpu_model": cpu_model()},
+            "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}), flush=True)
+        return
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    zo.set_packing(args.packing)
+    if world > 1:
+        dist.init_process_group("nccl", device_id=dev)
+    ps = param_set(args)
+    K, eps, lr, d = ps.K, ps.eps, W.TINY_LR, ps.d
+    schedule = "alg1" if args.schedule == "alg1" else "fused"
+    theta = torch.from_numpy(W.tiny_theta()).to(dev)
+    a = torch.from_numpy(W.tiny_curvatures()).to(dev)
+    q = QuadraticStep(theta, a, K, eps, lr, schedule=schedule)
+    stream = torch.cuda.current_stream(dev)
+    flush = torch.empty(L2_FLUSH_BYTES, dtype=torch.uint8, device=dev)
+    for s in range(args.warmup):
+        q.step(W.step_seed(s))
+    # timed steps, L2 flushed before each (the workload's 8 MB would stay in L2)
+    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(args.steps)]
+    host_s = []
+    clocks = ClockSampler(None, args.clocks_csv)
+    clocks.start()
+    dist_barrier(world, dev)
+    for i in range(args.steps):
+        flush.zero_()
+        ev[i][0].record(stream)
+        t0 = time.perf_counter()
+        q.step(W.step_seed(args.warmup + i))
+        host_s.append(time.perf_counter() - t0)
+        ev[i][1].record(stream)
+    dist_barrier(world, dev)
+    clk = clocks.stop()
+    ms_per_step = max_over_ranks(sum(a_.elapsed_time(b_) for a_, b_ in ev) / args.steps, world, dev)
+    launches = q.library_launches_per_step()
+    calls = 2 * K + 1 + (2 * K if schedule == "fused" else 3 * K) + 2     # C-ABI calls per step
+    host_us_per_call = 1e6 * statistics.median(host_s) / calls
+    # the same step replayed from a CUDA graph (no host cost per call)
+    graph_ms = None
+    try:
+        side = torch.cuda.Stream(dev)
+        side.wait_stream(stream)
+        with torch.cuda.stream(side):
+            q.step(W.step_seed(0))                                            # warm on the capture stream
+            g = torch.cuda.CUDAGraph()
+            with torch.cuda.graph(g, stream=side):
+                q.step(W.step_seed(1))
+        stream.wait_stream(side)
+        gev = []
+        for i in range(args.steps):
+            flush.zero_()
+            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            e0.record(stream)
+            g.replay()
+            e1.record(stream)
+            gev.append((e0, e1))
+        torch.cuda.synchronize(dev)
+        graph_ms = sum(x.elapsed_time(y) for x, y in gev) / len(gev)
+    except RuntimeError as e:      # graph capture unavailable: report without it
+        graph_ms = None
+        print(f"graph replay skipped: {e}", file=sys.stderr)
+    # end to end: per step the clean loss and the status read back to the host
+    l0_host = torch.empty(1, dtype=torch.float64).pin_memory()
+    st_host = torch.empty(1, dtype=torch.int32).pin_memory()
+    dist_barrier(world, dev)
+    t0 = time.perf_counter()
+    for i in range(args.steps):
+        q.step(W.step_seed(args.warmup + args.steps + i))
+        l0_host.copy_(q.losses[0, 2:3], non_blocking=True)
+        st_host.copy_(q.status, non_blocking=True)
+        stream.synchronize()
+        if int(st_host[0]) != 0:
+            raise RuntimeError("preconditioner reported non-finite losses")
+    e2e_s = max_over_ranks((time.perf_counter() - t0) / args.steps, world, dev)
+    if rank != 0:
+        if world > 1:
+            dist.destroy_process_group()
+        return
+    peaks, peak_kind = measured_peaks()
+    hbm_peak = float(peaks.get("hbm_gbs", FALLBACK_HBM_GBS))
+    # bytes the step must move: each weight pass reads and writes theta, each
+    # loss reads theta and a
+    passes = 2 * K + 1 if schedule == "fused" else 3 * K + 1
+    step_bytes = passes * 2 * d * 4 + (2 * K + 1) * 2 * d * 4
+    achieved = step_bytes / (ms_per_step * 1e-3) / 1e9
+    cpu = None if args.no_cpu_baseline or world > 1 else tiny_cpu_baseline(args, K, eps, lr, args.steps)
+    line = {
+        "metric": METRIC, "value": world * d * K / (ms_per_step * 1e-3) / 1e9, "unit": UNIT, "n_gpus": world,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms_per_step, "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "f32", "data": "synthetic",
+        "config": {"workload": ps.name, "K": K, "d": d, "eps": eps, "lr": lr, "schedule": schedule,
+                   "loss": "quadratic 1/2 sum a_i theta_i^2 on the device, a_i log-uniform in [1e-2, 1e2]",
+                   "parallelism": f"replicas{world}",
+                   "l2": f"flushed before every timed step ({L2_FLUSH_BYTES >> 20} MB write outside the events)"},
+        "roofline": {"bound": "hbm", "kernel": "whole step (launch-bound: every kernel moves 8 MB or less)",
+                     "achieved": achieved, "peak": hbm_peak, "unit": "GB/s", "frac": achieved / hbm_peak,
+                     "traffic": None, "traffic_source": "not captured for the small workload",
+                     "peak_source": f"{peak_kind} hbm_gbs", "bytes_per_step": step_bytes},
+        "tiny": {"us_per_step": ms_per_step * 1e3, "library_launches_per_step": launches,
+                 "torch_launches_per_step": 1 if K > 1 else 0, "abi_calls_per_step": calls,
+                 "host_us_per_call": host_us_per_call, "host_us_per_step": 1e6 * statistics.median(host_s),
+                 "graph_replay_us_per_step": graph_ms * 1e3 if graph_ms is not None else None},
+        "e2e": {"value": world * d * K / e2e_s / 1e9, "unit": UNIT, "h2d_bytes_per_step": 0,
+                "d2h_bytes_per_step": 12, "ms_per_step": e2e_s * 1e3},
+        "gpu_launches": launches * args.steps,
+        "clocks": clk,
+        "cpu_baseline": cpu,
+        "host": platform.machine(),
+    }
+    print(json.dumps(line), flush=True)
+    if world > 1:
+        dist.destroy_process_group()
 
 
 # ---------------------------------------------------------------- GPU arm
@@ -472,10 +772,9 @@ def run_zo(args):
 
     # ---- Algorithm 1's K-pass update against the fused one (same coefficients)
     seq = None
-    if args.sequential:
-        reps = 2
+    if not args.no_sequential:
+        reps = 1        # the kernels are warm: the sequential passes are zo_perturb's
         ev = [torch.cuda.Event(enable_timing=True) for _ in range(3)]
-        zo.update_sequential(plist, W.step_seed(0), c, eps, status=status)  # warm
         barrier()
         ev[0].record(stream)
         for _ in range(reps):
@@ -503,17 +802,17 @@ def run_zo(args):
     if pair:
         dom_kernel, dom_ms, dom_launches = ("pair_shift_kernel<*> (tensors off the 32-byte grid)" if shifted
                                             else "perturb_pair_kernel"), pair_ms, K
-        traffic = committed_traffic("perturb_pair_kernel", traffic_key)
+        traffic, traffic_how = committed_traffic("perturb_pair_kernel", traffic_key)
     elif n2 > 0 and n2 * perturb2_ms > n1 * perturb_ms:
         dom_kernel, dom_ms, dom_launches = ("perturb_shift_kernel<2, *> (zo_perturb2, tensors off the 32-byte grid)"
                                             if shifted else
                                             "perturb_kernel<2, *> (zo_perturb2, configuration tuned per list)",
                                             perturb2_ms, n2)
-        traffic = committed_traffic("perturb2_kernel", traffic_key)
+        traffic, traffic_how = committed_traffic("perturb2_kernel", traffic_key)
     else:
         dom_kernel, dom_ms, dom_launches = ("perturb_shift_kernel<1, *> (zo_perturb, tensors off the 32-byte grid)"
                                             if shifted else "perturb_kernel<1, 0> (zo_perturb)", perturb_ms, n1)
-        traffic = committed_traffic("perturb_kernel", traffic_key)
+        traffic, traffic_how = committed_traffic("perturb_kernel", traffic_key)
     dom_bytes = pair_bytes if pair else perturb_bytes
     # algorithmic HBM bytes of one step: every pass reads and writes theta once,
     # except the pair passes (read theta, write two copies)
@@ -530,7 +829,7 @@ def run_zo(args):
     cpu = None
     if world == 1 and not args.no_cpu_baseline:
         v, dt, M, cores, sample = time_oracle(ps, args.cpu_seconds, packing=args.packing, workers=args.cpu_workers)
-        cpu = {"value": v, "unit": UNIT, "cores": cores, "kind": "oracle", "sample": sample}
+        cpu = cpu_baseline_line(ps, args, v, M, cores, sample)
     line = {
         "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
         "warmup": args.warmup, "ms_per_step": ms_per_step, "higher_is_better": True, "scaling": "weak",
@@ -543,7 +842,7 @@ def run_zo(args):
                    **({"view_offset": args.view_offset} if args.view_offset else {}),
                    "l2": "inputs larger than L2 (every pass streams the whole parameter set)"},
         "roofline": {"bound": "hbm", "kernel": dom_kernel, "achieved": dom_achieved, "peak": hbm_peak,
-                     "unit": "GB/s", "frac": dom_achieved / hbm_peak, "traffic": traffic,
+                     "unit": "GB/s", "frac": dom_achieved / hbm_peak, "traffic": traffic, "traffic_source": traffic_how,
                      "peak_source": f"{peak_kind} hbm_gbs", "bytes_per_launch": dom_bytes,
                      "launches_per_step": dom_launches * chunks,
                      "step_share": dom_launches * dom_ms / ms_per_step},
@@ -579,7 +878,9 @@ def run_zo(args):
 
 def main():
     args = parse_args()
-    if args.impl == "reference":
+    if args.config == "tiny":
+        run_tiny(args)
+    elif args.impl == "reference":
         run_reference(args)
     else:
         run_zo(args)

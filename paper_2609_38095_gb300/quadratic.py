@@ -1,0 +1,75 @@
+"""One full 1.5-SPSA step on the small synthetic workload, on the device.
+
+Algorithm 1 with the quadratic f(theta) = 1/2 sum_i a_i theta_i^2 standing in
+for the model's forward pass (an ill-conditioned quadratic of the stiff
+paraboloid family, Sec. 5.3): the clean loss L0 once, then per probe k the
+loss at theta + eps z_k and at theta - eps z_k, the preconditioner on the
+K x 3 loss table (Eqs. 3-5) and the fused update (Eq. 6). Every step of it is
+a call of the C ABI; the only other device work is the copy of L0 into the
+table's third column (K doubles).
+
+Schedules (the weights at every forward point and after the step are the
+same bits in both):
+  fused  the restore of probe k and the +eps of probe k+1 in one pass
+         (zo_perturb2), the last restore inside the update pass (zo_update_ex)
+  alg1   Algorithm 1's +eps, -2 eps, +eps passes per probe, then the update
+"""
+import torch
+
+from . import zo
+
+SCHEDULES = ("fused", "alg1")
+
+
+class QuadraticStep:
+    """The device buffers of the workload's step: theta (fp32, updated in
+    place), the curvatures a (fp32), the loss table, coefficients, status and
+    the loss workspace. Nothing is allocated per step."""
+
+    def __init__(self, theta: torch.Tensor, a: torch.Tensor, K: int, eps: float, lr: float, schedule="fused"):
+        if schedule not in SCHEDULES:
+            raise ValueError(f"schedule must be one of {SCHEDULES}")
+        if theta.dtype != torch.float32 or a.dtype != torch.float32 or theta.numel() != a.numel():
+            raise ValueError("theta and a must be fp32 tensors of one size")
+        if theta.device != a.device:
+            raise ValueError("theta and a must live on one device")
+        self.theta, self.a, self.K, self.eps, self.lr, self.schedule = theta, a, int(K), float(eps), float(lr), schedule
+        dev = theta.device
+        self.plist = zo.ParamList([theta])
+        self.losses = torch.empty(self.K, 3, dtype=torch.float64, device=dev)
+        self.c = torch.empty(self.K, dtype=torch.float64, device=dev)
+        self.status = torch.zeros(1, dtype=torch.int32, device=dev)
+        self.ws = torch.empty(zo.quadratic_loss_workspace_size(theta.numel()), dtype=torch.uint8, device=dev)
+
+    def loss(self, out):
+        zo.quadratic_loss(self.theta, self.a, out=out, workspace=self.ws)
+
+    def step(self, seed: int):
+        """Enqueue one step on the current stream (nothing waits)."""
+        K, eps, L = self.K, self.eps, self.losses
+        self.loss(L[0, 2:3])                                   # clean loss L0 (Algorithm 1)
+        if K > 1:
+            L[1:, 2].copy_(L[0:1, 2].expand(K - 1))
+        fused = self.schedule == "fused"
+        if fused:
+            zo.perturb(self.plist, seed, 0, eps)
+        for k in range(K):
+            if not fused:
+                zo.perturb(self.plist, seed, k, eps)
+            self.loss(L[k, 0:1])                               # L+ at theta + eps z_k
+            zo.perturb(self.plist, seed, k, -2 * eps)
+            self.loss(L[k, 1:2])                               # L- at theta - eps z_k
+            if not fused:
+                zo.perturb(self.plist, seed, k, eps)           # restore
+            elif k + 1 < K:
+                zo.perturb2(self.plist, seed, k, eps, k + 1, eps)
+        zo.precondition(L, eps, out=(self.c, self.status))
+        zo.update(self.plist, seed, self.c, self.lr, status=self.status, pre=(K - 1, eps) if fused else None)
+
+    def library_launches_per_step(self) -> int:
+        """Kernels of this library one step launches (the loss is two: partial
+        sums, then their fold)."""
+        K = self.K
+        losses = 2 * (2 * K + 1)
+        passes = 2 * K if self.schedule == "fused" else 3 * K
+        return losses + passes + 2

@@ -79,3 +79,23 @@ def test_reference_arm_line_on_cpu(capsys, monkeypatch):
         assert key in d, key
     assert d["cpu_baseline"]["kind"] == "oracle" and d["cpu_baseline"]["value"] == d["value"]
     assert d["e2e"] == {"value": d["value"], "unit": d["unit"], "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}
+
+
+def test_reference_arm_small_workload_on_cpu(capsys, monkeypatch):
+    """--config tiny --impl reference runs the oracle's full steps on the
+    whole small workload (split over host processes) and prints one line."""
+    monkeypatch.setenv("RANK", "0")
+    monkeypatch.setattr(sys, "argv", ["bench.py", "--impl", "reference", "--config", "tiny", "--steps", "1",
+                                      "--cpu-workers", "2"])
+    bench.main()
+    import json
+    d = json.loads(capsys.readouterr().out.strip().splitlines()[-1])
+    assert d["impl"] == "reference" and d["value"] > 0 and d["config"]["d"] == 1 << 20
+    assert d["cpu_baseline"]["cores"] == 2 and d["e2e"]["value"] == d["value"]
+
+
+def test_cpu_model_and_single_thread_oracle():
+    assert isinstance(bench.cpu_model(), str) and bench.cpu_model()
+    ps = bench.W.OPT_1_3B
+    v, n = bench.time_oracle_single(ps, 0.2)
+    assert v > 0 and n % 16 == 0 and n >= 16
