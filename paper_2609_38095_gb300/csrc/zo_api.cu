@@ -206,21 +206,27 @@ int validate_params(const zo_tensor* params, int32_t n) {
 }
 
 // Fill `tab` with tensors t0, t0+1, ... while the launch holds fewer than
-// kMaxTensorsPerLaunch tensors and fewer than kMaxLaunchBlocks blocks; the
-// launch's first block has virtual index blk_base. Returns the first tensor
-// not taken; *nblocks receives the blocks the launch covers.
+// kMaxTensorsPerLaunch tensors and fewer than kMaxLaunchBlocks launch blocks;
+// the launch's first block has virtual index blk_base. In the launch
+// numbering every tensor starts on a multiple of kLaunchAlign blocks (see
+// TensorTable). Returns the first tensor not taken; *nblocks receives the
+// virtual blocks the launch covers (tab.blk_total its launch blocks).
 int32_t fill_table(TensorTable& tab, const zo_tensor* params, int32_t t0, int32_t n, int64_t blk_base,
                    int64_t* nblocks) {
   tab.n = 0;
   tab.blk_base = blk_base;
-  int64_t b = 0;
+  int64_t b = 0;  // launch blocks so far
+  int64_t v = 0;  // virtual blocks so far
   int32_t t = t0;
   for (; t < n && tab.n < zo::kMaxTensorsPerLaunch; ++t) {
     const zo_tensor& p = params[t];
     const int64_t nb = (p.numel + 15) / 16;
-    if (tab.n > 0 && b + nb >= zo::kMaxLaunchBlocks) break;
+    const int64_t start = (b + zo::kLaunchAlign - 1) / zo::kLaunchAlign * zo::kLaunchAlign;
+    if (tab.n > 0 && start + nb >= zo::kMaxLaunchBlocks) break;
     const int i = tab.n++;
-    b += nb;
+    tab.vdelta[i] = static_cast<uint32_t>(start - v);
+    b = start + nb;
+    v += nb;
     tab.blk_end[i] = static_cast<uint32_t>(b);
     tab.ptr[i] = reinterpret_cast<uint64_t>(p.ptr);
     tab.numel[i] = p.numel;
@@ -229,7 +235,7 @@ int32_t fill_table(TensorTable& tab, const zo_tensor* params, int32_t t0, int32_
     tab.flags[i] = fl;
   }
   tab.blk_total = static_cast<uint32_t>(b);
-  *nblocks = b;
+  *nblocks = v;
   return t;
 }
 
@@ -251,6 +257,13 @@ int grid_for(int64_t blocks, int sms, int bps) {
 // later calls use the candidate with the shortest time. Calls made while the
 // stream is being captured into a graph, or before a decision, use
 // candidate 0.
+// After a failed runtime call of this file's own bookkeeping (events, capture
+// query): reset the thread's last error only when it is that call's error, so
+// an unrelated error the caller has not collected yet stays pending.
+void clear_own_error(cudaError_t e) {
+  if (e != cudaSuccess && cudaPeekAtLastError() == e) cudaGetLastError();
+}
+
 class TwoOpTuner {
  public:
   // Candidate for this call; *slot receives the trial index when the call's
@@ -258,8 +271,9 @@ class TwoOpTuner {
   int pick(uint64_t key, cudaStream_t s, int* slot) {
     *slot = -1;
     cudaStreamCaptureStatus cap = cudaStreamCaptureStatusNone;
-    if (cudaStreamIsCapturing(s, &cap) != cudaSuccess || cap != cudaStreamCaptureStatusNone) {
-      cudaGetLastError();
+    const cudaError_t ce = cudaStreamIsCapturing(s, &cap);
+    if (ce != cudaSuccess || cap != cudaStreamCaptureStatusNone) {
+      clear_own_error(ce);
       return 0;
     }
     std::lock_guard<std::mutex> lock(mu_);
@@ -279,8 +293,9 @@ class TwoOpTuner {
     std::lock_guard<std::mutex> lock(mu_);
     Entry* e = find(key);
     if (e == nullptr || e->ev[slot][which] == nullptr) return;
-    if (cudaEventRecord(e->ev[slot][which], s) != cudaSuccess) {
-      cudaGetLastError();
+    const cudaError_t er = cudaEventRecord(e->ev[slot][which], s);
+    if (er != cudaSuccess) {
+      clear_own_error(er);
       e->failed = true;
     }
   }
@@ -307,8 +322,8 @@ class TwoOpTuner {
     e.key = key;
     for (auto& pair : e.ev)
       for (cudaEvent_t& ev : pair)
-        if (cudaEventCreate(&ev) != cudaSuccess) {
-          cudaGetLastError();
+        if (const cudaError_t ec = cudaEventCreate(&ev); ec != cudaSuccess) {
+          clear_own_error(ec);
           e.chosen = 0;
         }
     entries_.push_back(e);
@@ -323,13 +338,13 @@ class TwoOpTuner {
     if (e.next < kTrials) return;
     float best[kTwoOpCandidates];
     for (int i = 0; i < kTrials; ++i) {
-      if (cudaEventQuery(e.ev[i][1]) != cudaSuccess) {  // not done yet (or failed): decide later
-        cudaGetLastError();
+      if (const cudaError_t q = cudaEventQuery(e.ev[i][1]); q != cudaSuccess) {  // not done yet (or failed)
+        clear_own_error(q);
         return;
       }
       float ms = 0.0f;
-      if (cudaEventElapsedTime(&ms, e.ev[i][0], e.ev[i][1]) != cudaSuccess) {
-        cudaGetLastError();
+      if (const cudaError_t t = cudaEventElapsedTime(&ms, e.ev[i][0], e.ev[i][1]); t != cudaSuccess) {
+        clear_own_error(t);
         e.chosen = 0;
         return;
       }
@@ -432,7 +447,7 @@ int run_perturb(const zo_tensor* params, int32_t n, PerturbParams& pp, DeviceInf
       for (int i = 0; i < pp.tab.n && !f32v; ++i)
         f32v = (pp.tab.flags[i] & zo::kVec32) && (pp.tab.flags[i] & zo::kDtypeMask) == zo::kF32;
       if (main_work) {
-        cudaError_t e = zo::launch_perturb(pp, grid_for(nb, d->sms, bps), loop, f32v, s);
+        cudaError_t e = zo::launch_perturb(pp, grid_for(pp.tab.blk_total, d->sms, bps), loop, f32v, s);
         if (e != cudaSuccess) return cuda_fail(e, "perturb_kernel");
       }
       if (shift_types) tl_shift.p = pp;
@@ -712,11 +727,12 @@ int zo_update_ex(const zo_tensor* params, int32_t n_tensors, uint64_t seed, cons
       const unsigned shift_types = mark_shift(up.tab, &main_work);
       if (main_work && lut8) {
         // one CTA per 1024 blocks (its chunk), at most the resident CTAs
-        const int64_t want = (nb + 1023) / 1024, cap = static_cast<int64_t>(d->sms) * bps;
+        const int64_t want = (static_cast<int64_t>(up.tab.blk_total) + 1023) / 1024;
+        const int64_t cap = static_cast<int64_t>(d->sms) * bps;
         cudaError_t e = zo::launch_update_lut8(up, static_cast<int>(want < cap ? want : cap), s);
         if (e != cudaSuccess) return cuda_fail(e, "update_lut8_kernel");
       } else if (main_work) {
-        cudaError_t e = zo::launch_update(up, grid_for(nb, d->sms, bps * kUpdateWaves), s);
+        cudaError_t e = zo::launch_update(up, grid_for(up.tab.blk_total, d->sms, bps * kUpdateWaves), s);
         if (e != cudaSuccess) return cuda_fail(e, "update_kernel");
       }
       if (shift_types) tl_update_shift.u = up;

@@ -62,12 +62,16 @@ struct Cursor {
   int t;           // tensor index
   uint32_t tb;     // first launch block of tensor t
   uint32_t te;     // one past its last block
-  uint32_t tfe;    // one past its last full block when it takes the pipelined 16-bit path, else tb
-  uint32_t tfe32;  // the same for the pipelined fp32 path of the single-op loop
+  uint32_t n16;    // full blocks from tb on that take the pipelined 16-bit path (0 if it does not)
+  uint32_t n32;    // the same for the pipelined fp32 path of the single-op loop
   uint16_t* tp;    // base pointer
+  uint32_t vd;     // launch block minus virtual block (relative to blk_base) in tensor t
   uint8_t dt;      // storage dtype
 };
 
+// Launch blocks below tb (padding between tensors) give b - tb >= 2^31, so
+// they fail both n16 and n32 tests and go to perturb_block_other, which skips
+// them.
 __device__ __forceinline__ void cursor_seek(const TensorTable& tab, Cursor& c, uint32_t b) {
   c.t = advance_tensor(tab, c.t, b);
   c.tb = tensor_blk_begin(tab, c.t);
@@ -75,10 +79,11 @@ __device__ __forceinline__ void cursor_seek(const TensorTable& tab, Cursor& c, u
   const uint8_t fl = tab.flags[c.t];
   c.dt = fl & kDtypeMask;
   // pipelined path: full, 32-byte aligned blocks of a 16-bit tensor
-  const uint32_t full = c.tb + static_cast<uint32_t>(tab.numel[c.t] / 16);
-  c.tfe = ((fl & kVec32) && c.dt != kF32) ? full : c.tb;
-  c.tfe32 = ((fl & kVec32) && c.dt == kF32) ? full : c.tb;
+  const uint32_t full = static_cast<uint32_t>(tab.numel[c.t] / 16);
+  c.n16 = ((fl & kVec32) && c.dt != kF32) ? full : 0u;
+  c.n32 = ((fl & kVec32) && c.dt == kF32) ? full : 0u;
   c.tp = reinterpret_cast<uint16_t*>(tab.ptr[c.t]);
+  c.vd = tab.vdelta[c.t];
 }
 
 // Any other block: fp32, a partial last block, or an unaligned tensor. One
@@ -90,7 +95,7 @@ template <int NOPS, int TAG>
 __device__ __noinline__ void perturb_block_other(const TensorTable& tab, int t, uint32_t b, uint4 x0, uint4 x1,
                                                  PerturbOp op0, PerturbOp op1) {
   const uint8_t fl = tab.flags[t];
-  if (fl & kShift) return;
+  if ((fl & kShift) || b < tensor_blk_begin(tab, t)) return;  // perturb_shift_kernel's, or padding
   const int64_t e0 = static_cast<int64_t>(b - tensor_blk_begin(tab, t)) * 16;
   const int64_t cnt = min(static_cast<int64_t>(16), tab.numel[t] - e0);
   const uint8_t dt = fl & kDtypeMask;
@@ -168,8 +173,9 @@ enum : int { kBlockOther = 0, kBlock16 = 1, kBlock32 = 2 };
 
 template <bool F32V>
 __device__ __forceinline__ int block_kind(const Cursor& c, uint32_t b) {
-  if (b < c.tfe) return kBlock16;
-  if (F32V && b < c.tfe32) return kBlock32;
+  const uint32_t d = b - c.tb;
+  if (d < c.n16) return kBlock16;
+  if (F32V && d < c.n32) return kBlock32;
   return kBlockOther;
 }
 
@@ -192,6 +198,7 @@ __device__ __forceinline__ void perturb_blocks(const PerturbParams& P, const Per
   uint8_t dt = c.dt;
   int kind = block_kind<F32V>(c, b);
   void* p = block_addr(c, b, kind);
+  uint32_t vd = c.vd;
   uint32_t v[8], w[8];  // the block (16-bit), or its two halves (fp32)
   if (kind != kBlockOther) ld256(p, v);
   if (kind == kBlock32) ld256(static_cast<char*>(p) + 32, w);
@@ -207,7 +214,7 @@ __device__ __forceinline__ void perturb_blocks(const PerturbParams& P, const Per
       if (kindn != kBlockOther) ld256(pn, vn);
       if (kindn == kBlock32) ld256(static_cast<char*>(pn) + 32, wn);
     }
-    const int64_t vb = tab.blk_base + b;  // virtual block: the Philox counter
+    const int64_t vb = tab.blk_base + (b - vd);  // virtual block: the Philox counter
     uint4 x[2];
     x[0] = block_bits(vb, op[0].ctr2, P.keys);
     x[1] = x[0];
@@ -233,6 +240,7 @@ __device__ __forceinline__ void perturb_blocks(const PerturbParams& P, const Per
     b = bn;
     t = c.t;
     dt = c.dt;
+    vd = c.vd;
     kind = kindn;
     p = pn;
 #pragma unroll
@@ -243,30 +251,26 @@ __device__ __forceinline__ void perturb_blocks(const PerturbParams& P, const Per
   }
 }
 
-// Grid-stride by runs: while a thread's next blocks lie in the full, aligned
-// 16-bit region of its current tensor they go through the tight loop of
-// perturb_run16; any other block (fp32, a partial last block, an unaligned
-// tensor) is handled on its own. Fewer instructions per block than
-// perturb_blocks, but the lanes of a warp leave a run up to one iteration
-// apart, which costs most where runs are short (tensors of a few blocks per
-// thread).
-template <int NOPS>
-__device__ __forceinline__ void perturb_runs(const PerturbParams& P, const PerturbOp (&op)[2], bool same_ctr) {
+// By runs: while a thread's next blocks (b, b + stride, ... below end) lie in
+// the full, aligned 16-bit region of its current tensor they go through the
+// tight loop of perturb_run16; any other block (fp32, a partial last block,
+// an unaligned tensor) is handled on its own.
+template <int NOPS, int TAG>
+__device__ __forceinline__ void perturb_runs_range(const PerturbParams& P, const PerturbOp (&op)[2], bool same_ctr,
+                                                   uint32_t b, uint32_t end, uint32_t stride) {
   const TensorTable& tab = P.tab;
-  const uint32_t blk_total = tab.blk_total;
-  const uint32_t stride = gridDim.x * blockDim.x;
-  uint32_t b = blockIdx.x * blockDim.x + threadIdx.x;  // launch-relative; < 2^31 + stride never wraps
   Cursor c;
   c.t = 0;
   bool seeked = false;
-  while (b < blk_total) {
+  while (b < end) {
     if (!seeked || b >= c.te) {
       cursor_seek(tab, c, b);
       seeked = true;
     }
-    const int64_t vb = tab.blk_base + b;  // virtual block: the Philox counter
-    if (b < c.tfe) {
-      const uint32_t n = (c.tfe - b + stride - 1) / stride;  // this thread's blocks in the region
+    const int64_t vb = tab.blk_base + (b - c.vd);  // virtual block: the Philox counter
+    if (b - c.tb < c.n16) {
+      const uint32_t stop = min(c.tb + c.n16, end);
+      const uint32_t n = (stop - b + stride - 1) / stride;  // this thread's blocks in the region
       uint16_t* p = c.tp + static_cast<size_t>(b - c.tb) * 16;
       const size_t pstride = static_cast<size_t>(stride) * 16;
       if (c.dt == kBF16)
@@ -279,10 +283,20 @@ __device__ __forceinline__ void perturb_runs(const PerturbParams& P, const Pertu
       x[0] = block_bits(vb, op[0].ctr2, P.keys);
       x[1] = x[0];
       if (NOPS == 2 && !same_ctr) x[1] = block_bits(vb, op[1].ctr2, P.keys);
-      perturb_block_other<NOPS, kLoopRuns>(tab, c.t, b, x[0], x[1], op[0], op[1]);
+      perturb_block_other<NOPS, TAG>(tab, c.t, b, x[0], x[1], op[0], op[1]);
       b += stride;
     }
   }
+}
+
+// Grid-stride by runs. Fewer instructions per block than perturb_blocks, but
+// the lanes of a warp leave a run up to one iteration apart, which costs
+// most where runs are short (tensors of a few blocks per thread).
+template <int NOPS>
+__device__ __forceinline__ void perturb_runs(const PerturbParams& P, const PerturbOp (&op)[2], bool same_ctr) {
+  const uint32_t stride = gridDim.x * blockDim.x;
+  perturb_runs_range<NOPS, kLoopRuns>(P, op, same_ctr, blockIdx.x * blockDim.x + threadIdx.x, P.tab.blk_total,
+                                      stride);
 }
 
 // LOOP selects perturb_blocks (kLoopBlocks) or perturb_runs (kLoopRuns). The
@@ -368,7 +382,7 @@ __device__ __forceinline__ void shift_group(const PerturbParams& P, const Pertur
   const uint32_t a = static_cast<uint32_t>(ptr & 31u) / kElem;  // 1..15 (16-bit) or 1..7 (fp32)
   char* chunk0 = reinterpret_cast<char*>(ptr - (ptr & 31u));     // 32-byte aligned, a elements before the tensor
   const int64_t nchunks = (n + a + 15) / 16;
-  const int64_t vb0 = tab.blk_base + tensor_blk_begin(tab, t);  // virtual block of element 0
+  const int64_t vb0 = virtual_block(tab, t, tensor_blk_begin(tab, t));  // virtual block of element 0
   const int lane = static_cast<int>(threadIdx.x & 31u);
   int64_t c = c_first + lane - 1;  // lane 0: the block below lane 1's chunk, no chunk of its own
   bool full = shift_full(lane, c, a, n);
@@ -929,8 +943,10 @@ __global__ void __launch_bounds__(256) update_kernel(const __grid_constant__ Upd
   int t = 0;
   for (uint32_t bl = blockIdx.x * blockDim.x + threadIdx.x; bl < tab.blk_total; bl += stride) {
     t = advance_tensor(tab, t, bl);
-    const int64_t e0 = static_cast<int64_t>(bl - tensor_blk_begin(tab, t)) * 16;
-    const int64_t b = tab.blk_base + bl;  // virtual block: the Philox counter
+    const uint32_t tb = tensor_blk_begin(tab, t);
+    if (bl < tb) continue;  // padding between tensors
+    const int64_t e0 = static_cast<int64_t>(bl - tb) * 16;
+    const int64_t b = virtual_block(tab, t, bl);  // the Philox counter
     const int64_t cnt = min(static_cast<int64_t>(16), tab.numel[t] - e0);
     const uint8_t fl = tab.flags[t];
     const uint8_t dt = fl & kDtypeMask;
@@ -999,7 +1015,7 @@ __device__ __forceinline__ void update_shift_group(const UpdateParams& P, uint32
   const uint32_t a = static_cast<uint32_t>(ptr & 31u) / kElem;
   char* chunk0 = reinterpret_cast<char*>(ptr - (ptr & 31u));
   const int64_t nchunks = (n + a + 15) / 16;
-  const int64_t vb0 = tab.blk_base + tensor_blk_begin(tab, t);
+  const int64_t vb0 = virtual_block(tab, t, tensor_blk_begin(tab, t));
   const int lane = static_cast<int>(threadIdx.x & 31u);
 #pragma unroll 1
   for (int s = 0; s < kShiftSub; ++s) {

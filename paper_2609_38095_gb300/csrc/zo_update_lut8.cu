@@ -228,9 +228,11 @@ __global__ void __launch_bounds__(THREADS, 1) update_lut8_kernel(const __grid_co
       if (k.act) {
         t[j] = advance_tensor(tab, t[j], bl);
         k.fl = tab.flags[t[j]];
-        k.act = !(k.fl & kShift);  // unaligned tensors are update_shift_kernel's
-        k.b = tab.blk_base + bl;
-        k.e0 = static_cast<int64_t>(bl - tensor_blk_begin(tab, t[j])) * 16;
+        const uint32_t tb = tensor_blk_begin(tab, t[j]);
+        // unaligned tensors are update_shift_kernel's; blocks below tb are padding
+        k.act = !(k.fl & kShift) && bl >= tb;
+        k.b = virtual_block(tab, t[j], bl);
+        k.e0 = static_cast<int64_t>(bl - tb) * 16;
         k.cnt = static_cast<int>(min(static_cast<int64_t>(16), tab.numel[t[j]] - k.e0));
         k.base = reinterpret_cast<void*>(tab.ptr[t[j]]);
         k.vec16 = k.act && k.cnt == 16 && (k.fl & kVec32) && (k.fl & kDtypeMask) != kF32;

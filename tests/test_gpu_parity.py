@@ -516,10 +516,10 @@ def test_perturb2_is_two_perturbs(a, b, packing_mode):
 
 
 def test_perturb2_every_tuned_configuration():
-    """zo_perturb2 times its candidate configurations (three rounds) on the
-    first calls for a parameter list, then keeps the fastest: 12 calls on one
-    list run every candidate and the chosen one, each bit-exact with the
-    oracle."""
+    """zo_perturb2 times its three candidate configurations (three rounds) on
+    the first nine calls for a parameter list, then keeps the fastest: 12
+    calls on one list run every candidate and the chosen one, each bit-exact
+    with the oracle."""
     rng = np.random.default_rng(606)
     numels = [int(x) for x in rng.integers(1, 70000, 40)] + [4096 * 300, 17]
     dtypes = [DTS[int(x)] for x in rng.integers(0, 3, len(numels))]
