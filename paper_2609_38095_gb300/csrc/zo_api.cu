@@ -187,13 +187,19 @@ int update_blocks_per_sm(DeviceInfo* d, int groups, int packing, int* out) {
   return ZO_OK;
 }
 
-int validate_params(const zo_tensor* params, int32_t n) {
+// Checks a parameter list; *packing (optional) receives the probe packing
+// its tensors ask for (zo_tensor.packing: 0 = the process default, else 1
+// or 8, the same for every tensor of the list) resolved to 1 or 8.
+int validate_params(const zo_tensor* params, int32_t n, int* packing = nullptr) {
   if (n < 0) return ZO_ERR_ARG;
   if (n > 0 && params == nullptr) return ZO_ERR_ARG;
   int64_t blocks = 0;
+  const int32_t pk = n > 0 ? params[0].packing : 0;
+  if (pk != 0 && pk != zo::kPacking1 && pk != zo::kPacking8) return ZO_ERR_ARG;
+  if (packing != nullptr) *packing = pk != 0 ? pk : g_packing.load();
   for (int32_t t = 0; t < n; ++t) {
     const zo_tensor& p = params[t];
-    if (p.numel < 0 || p.reserved != 0) return ZO_ERR_ARG;
+    if (p.numel < 0 || p.packing != pk) return ZO_ERR_ARG;
     if (p.dtype != ZO_F32 && p.dtype != ZO_BF16 && p.dtype != ZO_F16) return ZO_ERR_DTYPE;
     if (p.numel > 0 && p.ptr == nullptr) return ZO_ERR_ARG;
     if (reinterpret_cast<uintptr_t>(p.ptr) % static_cast<uintptr_t>(elem_size(p.dtype)) != 0) return ZO_ERR_ALIGN;
@@ -598,7 +604,8 @@ int zo_get_packing(void) { return g_packing.load(); }
 
 int zo_perturb(const zo_tensor* params, int32_t n_tensors, uint64_t seed, uint32_t probe, float scale,
                void* stream) {
-  int rc = validate_params(params, n_tensors);
+  int packing = zo::kPacking1;
+  int rc = validate_params(params, n_tensors, &packing);
   if (rc != ZO_OK) return rc;
   if (!std::isfinite(scale)) return ZO_ERR_ARG;
   if (n_tensors == 0) return ZO_OK;
@@ -607,7 +614,7 @@ int zo_perturb(const zo_tensor* params, int32_t n_tensors, uint64_t seed, uint32
   PerturbParams& pp = tl_perturb;
   pp.keys = expand_keys(seed);
   pp.probe = probe;
-  pp.op[0] = make_op(probe, scale, g_packing.load());
+  pp.op[0] = make_op(probe, scale, packing);
   pp.op[1] = pp.op[0];
   pp.nops = 1;
   pp.coef = nullptr;
@@ -618,13 +625,13 @@ int zo_perturb(const zo_tensor* params, int32_t n_tensors, uint64_t seed, uint32
 
 int zo_perturb2(const zo_tensor* params, int32_t n_tensors, uint64_t seed, uint32_t probe_a, float scale_a,
                 uint32_t probe_b, float scale_b, void* stream) {
-  int rc = validate_params(params, n_tensors);
+  int packing = zo::kPacking1;
+  int rc = validate_params(params, n_tensors, &packing);
   if (rc != ZO_OK) return rc;
   if (!std::isfinite(scale_a) || !std::isfinite(scale_b)) return ZO_ERR_ARG;
   if (n_tensors == 0) return ZO_OK;
   DeviceInfo* d = nullptr;
   if ((rc = device_info(&d)) != ZO_OK) return rc;
-  const int packing = g_packing.load();
   PerturbParams& pp = tl_perturb;
   pp.keys = expand_keys(seed);
   pp.probe = probe_a;
@@ -639,10 +646,15 @@ int zo_perturb2(const zo_tensor* params, int32_t n_tensors, uint64_t seed, uint3
 
 int zo_perturb_pair(const zo_tensor* theta, const zo_tensor* plus, const zo_tensor* minus, int32_t n_tensors,
                     uint64_t seed, uint32_t probe, float scale, void* stream) {
-  int rc = validate_params(theta, n_tensors);
+  int packing = zo::kPacking1, pk_plus = 0, pk_minus = 0;
+  int rc = validate_params(theta, n_tensors, &packing);
   if (rc != ZO_OK) return rc;
-  if ((rc = validate_params(plus, n_tensors)) != ZO_OK) return rc;
-  if ((rc = validate_params(minus, n_tensors)) != ZO_OK) return rc;
+  if ((rc = validate_params(plus, n_tensors, &pk_plus)) != ZO_OK) return rc;
+  if ((rc = validate_params(minus, n_tensors, &pk_minus)) != ZO_OK) return rc;
+  // plus and minus follow theta's probes: they may name no packing or the same one
+  if (n_tensors > 0 && ((plus[0].packing != 0 && pk_plus != packing) ||
+                        (minus[0].packing != 0 && pk_minus != packing)))
+    return ZO_ERR_ARG;
   if (!std::isfinite(scale)) return ZO_ERR_ARG;
   for (int32_t t = 0; t < n_tensors; ++t) {
     if (plus[t].numel != theta[t].numel || minus[t].numel != theta[t].numel) return ZO_ERR_ARG;
@@ -654,7 +666,7 @@ int zo_perturb_pair(const zo_tensor* theta, const zo_tensor* plus, const zo_tens
   if ((rc = device_info(&d)) != ZO_OK) return rc;
   zo::PairParams& pp = tl_pair;
   pp.keys = expand_keys(seed);
-  pp.op = make_op(probe, scale, g_packing.load());
+  pp.op = make_op(probe, scale, packing);
   int64_t blk = 0;
   for (int32_t t0 = 0; t0 < n_tensors;) {
     int64_t nb = 0;
@@ -678,8 +690,9 @@ int zo_perturb_pair(const zo_tensor* theta, const zo_tensor* plus, const zo_tens
   return ZO_OK;
 }
 
-static int check_update_args(const zo_tensor* params, int32_t n, const double* c, int32_t K, double lr) {
-  int rc = validate_params(params, n);
+static int check_update_args(const zo_tensor* params, int32_t n, const double* c, int32_t K, double lr,
+                             int* packing) {
+  int rc = validate_params(params, n, packing);
   if (rc != ZO_OK) return rc;
   if (K < 1) return ZO_ERR_ARG;
   if (K > ZO_MAX_PROBES) return ZO_ERR_TOO_MANY_PROBES;
@@ -694,7 +707,8 @@ int zo_update(const zo_tensor* params, int32_t n_tensors, uint64_t seed, const d
 
 int zo_update_ex(const zo_tensor* params, int32_t n_tensors, uint64_t seed, const double* c, int32_t K, double lr,
                  const int32_t* status, int32_t has_pre, uint32_t pre_probe, float pre_scale, void* stream) {
-  int rc = check_update_args(params, n_tensors, c, K, lr);
+  int packing = zo::kPacking1;
+  int rc = check_update_args(params, n_tensors, c, K, lr, &packing);
   if (rc != ZO_OK) return rc;
   if (has_pre != 0 && !std::isfinite(pre_scale)) return ZO_ERR_ARG;
   if (n_tensors == 0) return rc;
@@ -706,7 +720,7 @@ int zo_update_ex(const zo_tensor* params, int32_t n_tensors, uint64_t seed, cons
   up.coef_mul = -(lr / static_cast<double>(K));
   up.K = K;
   up.groups = (K + 7) / 8;
-  up.packing = g_packing.load();
+  up.packing = packing;
   up.has_pre = has_pre != 0;
   up.pre = make_op(pre_probe, has_pre != 0 ? pre_scale : 0.0f, up.packing);
   up.status = status;
@@ -755,7 +769,8 @@ int zo_update_ex(const zo_tensor* params, int32_t n_tensors, uint64_t seed, cons
 
 int zo_update_sequential(const zo_tensor* params, int32_t n_tensors, uint64_t seed, const double* c, int32_t K,
                          double lr, const int32_t* status, void* stream) {
-  int rc = check_update_args(params, n_tensors, c, K, lr);
+  int packing = zo::kPacking1;
+  int rc = check_update_args(params, n_tensors, c, K, lr, &packing);
   if (rc != ZO_OK || n_tensors == 0) return rc;
   DeviceInfo* d = nullptr;
   if ((rc = device_info(&d)) != ZO_OK) return rc;
@@ -765,7 +780,6 @@ int zo_update_sequential(const zo_tensor* params, int32_t n_tensors, uint64_t se
   pp.coef_mul = -(lr / static_cast<double>(K));
   pp.status = status;
   pp.nops = 1;
-  const int packing = g_packing.load();
   for (int32_t k = 0; k < K; ++k) {
     pp.probe = static_cast<uint32_t>(k);
     pp.op[0] = make_op(pp.probe, 0.0f, packing);  // scale read from c on the device

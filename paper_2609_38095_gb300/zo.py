@@ -36,7 +36,7 @@ ZO_QUADRATIC_LOSS_STATIC_MAX_N = 8388608
 
 class zo_tensor(ctypes.Structure):
     _fields_ = [("ptr", ctypes.c_void_p), ("numel", ctypes.c_int64), ("dtype", ctypes.c_int32),
-                ("reserved", ctypes.c_int32)]
+                ("packing", ctypes.c_int32)]
 
 
 class ZoError(RuntimeError):
@@ -141,12 +141,24 @@ def _dev_ptr(t, dtype=None, what="tensor"):
     return ctypes.c_void_p(t.data_ptr())
 
 
+def _same_device(dev, **tensors):
+    """Raise unless every tensor lives on `dev` (the launch runs there)."""
+    for name, t in tensors.items():
+        if isinstance(t, torch.Tensor) and t.device != dev:
+            raise ValueError(f"{name} is on {t.device}, the weights on {dev}")
+
+
 class ParamList:
     """The parameter list of a training step: a fixed, ordered list of CUDA
     tensors, each updated in place. Build it once and pass it to every call of
-    every step: the probes are defined by each element's position in it."""
+    every step: the probes are defined by each element's position in it.
+    packing (1 or 8) fixes the list's probe packing; None follows the process
+    default (set_packing) at each call."""
 
-    def __init__(self, tensors):
+    def __init__(self, tensors, packing=None):
+        if packing not in (None, 1, 8):
+            raise ValueError("packing must be None, 1 or 8")
+        self.packing = packing
         self.tensors = list(tensors)
         n = len(self.tensors)
         arr = (zo_tensor * max(n, 1))()
@@ -165,7 +177,7 @@ class ParamList:
             arr[i].ptr = t.data_ptr()
             arr[i].numel = t.numel()
             arr[i].dtype = DTYPE_CODE[t.dtype]
-            arr[i].reserved = 0
+            arr[i].packing = packing or 0
         self._arr = arr
         self.n = n
         self.device = dev if dev is not None else torch.device("cuda", torch.cuda.current_device())
@@ -305,6 +317,7 @@ def quadratic_loss(theta, a, out=None, workspace=None):
         workspace = torch.empty(quadratic_loss_workspace_size(n), dtype=torch.uint8, device=dev)
     if out.numel() < 1:
         raise ValueError("out must hold one float64")
+    _same_device(dev, a=a, out=out, workspace=workspace)
     with torch.cuda.device(dev):
         rc = _lib().zo_quadratic_loss(_dev_ptr(theta, torch.float32, "theta"), _dev_ptr(a, torch.float32, "a"), n,
                                       _dev_ptr(out, torch.float64, "out"), _dev_ptr(workspace, what="workspace"),
@@ -325,6 +338,7 @@ def quadratic_loss_static(theta, a, out=None):
         out = torch.empty(1, dtype=torch.float64, device=dev)
     if out.numel() < 1:
         raise ValueError("out must hold one float64")
+    _same_device(dev, a=a, out=out)
     with torch.cuda.device(dev):
         rc = _lib().zo_quadratic_loss_static(_dev_ptr(theta, torch.float32, "theta"), _dev_ptr(a, torch.float32, "a"),
                                              n, _dev_ptr(out, torch.float64, "out"), _stream(dev))

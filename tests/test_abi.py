@@ -41,10 +41,10 @@ def test_version_and_strings(L):
     assert L.zo_last_cuda_error() == b""
 
 
-def tensors(*specs):
+def tensors(*specs, packing=0):
     arr = (zo.zo_tensor * len(specs))()
     for i, (ptr, numel, dtype) in enumerate(specs):
-        arr[i].ptr, arr[i].numel, arr[i].dtype, arr[i].reserved = ptr, numel, dtype, 0
+        arr[i].ptr, arr[i].numel, arr[i].dtype, arr[i].packing = ptr, numel, dtype, packing
     return arr
 
 
@@ -62,9 +62,13 @@ def test_perturb_validation(L):
     assert L.zo_perturb(tensors((FAKE, -1, 1)), 1, 1, 0, 1e-3, None) == zo.ZO_ERR_ARG
     assert L.zo_perturb(ok, 1, 1, 0, float("nan"), None) == zo.ZO_ERR_ARG
     assert L.zo_perturb(ok, 1, 1, 0, float("inf"), None) == zo.ZO_ERR_ARG
-    bad_res = tensors((FAKE, 16, 1))
-    bad_res[0].reserved = 1
-    assert L.zo_perturb(bad_res, 1, 1, 0, 1e-3, None) == zo.ZO_ERR_ARG
+    for bad in (2, 3, -1, 16):
+        assert L.zo_perturb(tensors((FAKE, 16, 1), packing=bad), 1, 1, 0, 1e-3, None) == zo.ZO_ERR_ARG
+    mixed = tensors((FAKE, 16, 1), (FAKE + 64, 16, 1), packing=8)
+    mixed[1].packing = 1                     # every tensor of a list names the same packing
+    assert L.zo_perturb(mixed, 2, 1, 0, 1e-3, None) == zo.ZO_ERR_ARG
+    mixed[1].packing = 0
+    assert L.zo_perturb(mixed, 2, 1, 0, 1e-3, None) == zo.ZO_ERR_ARG
     assert L.zo_perturb(None, 0, 1, 0, 1e-3, None) == zo.ZO_OK  # empty list: nothing to do
 
 
@@ -82,6 +86,17 @@ def test_perturb_pair_validation(L):
     assert f(th, pl, tensors((FAKE + 16385, 16, 1), (FAKE + 32768, 40, 2)), 2, 1, 0, 1e-3, None) == zo.ZO_ERR_ALIGN
     assert f(th, pl, tensors((FAKE + 16384, 16, 3), (FAKE + 32768, 40, 2)), 2, 1, 0, 1e-3, None) == zo.ZO_ERR_DTYPE
     assert f(None, None, None, 0, 1, 0, 1e-3, None) == zo.ZO_OK
+    # plus / minus follow theta's probes: no packing of their own, or theta's
+    th8 = tensors((FAKE, 16, 1), (FAKE + 64, 40, 2), packing=8)
+    pl1 = tensors((FAKE + 4096, 16, 1), (FAKE + 8192, 40, 2), packing=1)
+    assert f(th8, pl1, mi, 2, 1, 0, 1e-3, None) == zo.ZO_ERR_ARG
+    assert f(th, tensors((FAKE + 4096, 16, 1), (FAKE + 8192, 40, 2), packing=8), mi, 2, 1, 0, 1e-3,
+             None) == zo.ZO_ERR_ARG     # theta follows the default (1)
+
+
+def test_param_list_packing_argument():
+    with pytest.raises(ValueError):
+        zo.ParamList([], packing=4)
 
 
 def test_update_validation(L):

@@ -301,6 +301,39 @@ def test_empty_and_zero_length():
     assert_storage_equal(dev, host)
 
 
+def test_lists_with_their_own_packing_in_one_process():
+    """Two parameter lists naming different probe packings, used in turn in
+    one process: each follows its own packing whatever the process default."""
+    dts_t = [torch.bfloat16, torch.float32, torch.float16]
+    host8, dev8 = make_list([4099, 333, 16], dts_t, seed=808)
+    host1, dev1 = make_list([4099, 333, 16], dts_t, seed=808)
+    dts = [TORCH_TO_DT[d] for d in dts_t]
+    l8, l1 = zo.ParamList(dev8, packing=8), zo.ParamList(dev1, packing=1)
+    seed, K = W.step_seed(808), 12
+    c_np = np.random.default_rng(808).normal(0, 5, K)
+    c = torch.tensor(c_np, device="cuda")
+    with zo.packing(8):                       # the default names neither list's packing
+        zo.perturb(l1, seed, 9, 1e-3)
+        zo.perturb2(l1, seed, 3, 1e-3, 11, -1e-3)
+        zo.update(l1, seed, c, 1e-2, pre=(K - 1, 1e-3))
+    with zo.packing(1):
+        zo.perturb(l8, seed, 9, 1e-3)
+        zo.perturb2(l8, seed, 3, 1e-3, 11, -1e-3)
+        zo.update(l8, seed, c, 1e-2, pre=(K - 1, 1e-3))
+    for host, bits in ((host8, 8), (host1, 1)):
+        with oracle.packing(bits):
+            oracle.perturb(host, dts, seed, 9, 1e-3)
+            oracle.perturb(host, dts, seed, 3, 1e-3)
+            oracle.perturb(host, dts, seed, 11, -1e-3)
+            oracle.perturb(host, dts, seed, K - 1, 1e-3)
+            oracle.update(host, dts, seed, c_np, 1e-2)
+    for dev, host in ((dev8, host8), (dev1, host1)):
+        for i, (d, h, dt) in enumerate(zip(dev, host, dts)):
+            assert_update_close(storage_bits(d), storage_bits(h), dt, c_np, 1e-2, context=f"tensor {i}")
+    # the two packings give different probes: the lists really differ
+    assert not np.array_equal(storage_bits(dev8[0]), storage_bits(dev1[0]))
+
+
 # ------------------------------------------------------------------- update
 @pytest.mark.parametrize("K", [1, 3, 8, 13, 64, 256])
 def test_update_within_tolerance(K, packing_mode):
