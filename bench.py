@@ -9,7 +9,11 @@ parameter set (772 tensors, 29.97e9 weights, 60 GB), K = 256.
 
 Metric: Gparam*probe/s = d * K / step time, whole job over all ranks.
 Prints one JSON line (rank 0). Multi-GPU runs (torchrun) are independent
-replicas: every rank trains its own copy; nothing is exchanged.
+replicas by default: every rank trains its own copy; nothing is exchanged.
+--probe-parallel runs the paper's probe-parallel step instead (Algorithm 1,
+Sec. 4.3): probe k on rank k mod R (its out-of-place pair pass and its two
+forwards), the K x 3 loss table all-gathered, the same preconditioner and
+fused update on every rank; K probes per step over the whole job.
 
 --impl reference times the CPU oracle instead (rank 0 only), on a bounded
 prefix sample of the same workload.
@@ -69,6 +73,9 @@ def parse_args():
                          "the update (2K+1 passes); alg1: Algorithm 1's +eps, -2eps, +eps per probe (3K+1); "
                          "pair: theta +- eps z_k written out of place by one pass per probe into two extra "
                          "copies of the weights (K+1 passes, 3 copies in device memory)")
+    ap.add_argument("--probe-parallel", action="store_true",
+                    help="the probe-parallel step over the ranks (probe k on rank k mod R, the loss table "
+                         "all-gathered, every rank updates); implies the pair schedule")
     ap.add_argument("--no-pair", action="store_true",
                     help="skip the extra measurement of the out-of-place pair schedule")
     ap.add_argument("--no-sequential", action="store_true",
@@ -588,6 +595,26 @@ def run_tiny(args):
         dist.destroy_process_group()
 
 
+# ------------------------------------------------ probe-parallel step
+def probe_parallel_step(L, K, rank, world, pair_pass, gather, finish):
+    """One probe-parallel step as --probe-parallel runs it (Algorithm 1,
+    Sec. 4.3, without the parameter broadcast: the pair passes leave theta
+    untouched, so replicas stay identical): this rank's probes k = rank,
+    rank + world, ... each get their out-of-place pair pass (pair_pass(k));
+    their loss rows -- the seeded triples of L standing in for the forwards
+    at theta +- eps z_k and the clean loss -- are all-gathered into the full
+    K x 3 table (gather(rows)), and every rank runs the preconditioner and
+    the fused update on it (finish(table)). The arithmetic is injected, so
+    the rank logic runs on CPU with the oracle. Returns the table."""
+    from paper_2609_38095_gb300 import replicas as R
+    mine = list(R.probes_of_rank(K, rank, world))
+    for k in mine:
+        pair_pass(k)
+    table = gather(L[mine])
+    finish(table)
+    return table
+
+
 # ---------------------------------------------------------------- GPU arm
 def run_zo(args):
     import torch
@@ -629,13 +656,18 @@ def run_zo(args):
     status = torch.zeros(1, dtype=torch.int32, device=dev)
     stream = torch.cuda.current_stream(dev)
     chunks = (len(params) + 1023) // 1024
-    pair = args.schedule == "pair"
+    pp = args.probe_parallel
+    pair = args.schedule == "pair" or pp
+    my_probes = K          # probes whose passes this rank runs
+    if pp:
+        from paper_2609_38095_gb300 import replicas
+        my_probes = len(replicas.probes_of_rank(K, rank, world))
     if pair:
         plus = zo.ParamList([like_param(t) for t in params])
         minus = zo.ParamList([like_param(t) for t in params])
 
     timing = {"perturb": [], "perturb2": [], "pair": [], "update": [], "precondition": []}
-    fused = args.schedule == "fused"
+    fused = args.schedule == "fused" and not pp
 
     def timed(key, record, fn, *a, **kw):
         if not record:
@@ -652,6 +684,14 @@ def run_zo(args):
         +eps and each -2eps pass. The fused schedule leaves the weights at
         those points, and at the end, bit for bit as Algorithm 1's does."""
         seed = W.step_seed(s)
+        if pp:
+            def finish(table):
+                timed("precondition", record, zo.precondition, table, eps, out=(c, status))
+                timed("update", record, zo.update, plist, seed, c, eps, status=status)
+            probe_parallel_step(losses_d, K, rank, world,
+                                lambda k: timed("pair", record, zo.perturb_pair, plist, plus, minus, seed, k, eps),
+                                lambda rows: replicas.all_gather_losses(rows, K), finish)
+            return
         if pair:
             for k in range(K):
                 timed("pair", record, zo.perturb_pair, plist, plus, minus, seed, k, eps)
@@ -693,7 +733,10 @@ def run_zo(args):
     elapsed_ms = ranks_max(t_start.elapsed_time(t_end))
     ms_per_step = elapsed_ms / args.steps
     passes = K + 1 if pair else (2 * K + 1 if fused else 3 * K + 1)   # sweeps over the weights, update included
-    if pair:
+    if pp:
+        passes = my_probes + 1                                            # on each rank
+        launches = args.steps * (my_probes * chunks + 1 + chunks)
+    elif pair:
         launches = args.steps * (K * chunks + 1 + chunks)
     else:
         launches = args.steps * ((passes - 1) * chunks + 1 + chunks)
@@ -728,12 +771,12 @@ def run_zo(args):
                 raise RuntimeError("preconditioner reported non-finite losses")
         barrier()
         e2e_s = ranks_max((time.perf_counter() - t0) / args.steps)
-        e2e = {"value": whole_job_rate(world, d, K, e2e_s), "unit": UNIT, "h2d_bytes_per_step": K * 3 * 8,
+        e2e = {"value": whole_job_rate(1 if pp else world, d, K, e2e_s), "unit": UNIT, "h2d_bytes_per_step": K * 3 * 8,
                "d2h_bytes_per_step": K * 8 + 4, "ms_per_step": e2e_s * 1e3}
 
     # ---- the out-of-place pair schedule on the same weights (two more copies)
     pair_alt = None
-    if not pair and not args.no_pair:
+    if not pair and not args.no_pair and not pp:
         free, _ = torch.cuda.mem_get_info(dev)
         if free > 2.05 * d * ps.bytes_per_elem:
             plus_a = zo.ParamList([like_param(t) for t in params])
@@ -801,7 +844,7 @@ def run_zo(args):
     n1, n2 = (K + 1, K - 1) if fused else ((0, 0) if pair else (3 * K, 0))
     if pair:
         dom_kernel, dom_ms, dom_launches = ("pair_shift_kernel<*> (tensors off the 32-byte grid)" if shifted
-                                            else "perturb_pair_kernel"), pair_ms, K
+                                            else "perturb_pair_kernel"), pair_ms, my_probes
         traffic, traffic_how = committed_traffic("perturb_pair_kernel", traffic_key)
     elif n2 > 0 and n2 * perturb2_ms > n1 * perturb_ms:
         dom_kernel, dom_ms, dom_launches = ("perturb_shift_kernel<2, *> (zo_perturb2, tensors off the 32-byte grid)"
@@ -816,13 +859,15 @@ def run_zo(args):
     dom_bytes = pair_bytes if pair else perturb_bytes
     # algorithmic HBM bytes of one step: every pass reads and writes theta once,
     # except the pair passes (read theta, write two copies)
-    step_bytes = K * pair_bytes + perturb_bytes if pair else passes * perturb_bytes
+    step_bytes = my_probes * pair_bytes + perturb_bytes if pair else passes * perturb_bytes
     dom_achieved = dom_bytes / (dom_ms * 1e-3) / 1e9
     sms = torch.cuda.get_device_properties(dev).multi_processor_count
     sm_mhz = (clk or {}).get("sm_mhz") or float(peaks.get("sm_max_mhz", 2070.0))
     alu_peak = sms * LANES_PER_SM * sm_mhz * 1e6 / 1e9    # Gparam*probe/s at one instruction per pair
     upd_rate = d * K / (update_ms * 1e-3) / 1e9
-    value = whole_job_rate(world, d, K, ms_per_step * 1e-3)
+    # replicas: every rank does the whole step (d x K each); probe-parallel: the
+    # ranks share one step's K probes
+    value = whole_job_rate(1 if pp else world, d, K, ms_per_step * 1e-3)
 
     if rank != 0:
         return
@@ -832,13 +877,15 @@ def run_zo(args):
         cpu = cpu_baseline_line(ps, args, v, M, cores, sample)
     line = {
         "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
-        "warmup": args.warmup, "ms_per_step": ms_per_step, "higher_is_better": True, "scaling": "weak",
-        "vs_baseline": None, "dtype": "f32", "data": "synthetic",
+        "warmup": args.warmup, "ms_per_step": ms_per_step, "higher_is_better": True,
+        "scaling": "strong" if pp else "weak", "vs_baseline": None, "dtype": "f32", "data": "synthetic",
         "config": {"workload": ps.name, "K": K, "d": d, "tensors": len(params), "packing": args.packing,
-                   "schedule": f"{args.schedule} ({passes} passes over the weights per step)",
+                   "schedule": (f"probe-parallel pair schedule ({passes} passes over the weights per step on each "
+                                f"of {world} ranks, the K x 3 loss table all-gathered)" if pp else
+                                f"{args.schedule} ({passes} passes over the weights per step)"),
                    "storage": "fp16" if
                    ps.dtype == W.DT_F16 else ("bf16" if ps.dtype == W.DT_BF16 else "fp32"),
-                   "eps": eps, "lr": eps, "parallelism": f"replicas{world}",
+                   "eps": eps, "lr": eps, "parallelism": f"probe-parallel{world}" if pp else f"replicas{world}",
                    **({"view_offset": args.view_offset} if args.view_offset else {}),
                    "l2": "inputs larger than L2 (every pass streams the whole parameter set)"},
         "roofline": {"bound": "hbm", "kernel": dom_kernel, "achieved": dom_achieved, "peak": hbm_peak,
@@ -852,7 +899,7 @@ def run_zo(args):
                          "launches_per_step": (K + 1 if fused else 3 * K) * chunks} if not pair else None),
             "pair": ({"ms": pair_ms, "GB/s": pair_bytes / (pair_ms * 1e-3) / 1e9,
                       "frac_of_measured_hbm": pair_bytes / (pair_ms * 1e-3) / 1e9 / hbm_peak,
-                      "bytes_per_pass": pair_bytes, "launches_per_step": K * chunks} if pair else None),
+                      "bytes_per_pass": pair_bytes, "launches_per_step": my_probes * chunks} if pair else None),
             "perturb2": ({"ms": perturb2_ms, "GB/s": perturb_bytes / (perturb2_ms * 1e-3) / 1e9,
                           "frac_of_measured_hbm": perturb_bytes / (perturb2_ms * 1e-3) / 1e9 / hbm_peak,
                           "launches_per_step": (K - 1) * chunks} if fused and K > 1 else None),

@@ -1,7 +1,9 @@
-"""bench.py's multi-GPU path is replicas only: every rank runs the whole
-workload on its own GPU and nothing is exchanged but the timing. Its rank
-logic (barrier, max over ranks, whole-job rate, rank-0-only reference arm)
-runs here on CPU with world_size-2 gloo process groups."""
+"""bench.py's rank logic on CPU with world_size-2 gloo process groups: the
+default multi-GPU path (replicas: every rank runs the whole workload on its
+own GPU, only the timing is exchanged -- barrier, max over ranks, whole-job
+rate, rank-0-only reference arm) and the --probe-parallel step (probe k on
+rank k mod R, the loss table all-gathered, every rank updating), the latter
+with the oracle as each rank's arithmetic."""
 import os
 import socket
 import sys
@@ -99,3 +101,75 @@ def test_cpu_model_and_single_thread_oracle():
     ps = bench.W.OPT_1_3B
     v, n = bench.time_oracle_single(ps, 0.2)
     assert v > 0 and n % 16 == 0 and n >= 16
+
+
+# ------------------------------------------- --probe-parallel, oracle arithmetic
+def pp_worker(rank, world, port, out):
+    """One rank of bench.py's probe-parallel step with the oracle as the
+    arithmetic: out-of-place pair passes of its probes on host copies, the
+    loss rows all-gathered over gloo, the oracle's preconditioner and update."""
+    import numpy as np
+
+    import oracle
+    from paper_2609_38095_gb300 import replicas as R
+    from paper_2609_38095_gb300 import workloads as W
+    os.environ.update(MASTER_ADDR="127.0.0.1", MASTER_PORT=str(port), RANK=str(rank), WORLD_SIZE=str(world))
+    if world > 1:
+        dist.init_process_group("gloo", rank=rank, world_size=world)
+    try:
+        dts = [W.DT_BF16, W.DT_F32]
+        rng = np.random.default_rng(5)
+        theta = [W.random_storage(rng, n, dt) for n, dt in zip([1000, 333], dts)]
+        K, eps, seed = 7, 1e-3, W.step_seed(9)
+        L = torch.from_numpy(W.synthetic_losses(K, 9))
+        passes = []
+
+        def pair_pass(k):
+            plus, minus = [t.copy() for t in theta], [t.copy() for t in theta]
+            oracle.perturb(plus, dts, seed, k, eps)
+            oracle.perturb(minus, dts, seed, k, -eps)
+            passes.append(k)
+
+        def finish(table):
+            rc, c, _, _ = oracle.precondition(table.numpy(), eps)
+            assert rc == oracle.OK
+            oracle.update(theta, dts, seed, c, eps)
+
+        table = bench.probe_parallel_step(L, K, rank, world, pair_pass, lambda rows: R.all_gather_losses(rows, K),
+                                          finish)
+        out.put((rank, passes, table.numpy(), [t.copy() for t in theta]))
+    finally:
+        if world > 1:
+            dist.destroy_process_group()
+
+
+def run_pp(world):
+    port = free_port()
+    ctx = mp.get_context("spawn")
+    q = ctx.Queue()
+    procs = [ctx.Process(target=pp_worker, args=(r, world, port, q)) for r in range(world)]
+    for p in procs:
+        p.start()
+    res = sorted((q.get(timeout=300) for _ in range(world)), key=lambda x: x[0])
+    for p in procs:
+        p.join(timeout=120)
+        assert p.exitcode == 0
+    return res
+
+
+def test_probe_parallel_step_gloo_two_ranks():
+    """Two gloo ranks split the probes (0, 2, 4, 6 and 1, 3, 5), both end up
+    with the full seeded loss table and with the same weights, bit for bit
+    those of one process running every probe."""
+    import numpy as np
+    from paper_2609_38095_gb300 import workloads as W
+    two = run_pp(2)
+    one = run_pp(1)
+    assert two[0][1] == [0, 2, 4, 6] and two[1][1] == [1, 3, 5] and one[0][1] == list(range(7))
+    want = W.synthetic_losses(7, 9)
+    for _, _, table, _ in two + one:
+        np.testing.assert_array_equal(table, want)
+    for r in range(2):
+        for a, b in zip(two[r][3], one[0][3]):
+            view = np.uint32 if a.dtype == np.float32 else np.uint16
+            np.testing.assert_array_equal(a.view(view), b.view(view))
