@@ -78,6 +78,8 @@ def parse_args():
                          "all-gathered, every rank updates); implies the pair schedule")
     ap.add_argument("--no-pair", action="store_true",
                     help="skip the extra measurement of the out-of-place pair schedule")
+    ap.add_argument("--no-other-sets", action="store_true",
+                    help="skip the short timings of the other parameter sets (and of the aligned-chunk kernels)")
     ap.add_argument("--no-sequential", action="store_true",
                     help="skip timing Algorithm 1's K sequential update passes against the fused update")
     ap.add_argument("--view-offset", type=int, default=0,
@@ -615,6 +617,52 @@ def probe_parallel_step(L, K, rank, world, pair_pass, gather, finish):
     return table
 
 
+# ------------------------------------------------ the other parameter sets
+def time_kernels_on_set(key, dev, hbm_peak, alu_peak, view_offset=0):
+    """Short CUDA-event timings of the single-op and two-op passes and the
+    fused update (with the leading restore, at the set's K) on one parameter
+    set: the evidence for the configurations the headline line does not run."""
+    import torch
+
+    import paper_2609_38095_gb300 as zo
+    ps = W.BY_KEY[key]
+    params = W.allocate_params(ps, device=dev, view_offset=view_offset)
+    try:
+        plist = zo.ParamList(params)
+        stream = torch.cuda.current_stream(dev)
+        seed, eps, K = W.step_seed(0), ps.eps, ps.K
+        c = torch.tensor(W.synthetic_losses(K, 0)[:, 0] - 2.5, dtype=torch.float64, device=dev)
+
+        def ms_of(fn, n):
+            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            torch.cuda.synchronize(dev)
+            e0.record(stream)
+            for i in range(n):
+                fn(i)
+            e1.record(stream)
+            torch.cuda.synchronize(dev)
+            return e0.elapsed_time(e1) / n
+
+        for i in range(12):                       # the two-op tuner's trials, then its choice
+            zo.perturb2(plist, seed, i, eps, i + 1, eps)
+        torch.cuda.synchronize(dev)
+        zo.perturb2(plist, seed, 0, eps, 1, eps)
+        zo.update(plist, seed, c, eps, pre=(K - 1, eps))
+        p1 = ms_of(lambda i: zo.perturb(plist, seed, i, eps if i % 2 else -eps), 6)
+        p2 = ms_of(lambda i: zo.perturb2(plist, seed, i, eps, i + 1, -eps), 6)
+        up = ms_of(lambda i: zo.update(plist, seed + i, c, eps, pre=(K - 1, eps)), 3)
+        byt = 2.0 * ps.d * ps.bytes_per_elem
+        rate = ps.d * K / (up * 1e-3) / 1e9
+        return {"workload": ps.name + (f"+view{view_offset}" if view_offset else ""), "d": ps.d, "K": K,
+                "perturb_ms": p1, "perturb_frac_of_measured_hbm": byt / (p1 * 1e-3) / 1e9 / hbm_peak,
+                "perturb2_ms": p2, "perturb2_frac_of_measured_hbm": byt / (p2 * 1e-3) / 1e9 / hbm_peak,
+                "update_ms": up, "update_gparam_probe_per_s": rate, "update_frac_alu_1instr": rate / alu_peak,
+                "update_frac_of_measured_hbm": byt / (up * 1e-3) / 1e9 / hbm_peak}
+    finally:
+        del params
+        torch.cuda.empty_cache()
+
+
 # ---------------------------------------------------------------- GPU arm
 def run_zo(args):
     import torch
@@ -641,6 +689,7 @@ def run_zo(args):
     K, eps, d = ps.K, ps.eps, ps.d
     params = W.allocate_params(ps, device=dev, view_offset=args.view_offset)
     plist = zo.ParamList(params)
+    n_tensors = len(params)
     shifted = any(t.data_ptr() % 32 for t in params)   # the perturbation passes use perturb_shift_kernel
 
     def like_param(t):
@@ -869,6 +918,15 @@ def run_zo(args):
     # ranks share one step's K probes
     value = whole_job_rate(1 if pp else world, d, K, ms_per_step * 1e-3)
 
+    others = None
+    if world == 1 and not args.no_other_sets:
+        del params, plist
+        if pair:
+            del plus, minus
+        torch.cuda.empty_cache()
+        others = [time_kernels_on_set(k, dev, hbm_peak, alu_peak) for k in ("opt-1.3b", "qwen3-8b", "opt-13b", "opt-30b")
+                  if k != args.config]
+        others.append(time_kernels_on_set("opt-1.3b", dev, hbm_peak, alu_peak, view_offset=1))
     if rank != 0:
         return
     cpu = None
@@ -879,7 +937,7 @@ def run_zo(args):
         "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
         "warmup": args.warmup, "ms_per_step": ms_per_step, "higher_is_better": True,
         "scaling": "strong" if pp else "weak", "vs_baseline": None, "dtype": "f32", "data": "synthetic",
-        "config": {"workload": ps.name, "K": K, "d": d, "tensors": len(params), "packing": args.packing,
+        "config": {"workload": ps.name, "K": K, "d": d, "tensors": n_tensors, "packing": args.packing,
                    "schedule": (f"probe-parallel pair schedule ({passes} passes over the weights per step on each "
                                 f"of {world} ranks, the K x 3 loss table all-gathered)" if pp else
                                 f"{args.schedule} ({passes} passes over the weights per step)"),
@@ -913,6 +971,7 @@ def run_zo(args):
         "e2e": e2e,
         "sequential": seq,
         "pair_schedule": pair_alt,
+        "other_sets": others,
         "gpu_launches": launches,
         "clocks": clk,
         "cpu_baseline": cpu,
