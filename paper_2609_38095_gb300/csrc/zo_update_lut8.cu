@@ -284,6 +284,185 @@ __global__ void __launch_bounds__(THREADS, 1) update_lut8_kernel(const __grid_co
   }
 }
 
+// ---------------------------------------------------------------------------
+// One or two probe groups (K <= 16): both tables stay in the first region for
+// the whole launch, so there is no chunking and no barrier. The kernel walks
+// blocks grid-stride like the perturbation passes, the next block's 256-bit
+// load issued before the current block is computed, and every element takes
+// its one or two lookups and is stored at once: the same sums, in the same
+// order (0 + T8_0 [+ T8_1]), as the chunked kernel. The leading perturbation
+// reuses the Philox word of its own group when it is one of the two.
+// ---------------------------------------------------------------------------
+constexpr int kSmallThreads = 1024;
+size_t lut8_small_smem_bytes() { return 2 * static_cast<size_t>(kLut8Region) + 16u; }
+
+struct SmallCursor {
+  int t;
+  uint32_t tb, te, n16;  // first and one-past-last launch block; full aligned 16-bit blocks from tb
+  uint32_t vd;           // launch block minus virtual block offset
+  uint16_t* tp;
+  uint8_t dt;
+};
+
+__device__ __forceinline__ void small_seek(const TensorTable& tab, SmallCursor& c, uint32_t b) {
+  c.t = advance_tensor(tab, c.t, b);
+  c.tb = tensor_blk_begin(tab, c.t);
+  c.te = tab.blk_end[c.t];
+  const uint8_t fl = tab.flags[c.t];
+  c.dt = fl & kDtypeMask;
+  c.n16 = ((fl & kVec32) && c.dt != kF32) ? static_cast<uint32_t>(tab.numel[c.t] / 16) : 0u;
+  c.vd = tab.vdelta[c.t];
+  c.tp = reinterpret_cast<uint16_t*>(tab.ptr[c.t]);
+}
+
+// Sum of element e's lookups (groups in order) from the Philox words of groups 0 and 1.
+template <int E>
+__device__ __forceinline__ float small_sum(const uint4& x0, const uint4& x1, uint32_t frame, bool two) {
+  constexpr uint32_t sel = 0x7604u | (static_cast<uint32_t>(E & 3) << 4);
+  float acc = __fadd_rn(0.0f, lds_f32(__byte_perm(word_of(x0, E >> 2), frame, sel)));
+  if (two) acc = __fadd_rn(acc, lds_f32(__byte_perm(word_of(x1, E >> 2), frame | 128u, sel)));
+  return acc;
+}
+
+template <uint8_t DT>
+__device__ __forceinline__ void small_block16(uint32_t (&v)[8], const uint4& x0, const uint4& x1, const uint4& xp,
+                                              uint32_t frame, bool two, const UpdateParams& P, bool do_sum) {
+#pragma unroll
+  for (int r = 0; r < 8; ++r) {
+    if (P.has_pre) v[r] = pre_regs16<DT>(v[r], xp, r, P.pre);
+    if (do_sum) {
+      const float2 f = unpack2<DT>(v[r]);
+      float lo, hi;
+      switch (r) {  // element indices must be constants for the word and byte selects
+        case 0: lo = small_sum<0>(x0, x1, frame, two); hi = small_sum<1>(x0, x1, frame, two); break;
+        case 1: lo = small_sum<2>(x0, x1, frame, two); hi = small_sum<3>(x0, x1, frame, two); break;
+        case 2: lo = small_sum<4>(x0, x1, frame, two); hi = small_sum<5>(x0, x1, frame, two); break;
+        case 3: lo = small_sum<6>(x0, x1, frame, two); hi = small_sum<7>(x0, x1, frame, two); break;
+        case 4: lo = small_sum<8>(x0, x1, frame, two); hi = small_sum<9>(x0, x1, frame, two); break;
+        case 5: lo = small_sum<10>(x0, x1, frame, two); hi = small_sum<11>(x0, x1, frame, two); break;
+        case 6: lo = small_sum<12>(x0, x1, frame, two); hi = small_sum<13>(x0, x1, frame, two); break;
+        default: lo = small_sum<14>(x0, x1, frame, two); hi = small_sum<15>(x0, x1, frame, two); break;
+      }
+      v[r] = pack2<DT>(__fadd_rn(f.x, lo), __fadd_rn(f.y, hi));
+    }
+  }
+}
+
+// Any other block of the launch: fp32, a partial last block, padding, or an
+// unaligned tensor (update_shift_kernel's).
+__device__ __noinline__ void small_block_other(const TensorTable& tab, int t, uint32_t b, const UpdateParams& P,
+                                               uint32_t frame, bool do_sum) {
+  const uint32_t tb = tensor_blk_begin(tab, t);
+  const uint8_t fl = tab.flags[t];
+  if ((fl & kShift) || b < tb) return;
+  Lut8Block k;
+  k.b = virtual_block(tab, t, b);
+  k.e0 = static_cast<int64_t>(b - tb) * 16;
+  k.cnt = static_cast<int>(min(static_cast<int64_t>(16), tab.numel[t] - k.e0));
+  k.base = reinterpret_cast<void*>(tab.ptr[t]);
+  k.fl = fl;
+  k.act = true;
+  k.vec16 = false;
+  float acc[16];
+#pragma unroll
+  for (int i = 0; i < 16; ++i) acc[i] = 0.0f;
+  if (do_sum) {
+    lut8_lookup(acc, block_bits(k.b, 0u, P.keys), frame);
+    if (P.groups > 1) lut8_lookup(acc, block_bits(k.b, 1u, P.keys), frame | 128u);
+  }
+  lut8_apply_other(k, acc, P, do_sum);
+}
+
+__global__ void __launch_bounds__(kSmallThreads, 1) update_lut8_small_kernel(const __grid_constant__ UpdateParams P) {
+  extern __shared__ __align__(16) unsigned char smem[];
+  __shared__ int skip_s;
+  const int G = P.groups;  // 1 or 2
+  const uint32_t sbase = static_cast<uint32_t>(__cvta_generic_to_shared(smem));
+  const uint32_t region0 = (sbase + kLut8Region - 1u) & ~(kLut8Region - 1u);
+  // coefficients and unreplicated tables (2 KB at most) below the region, or after it when the window starts on
+  // a 64 KB boundary
+  const uint32_t hdr = region0 - sbase >= 32u * G + 1024u * G ? sbase : region0 + kLut8Region;
+  float* a_s = reinterpret_cast<float*>(smem + (hdr - sbase));
+  float* t8 = a_s + 8 * G;
+  if (threadIdx.x == 0) skip_s = (P.status != nullptr && *P.status != 0);
+  for (int k = threadIdx.x; k < 8 * G; k += kSmallThreads)
+    a_s[k] = k < P.K ? __double2float_rn(P.coef_mul * P.coef[k]) : 0.0f;
+  __syncthreads();
+  const bool skip = skip_s != 0;
+  if (skip && !P.has_pre) return;
+  const bool do_sum = !skip;
+  if (do_sum) {
+    for (int e = threadIdx.x; e < 256 * G; e += kSmallThreads) {
+      const float* a = a_s + 8 * (e >> 8);
+      const uint32_t n = static_cast<uint32_t>(e) & 255u;
+      t8[e] = __fadd_rn(quad_partial(a, n & 15u), quad_partial(a + 4, n >> 4));
+    }
+    __syncthreads();
+    const uint32_t src_t = hdr + 32u * G + 4u * (threadIdx.x >> 3);
+    const uint32_t dst_t = 256u * (threadIdx.x >> 3) + 16u * (threadIdx.x & 7u);
+    lut8_replicate<kSmallThreads>(src_t, region0 + dst_t, 0, G > 1);
+    __syncthreads();
+  }
+  const TensorTable& tab = P.tab;
+  const uint32_t total = tab.blk_total;
+  const uint32_t stride = gridDim.x * kSmallThreads;
+  const uint32_t frame = (region0 & 0xFFFF0000u) | ((threadIdx.x & 31u) << 2);
+  const bool two = G > 1;
+  // the leading perturbation's Philox word: group 0's, group 1's, or its own
+  const int pre_src = !P.has_pre ? -1 : (P.pre.ctr2 == 0u ? 0 : (P.pre.ctr2 == 1u && two ? 1 : 2));
+  uint32_t b = blockIdx.x * kSmallThreads + threadIdx.x;
+  if (b >= total) return;
+  SmallCursor c;
+  c.t = 0;
+  small_seek(tab, c, b);
+  int t = c.t;
+  uint8_t dt = c.dt;
+  uint32_t vd = c.vd;
+  bool fast = b - c.tb < c.n16;
+  uint16_t* p = c.tp + static_cast<size_t>(b - c.tb) * 16;
+  uint32_t v[8];
+  if (fast) ld256(p, v);
+  while (true) {
+    const uint32_t bn = b + stride;
+    bool fastn = false;
+    uint16_t* pn = nullptr;
+    uint32_t vn[8];
+    if (bn < total) {
+      if (bn >= c.te) small_seek(tab, c, bn);
+      fastn = bn - c.tb < c.n16;
+      pn = c.tp + static_cast<size_t>(bn - c.tb) * 16;
+      if (fastn) ld256(pn, vn);
+    }
+    if (fast) {
+      const int64_t vb = tab.blk_base + (b - vd);
+      uint4 x0 = make_uint4(0u, 0u, 0u, 0u), x1 = x0, xp = x0;
+      if (do_sum || pre_src == 0 || pre_src == 1) {
+        x0 = block_bits(vb, 0u, P.keys);
+        if (two) x1 = block_bits(vb, 1u, P.keys);
+      }
+      if (pre_src == 0) xp = x0;
+      if (pre_src == 1) xp = x1;
+      if (pre_src == 2) xp = block_bits(vb, P.pre.ctr2, P.keys);
+      if (dt == kBF16)
+        small_block16<kBF16>(v, x0, x1, xp, frame, two, P, do_sum);
+      else
+        small_block16<kF16>(v, x0, x1, xp, frame, two, P, do_sum);
+      st256(p, v);
+    } else {
+      small_block_other(tab, t, b, P, frame, do_sum);
+    }
+    if (bn >= total) break;
+    b = bn;
+    t = c.t;
+    dt = c.dt;
+    vd = c.vd;
+    fast = fastn;
+    p = pn;
+#pragma unroll
+    for (int r = 0; r < 8; ++r) v[r] = vn[r];
+  }
+}
+
 template <int THREADS, int BPT>
 cudaError_t launch_lut8_cfg(const UpdateParams& p, int grid, cudaStream_t stream) {
   const size_t smem = lut8_smem_bytes(p.groups);
@@ -304,9 +483,22 @@ cudaError_t lut8_prepare_cfg(int groups, int* blocks_per_sm) {
 
 bool lut8_supported(int groups, int packing) { return packing == kPacking1 && groups >= 1 && groups <= kLut8MaxGroups; }
 
-cudaError_t lut8_prepare(int groups, int* blocks_per_sm) { return lut8_prepare_cfg<512, 2>(groups, blocks_per_sm); }
+cudaError_t lut8_prepare(int groups, int* blocks_per_sm) {
+  if (groups <= 2) {
+    cudaError_t e = cudaFuncSetAttribute(update_lut8_small_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         static_cast<int>(lut8_small_smem_bytes()));
+    if (e != cudaSuccess) return e;
+    return cudaOccupancyMaxActiveBlocksPerMultiprocessor(blocks_per_sm, update_lut8_small_kernel, kSmallThreads,
+                                                         lut8_small_smem_bytes());
+  }
+  return lut8_prepare_cfg<512, 2>(groups, blocks_per_sm);
+}
 
 cudaError_t launch_update_lut8(const UpdateParams& p, int grid, cudaStream_t stream) {
+  if (p.groups <= 2) {
+    update_lut8_small_kernel<<<grid, kSmallThreads, lut8_small_smem_bytes(), stream>>>(p);
+    return cudaGetLastError();
+  }
   return launch_lut8_cfg<512, 2>(p, grid, stream);
 }
 
