@@ -740,10 +740,7 @@ int zo_update_ex(const zo_tensor* params, int32_t n_tensors, uint64_t seed, cons
       bool main_work = false;
       const unsigned shift_types = mark_shift(up.tab, &main_work);
       if (main_work && lut8) {
-        // one CTA per 1024 blocks (its chunk), at most the resident CTAs
-        const int64_t want = (static_cast<int64_t>(up.tab.blk_total) + 1023) / 1024;
-        const int64_t cap = static_cast<int64_t>(d->sms) * bps;
-        cudaError_t e = zo::launch_update_lut8(up, static_cast<int>(want < cap ? want : cap), s);
+        cudaError_t e = zo::launch_update_lut8(up, d->sms, bps, s);
         if (e != cudaSuccess) return cuda_fail(e, "update_lut8_kernel");
       } else if (main_work) {
         cudaError_t e = zo::launch_update(up, grid_for(up.tab.blk_total, d->sms, bps * kUpdateWaves), s);

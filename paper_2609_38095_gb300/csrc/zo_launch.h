@@ -29,7 +29,7 @@ cudaError_t launch_update(const UpdateParams& p, int grid, cudaStream_t stream);
 size_t lut8_smem_bytes(int groups);
 bool lut8_supported(int groups, int packing);
 cudaError_t lut8_prepare(int groups, int* blocks_per_sm);  // sets the shared-memory limit, occupancy
-cudaError_t launch_update_lut8(const UpdateParams& p, int grid, cudaStream_t stream);
+cudaError_t launch_update_lut8(const UpdateParams& p, int sms, int blocks_per_sm, cudaStream_t stream);
 cudaError_t launch_update_shift(const UpdateShiftParams& p, uint8_t dt, int grid, cudaStream_t stream);
 cudaError_t update_shift_blocks_per_sm(int groups, int packing, uint8_t dt, int* out);
 size_t update_smem_bytes(int groups);

@@ -25,13 +25,17 @@
 //
 // Loop order. The replicated tables of all groups do not fit in shared memory
 // (32 KB per group), so probe groups are the outer loop: a CTA owns a chunk of
-// THREADS * BPT = 1024 consecutive blocks; each thread accumulates its blocks
-// over all groups in registers and then applies the sums to theta (read once,
+// 512 * BPT consecutive blocks (BPT = 8 on large launches), accumulates every
+// block's sums over all groups and then applies them to theta (read once,
 // written once). Two regions of 64 KB each hold a pair of groups (one per
 // half): while the lanes look up groups 2p and 2p+1 in one region, they copy
 // the next pair's tables into the other; one barrier per pair separates the
-// two. With one or two groups the first region holds them for the whole
-// launch and the loop has no barrier.
+// two. The sums live in tensor memory (TMEM) between pairs, so the chunk is
+// not limited by registers: per pair, each 64 KB table copy and its barrier
+// serve 4096 blocks. With one or two groups (update_lut8_small_kernel) the
+// first region holds them for the whole launch and there is no chunking.
+#include <type_traits>
+
 #include "zo_device.cuh"
 #include "zo_launch.h"
 
@@ -41,10 +45,10 @@ constexpr uint32_t kLut8Region = 65536;   // 256 rows x 256 bytes: the tables of
 constexpr int kLut8MaxGroups = 48;        // larger K takes update_kernel
 
 // Shared-memory request: two 64 KB regions starting on a 64 KB boundary of
-// the shared window, plus the coefficients (8 per group) and unreplicated
-// tables (1 KB per group), placed in the slack below the first region when
-// they fit there (the window starts a few bytes in), else after the second:
-// 192 KB covers both cases for up to kLut8MaxGroups groups.
+// the shared window, plus the coefficients, 4-probe tables and the chunk's
+// virtual blocks (lut8_side_bytes: at most 24 KB), placed in the slack below
+// the first region when they fit there (the window starts a few bytes in),
+// else after the second: 192 KB covers both cases.
 size_t lut8_smem_bytes(int) { return 3 * static_cast<size_t>(kLut8Region) + 16u; }
 
 __device__ __forceinline__ float lds_f32(uint32_t addr) {
@@ -168,20 +172,174 @@ __device__ __forceinline__ void lut8_apply_other(const Lut8Block& k, const float
   }
 }
 
-template <int THREADS, int BPT>
-__global__ void __launch_bounds__(THREADS, 1) update_lut8_kernel(const __grid_constant__ UpdateParams P) {
+// Tensor-memory accumulators. A thread's sums for the blocks of its chunk live
+// in TMEM between probe-group pairs: 512 threads (16 warps), warp w reaching
+// TMEM lanes 32 (w mod 4) .. +31 and, of their 512 columns, the 128 from
+// 128 (w / 4); a thread's block j takes 16 columns (one per element). So a CTA
+// owns BPT = 8 blocks per thread (4096 blocks, 64 K elements) while its
+// registers hold two blocks' sums at a time, and each table copy and barrier
+// serves four times the elements of a register-only chunk of two blocks per
+// thread. The copies are what the chunk size is for: a pair's replicated
+// tables are 64 KB of shared-memory stores, against 32 KB of lookups per 1024
+// blocks.
+constexpr int kLut8Threads = 512;
+constexpr uint32_t kTmemCols = 512;
+
+__device__ __forceinline__ void tm_ld16(float (&r)[16], uint32_t taddr) {
+  asm volatile(
+      "tcgen05.ld.sync.aligned.32x32b.x16.b32 {%0, %1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, "
+      "%15}, [%16];"
+      : "=f"(r[0]), "=f"(r[1]), "=f"(r[2]), "=f"(r[3]), "=f"(r[4]), "=f"(r[5]), "=f"(r[6]), "=f"(r[7]), "=f"(r[8]),
+        "=f"(r[9]), "=f"(r[10]), "=f"(r[11]), "=f"(r[12]), "=f"(r[13]), "=f"(r[14]), "=f"(r[15])
+      : "r"(taddr));
+}
+
+// Wait for this thread's TMEM loads; the loaded registers pass through the
+// wait so that no use of them can be scheduled before it.
+__device__ __forceinline__ void tm_wait_ld(float (&r)[16]) {
+  asm volatile("tcgen05.wait::ld.sync.aligned;"
+               : "+f"(r[0]), "+f"(r[1]), "+f"(r[2]), "+f"(r[3]), "+f"(r[4]), "+f"(r[5]), "+f"(r[6]), "+f"(r[7]),
+                 "+f"(r[8]), "+f"(r[9]), "+f"(r[10]), "+f"(r[11]), "+f"(r[12]), "+f"(r[13]), "+f"(r[14]), "+f"(r[15])
+               :
+               : "memory");
+}
+
+__device__ __forceinline__ void tm_wait_ld2(float (&r)[16], float (&s)[16]) {
+  asm volatile("tcgen05.wait::ld.sync.aligned;"
+               : "+f"(r[0]), "+f"(r[1]), "+f"(r[2]), "+f"(r[3]), "+f"(r[4]), "+f"(r[5]), "+f"(r[6]), "+f"(r[7]),
+                 "+f"(r[8]), "+f"(r[9]), "+f"(r[10]), "+f"(r[11]), "+f"(r[12]), "+f"(r[13]), "+f"(r[14]), "+f"(r[15]),
+                 "+f"(s[0]), "+f"(s[1]), "+f"(s[2]), "+f"(s[3]), "+f"(s[4]), "+f"(s[5]), "+f"(s[6]), "+f"(s[7]),
+                 "+f"(s[8]), "+f"(s[9]), "+f"(s[10]), "+f"(s[11]), "+f"(s[12]), "+f"(s[13]), "+f"(s[14]), "+f"(s[15])
+               :
+               : "memory");
+}
+
+__device__ __forceinline__ void tm_st16(uint32_t taddr, const float (&a)[16]) {
+  asm volatile(
+      "tcgen05.st.sync.aligned.32x32b.x16.b32 [%0], {%1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, "
+      "%15, %16};" ::"r"(taddr),
+      "f"(a[0]), "f"(a[1]), "f"(a[2]), "f"(a[3]), "f"(a[4]), "f"(a[5]), "f"(a[6]), "f"(a[7]), "f"(a[8]), "f"(a[9]),
+      "f"(a[10]), "f"(a[11]), "f"(a[12]), "f"(a[13]), "f"(a[14]), "f"(a[15])
+      : "memory");
+}
+
+__device__ __forceinline__ void tm_wait_st() { asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory"); }
+__device__ __forceinline__ void tm_fence_before() { asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory"); }
+__device__ __forceinline__ void tm_fence_after() { asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory"); }
+
+__device__ __forceinline__ void tm_get16(float (&a)[16], uint32_t taddr) {
+  tm_ld16(a, taddr);
+  tm_wait_ld(a);
+}
+
+__device__ __forceinline__ void zero16(float (&a)[16]) {
+#pragma unroll
+  for (int i = 0; i < 16; ++i) a[i] = 0.0f;
+}
+
+// Copy the tables of groups q (and q + 1 when `two`) into the two halves of a
+// region, forming each entry T8[n] = T_lo[n & 15] + T_hi[n >> 4] from the
+// group's 16-entry 4-probe tables (t4: T_lo then T_hi, 32 floats per group).
+// Rows and pieces as in lut8_replicate; a thread's rows are 64 apart, so
+// n & 15 is the same in all of them.
+template <int THREADS>
+__device__ __forceinline__ void lut8_replicate4(uint32_t t4, uint32_t dst_t, int q, bool two) {
+  constexpr int S = 2048 / THREADS;
+  constexpr uint32_t kRowStep = THREADS / 8;
+  static_assert(kRowStep % 16 == 0, "rows of a thread must share n mod 16");
+  const uint32_t r0 = threadIdx.x >> 3;
+  float v0[S], v1[S];
+  const uint32_t g0 = t4 + 128u * static_cast<uint32_t>(q);
+  {
+    const float lo = lds_f32(g0 + 4u * (r0 & 15u));
+#pragma unroll
+    for (int p = 0; p < S; ++p) v0[p] = __fadd_rn(lo, lds_f32(g0 + 64u + 4u * ((p * kRowStep + r0) >> 4)));
+  }
+  if (two) {
+    const float lo = lds_f32(g0 + 128u + 4u * (r0 & 15u));
+#pragma unroll
+    for (int p = 0; p < S; ++p) v1[p] = __fadd_rn(lo, lds_f32(g0 + 192u + 4u * ((p * kRowStep + r0) >> 4)));
+  }
+#pragma unroll
+  for (int p = 0; p < S; ++p) sts_f32x4(dst_t + p * kRowStep * 256u, v0[p]);
+  if (two) {
+#pragma unroll
+    for (int p = 0; p < S; ++p) sts_f32x4(dst_t + 128u + p * kRowStep * 256u, v1[p]);
+  }
+}
+
+// Block bl of the launch: its tensor (cursor t, moved forward) and place.
+__device__ __forceinline__ void lut8_block_info(const TensorTable& tab, int& t, uint32_t bl, Lut8Block& k) {
+  k.act = bl < tab.blk_total;
+  k.vec16 = false;
+  if (!k.act) return;
+  t = advance_tensor(tab, t, bl);
+  k.fl = tab.flags[t];
+  const uint32_t tb = tensor_blk_begin(tab, t);
+  // unaligned tensors are update_shift_kernel's; blocks below tb are padding
+  k.act = !(k.fl & kShift) && bl >= tb;
+  k.b = virtual_block(tab, t, bl);
+  k.e0 = static_cast<int64_t>(bl - tb) * 16;
+  k.cnt = static_cast<int>(min(static_cast<int64_t>(16), tab.numel[t] - k.e0));
+  k.base = reinterpret_cast<void*>(tab.ptr[t]);
+  k.vec16 = k.act && k.cnt == 16 && (k.fl & kVec32) && (k.fl & kDtypeMask) != kF32;
+}
+
+// One step of a probe-group pair: this thread's blocks j and j + 1 (sums at
+// TMEM address ta and ta + 16) over group q and, when `two`, q + 1. Every lane
+// takes part (an inactive lane's sums are never applied), so the step has no
+// branch; four independent Philox calls per step keep the lanes busy while
+// the sums come in from TMEM. Per block the groups are added in order.
+template <bool FIRST>
+__device__ __forceinline__ void lut8_tm_step(uint32_t ta, int64_t b0, int64_t b1, uint32_t q, bool two,
+                                             uint32_t frame, const RoundKeys& keys) {
+  float acc0[16], acc1[16];
+  if (FIRST) {
+    zero16(acc0);
+    zero16(acc1);
+  } else {
+    tm_ld16(acc0, ta);
+    tm_ld16(acc1, ta + 16u);
+  }
+  const uint4 x00 = block_bits(b0, q, keys), x10 = block_bits(b1, q, keys);
+  if (!FIRST) tm_wait_ld2(acc0, acc1);
+  lut8_lookup(acc0, x00, frame);
+  lut8_lookup(acc1, x10, frame);
+  if (two) {
+    const uint4 x01 = block_bits(b0, q + 1u, keys), x11 = block_bits(b1, q + 1u, keys);
+    lut8_lookup(acc0, x01, frame | 128u);
+    lut8_lookup(acc1, x11, frame | 128u);
+  }
+  tm_st16(ta, acc0);
+  tm_st16(ta + 16u, acc1);
+}
+
+// Shared memory besides the two regions: coefficients (8 per group), 4-probe
+// tables (32 per group) and the chunk's virtual blocks (one per thread and
+// block), below the first region when they fit there, else after the second.
+__host__ __device__ constexpr uint32_t lut8_side_bytes(int groups, int bpt) {
+  return 160u * static_cast<uint32_t>(groups) + 4u * kLut8Threads * static_cast<uint32_t>(bpt);
+}
+// Placed after the second region only when the slack below the first is
+// smaller than it, so the layout ends within 2 * side + 128 KB of the window's
+// start: inside the 192 KB request while side <= 32 KB.
+static_assert(lut8_side_bytes(kLut8MaxGroups, 8) <= kLut8Region / 2, "side data must fit the request");
+
+template <int BPT>
+__global__ void __launch_bounds__(kLut8Threads, 1) update_lut8_kernel(const __grid_constant__ UpdateParams P) {
+  constexpr int THREADS = kLut8Threads;
   extern __shared__ __align__(16) unsigned char smem[];
   __shared__ int skip_s;
+  __shared__ uint32_t tmem_s;
   const int G = P.groups;
   const int NP = (G + 1) / 2;  // group pairs: groups 2p, 2p + 1 share one region
-  // Two regions on 64 KB boundaries; the coefficients and unreplicated tables
-  // below the first one when they fit there, else after the second.
   const uint32_t sbase = static_cast<uint32_t>(__cvta_generic_to_shared(smem));
   const uint32_t region0 = (sbase + kLut8Region - 1u) & ~(kLut8Region - 1u);
-  const uint32_t hdr_bytes = 32u * G + 1024u * G;
-  const uint32_t hdr = region0 - sbase >= hdr_bytes ? sbase : region0 + 2u * kLut8Region;
+  const uint32_t side = lut8_side_bytes(G, BPT);
+  const uint32_t hdr = region0 - sbase >= side ? sbase : region0 + 2u * kLut8Region;
   float* a_s = reinterpret_cast<float*>(smem + (hdr - sbase));  // 8 G coefficients
-  float* t8 = a_s + 8 * G;                                      // 256 G partials
+  float* t4 = a_s + 8 * G;                                      // 32 G 4-probe partials
+  uint32_t* vr_s = reinterpret_cast<uint32_t*>(t4 + 32 * G);     // BPT x THREADS virtual blocks
 
   if (threadIdx.x == 0) skip_s = (P.status != nullptr && *P.status != 0);
   for (int k = threadIdx.x; k < 8 * G; k += THREADS)
@@ -190,96 +348,129 @@ __global__ void __launch_bounds__(THREADS, 1) update_lut8_kernel(const __grid_co
   const bool skip = skip_s != 0;
   if (skip && !P.has_pre) return;
   const bool do_sum = !skip;  // a failed preconditioner still gets the leading perturbation
+  const uint32_t warp = threadIdx.x >> 5;
+  const uint32_t t4_s = hdr + 32u * G;
+  const uint32_t dst_t = 256u * (threadIdx.x >> 3) + 16u * (threadIdx.x & 7u);
+  uint32_t trow = 0;
   if (do_sum) {
-    for (int e = threadIdx.x; e < 256 * G; e += THREADS) {
-      const float* a = a_s + 8 * (e >> 8);
-      const uint32_t n = static_cast<uint32_t>(e) & 255u;
-      t8[e] = __fadd_rn(quad_partial(a, n & 15u), quad_partial(a + 4, n >> 4));
+    for (int e = threadIdx.x; e < 32 * G; e += THREADS) {
+      const float* a = a_s + 8 * (e >> 5) + ((e & 16) ? 4 : 0);
+      t4[e] = quad_partial(a, static_cast<uint32_t>(e) & 15u);
     }
     __syncthreads();
-  }
-  const uint32_t src_t = hdr + 32u * G + 4u * (threadIdx.x >> 3);  // this thread's rows of t8
-  const uint32_t dst_t = 256u * (threadIdx.x >> 3) + 16u * (threadIdx.x & 7u);
-  if (do_sum) {
-    lut8_replicate<THREADS>(src_t, region0 + dst_t, 0, G > 1);
+    lut8_replicate4<THREADS>(t4_s, region0 + dst_t, 0, G > 1);
+    if (warp == 0) {
+      __syncwarp();
+      const uint32_t dst = static_cast<uint32_t>(__cvta_generic_to_shared(&tmem_s));
+      asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(dst), "r"(kTmemCols)
+                   : "memory");
+      asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+    }
+    tm_fence_before();
     __syncthreads();
+    tm_fence_after();
+    // TMEM lane 32 (warp mod 4) + lane id, columns from 128 (warp / 4)
+    trow = tmem_s + (((warp & 3u) * 32u) << 16) + (warp >> 2) * 128u;
   }
 
   const TensorTable& tab = P.tab;
   const uint32_t lane = threadIdx.x & 31u;
-  const uint32_t chunk = static_cast<uint32_t>(THREADS * BPT);
+  constexpr uint32_t chunk = static_cast<uint32_t>(THREADS * BPT);
   const uint32_t per_round = gridDim.x * chunk;
   const uint32_t rounds = (tab.blk_total + per_round - 1u) / per_round;
   uint32_t cur = 0;  // region holding the current pair (0 or 1)
-  int t[BPT];
-#pragma unroll
-  for (int j = 0; j < BPT; ++j) t[j] = 0;
+  int tc = 0;        // tensor cursor: the tensor of this thread's first block of the chunk
 
   for (uint32_t rnd = 0; rnd < rounds; ++rnd) {
-    Lut8Block blk[BPT];
-    uint32_t v[BPT][8];
-    float acc[BPT][16];
-#pragma unroll
-    for (int j = 0; j < BPT; ++j) {
-      const uint32_t bl = (rnd * gridDim.x + blockIdx.x) * chunk + static_cast<uint32_t>(j * THREADS) + threadIdx.x;
-      Lut8Block& k = blk[j];
-      k.act = bl < tab.blk_total;
-      k.vec16 = false;
-      if (k.act) {
-        t[j] = advance_tensor(tab, t[j], bl);
-        k.fl = tab.flags[t[j]];
-        const uint32_t tb = tensor_blk_begin(tab, t[j]);
-        // unaligned tensors are update_shift_kernel's; blocks below tb are padding
-        k.act = !(k.fl & kShift) && bl >= tb;
-        k.b = virtual_block(tab, t[j], bl);
-        k.e0 = static_cast<int64_t>(bl - tb) * 16;
-        k.cnt = static_cast<int>(min(static_cast<int64_t>(16), tab.numel[t[j]] - k.e0));
-        k.base = reinterpret_cast<void*>(tab.ptr[t[j]]);
-        k.vec16 = k.act && k.cnt == 16 && (k.fl & kVec32) && (k.fl & kDtypeMask) != kF32;
-        if (k.vec16) ld256(static_cast<uint16_t*>(k.base) + k.e0, v[j]);
-      }
-#pragma unroll
-      for (int i = 0; i < 16; ++i) acc[j][i] = 0.0f;
-    }
+    // this thread's blocks of the chunk: cb, cb + THREADS, ..
+    const uint32_t cb = (rnd * gridDim.x + blockIdx.x) * chunk + threadIdx.x;
     if (do_sum) {
+      uint32_t wact = 0;  // blocks of the chunk that some lane of the warp sums
+      int t = tc;
+#pragma unroll
+      for (int j = 0; j < BPT; ++j) {
+        Lut8Block k;
+        lut8_block_info(tab, t, cb + static_cast<uint32_t>(j * THREADS), k);
+        vr_s[j * THREADS + threadIdx.x] = k.act ? static_cast<uint32_t>(k.b - tab.blk_base) : 0u;
+        if (__any_sync(0xFFFFFFFFu, k.act)) wact |= 1u << j;
+        // theta is read after all pairs: bring it into L2 meanwhile
+        if (k.vec16) asm volatile("prefetch.L2 [%0];" ::"l"(static_cast<uint16_t*>(k.base) + k.e0));
+      }
       for (int pr = 0; pr < NP; ++pr) {
         const uint32_t frame = ((region0 + cur * kLut8Region) & 0xFFFF0000u) | (lane << 2);
-        const int q = 2 * pr;
+        const uint32_t q = 2u * static_cast<uint32_t>(pr);
+        const bool two = static_cast<int>(q) + 1 < G;
+        const auto run = [&](auto first) {
 #pragma unroll
-        for (int j = 0; j < BPT; ++j) {
-          if (blk[j].act) lut8_lookup(acc[j], block_bits(blk[j].b, static_cast<uint32_t>(q), P.keys), frame);
-        }
-        if (q + 1 < G) {
-#pragma unroll
-          for (int j = 0; j < BPT; ++j) {
-            if (blk[j].act)
-              lut8_lookup(acc[j], block_bits(blk[j].b, static_cast<uint32_t>(q + 1), P.keys), frame | 128u);
+          for (int j = 0; j < BPT; j += 2) {
+            if (!((wact >> j) & 3u)) continue;  // no lane of the warp has either block
+            const int64_t b0 = tab.blk_base + vr_s[j * THREADS + threadIdx.x];
+            const int64_t b1 = tab.blk_base + vr_s[(j + 1) * THREADS + threadIdx.x];
+            lut8_tm_step<decltype(first)::value>(trow + 16u * static_cast<uint32_t>(j), b0, b1, q, two, frame,
+                                                 P.keys);
           }
-        }
+        };
+        if (pr == 0)
+          run(std::true_type());
+        else
+          run(std::false_type());
+        tm_wait_st();  // this pair's sums are in TMEM before the next pair reads them
         if (NP > 1) {
           // the next pair (wrapping to pair 0 for the next chunk) into the other region
-          const int qn = pr + 1 < NP ? q + 2 : 0;
-          lut8_replicate<THREADS>(src_t, region0 + (cur ^ 1u) * kLut8Region + dst_t, qn, qn + 1 < G);
+          const int qn = pr + 1 < NP ? static_cast<int>(q) + 2 : 0;
+          lut8_replicate4<THREADS>(t4_s, region0 + (cur ^ 1u) * kLut8Region + dst_t, qn, qn + 1 < G);
           __syncthreads();
           cur ^= 1u;
         }
       }
     }
-#pragma unroll
+    // Apply: each block's sums read back from TMEM and added to theta (in L2
+    // by now). Full aligned 16-bit blocks here; the rare others (fp32, partial
+    // last blocks) in a loop of their own, which keeps their code out of this one.
+    int t = tc;
+    bool others = false;
+#pragma unroll 1
     for (int j = 0; j < BPT; ++j) {
-      const Lut8Block& k = blk[j];
-      if (!k.act) continue;
+      Lut8Block k;
+      lut8_block_info(tab, t, cb + static_cast<uint32_t>(j * THREADS), k);
+      others |= k.act && !k.vec16;
+      uint32_t v[8];
+      if (k.vec16) ld256(static_cast<uint16_t*>(k.base) + k.e0, v);
+      float acc[16];
+      zero16(acc);
+      if (do_sum && __any_sync(0xFFFFFFFFu, k.vec16)) tm_get16(acc, trow + 16u * static_cast<uint32_t>(j));
       if (k.vec16) {
         uint4 xp = make_uint4(0u, 0u, 0u, 0u);
         if (P.has_pre) xp = block_bits(k.b, P.pre.ctr2, P.keys);
         if ((k.fl & kDtypeMask) == kBF16)
-          lut8_apply16<kBF16>(v[j], acc[j], xp, P, do_sum);
+          lut8_apply16<kBF16>(v, acc, xp, P, do_sum);
         else
-          lut8_apply16<kF16>(v[j], acc[j], xp, P, do_sum);
-        st256(static_cast<uint16_t*>(k.base) + k.e0, v[j]);
-      } else {
-        lut8_apply_other(k, acc[j], P, do_sum);
+          lut8_apply16<kF16>(v, acc, xp, P, do_sum);
+        st256(static_cast<uint16_t*>(k.base) + k.e0, v);
       }
+    }
+    if (__any_sync(0xFFFFFFFFu, others)) {
+      t = tc;
+#pragma unroll 1
+      for (int j = 0; j < BPT; ++j) {
+        Lut8Block k;
+        lut8_block_info(tab, t, cb + static_cast<uint32_t>(j * THREADS), k);
+        const bool mine = k.act && !k.vec16;
+        float acc[16];
+        zero16(acc);
+        if (do_sum && __any_sync(0xFFFFFFFFu, mine)) tm_get16(acc, trow + 16u * static_cast<uint32_t>(j));
+        if (mine) lut8_apply_other(k, acc, P, do_sum);
+      }
+    }
+    tc = t;
+  }
+  if (do_sum) {
+    tm_fence_before();
+    __syncthreads();
+    tm_fence_after();
+    if (warp == 0) {
+      __syncwarp();
+      asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem_s), "r"(kTmemCols) : "memory");
     }
   }
 }
@@ -463,22 +654,20 @@ __global__ void __launch_bounds__(kSmallThreads, 1) update_lut8_small_kernel(con
   }
 }
 
-template <int THREADS, int BPT>
+template <int BPT>
 cudaError_t launch_lut8_cfg(const UpdateParams& p, int grid, cudaStream_t stream) {
-  const size_t smem = lut8_smem_bytes(p.groups);
-  static_assert(2048 % THREADS == 0, "replication assumes THREADS divides 2048");
-  update_lut8_kernel<THREADS, BPT><<<grid, THREADS, smem, stream>>>(p);
+  update_lut8_kernel<BPT><<<grid, kLut8Threads, lut8_smem_bytes(p.groups), stream>>>(p);
   return cudaGetLastError();
 }
 
-template <int THREADS, int BPT>
+template <int BPT>
 cudaError_t lut8_prepare_cfg(int groups, int* blocks_per_sm) {
   // the limit covers every group count, so later launches with more groups still fit
-  cudaError_t e = cudaFuncSetAttribute(update_lut8_kernel<THREADS, BPT>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+  cudaError_t e = cudaFuncSetAttribute(update_lut8_kernel<BPT>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                        static_cast<int>(lut8_smem_bytes(kLut8MaxGroups)));
-  const size_t smem = lut8_smem_bytes(groups);
   if (e != cudaSuccess) return e;
-  return cudaOccupancyMaxActiveBlocksPerMultiprocessor(blocks_per_sm, update_lut8_kernel<THREADS, BPT>, THREADS, smem);
+  return cudaOccupancyMaxActiveBlocksPerMultiprocessor(blocks_per_sm, update_lut8_kernel<BPT>, kLut8Threads,
+                                                       lut8_smem_bytes(groups));
 }
 
 bool lut8_supported(int groups, int packing) { return packing == kPacking1 && groups >= 1 && groups <= kLut8MaxGroups; }
@@ -491,15 +680,39 @@ cudaError_t lut8_prepare(int groups, int* blocks_per_sm) {
     return cudaOccupancyMaxActiveBlocksPerMultiprocessor(blocks_per_sm, update_lut8_small_kernel, kSmallThreads,
                                                          lut8_small_smem_bytes());
   }
-  return lut8_prepare_cfg<512, 2>(groups, blocks_per_sm);
+  cudaError_t e = lut8_prepare_cfg<2>(groups, blocks_per_sm);
+  if (e == cudaSuccess) e = lut8_prepare_cfg<4>(groups, blocks_per_sm);
+  if (e == cudaSuccess) e = lut8_prepare_cfg<8>(groups, blocks_per_sm);
+  return e;
 }
 
-cudaError_t launch_update_lut8(const UpdateParams& p, int grid, cudaStream_t stream) {
+// Blocks per thread: the largest of 8, 4, 2 that still gives every SM a chunk.
+int lut8_bpt(uint32_t blk_total, int sms) {
+  for (int bpt = 8; bpt > 2; bpt /= 2)
+    if (static_cast<int64_t>(blk_total) >= static_cast<int64_t>(sms) * kLut8Threads * bpt) return bpt;
+  return 2;
+}
+
+
+cudaError_t launch_update_lut8(const UpdateParams& p, int sms, int blocks_per_sm, cudaStream_t stream) {
+  const int64_t total = p.tab.blk_total;
+  const int64_t cap = static_cast<int64_t>(sms) * blocks_per_sm;
   if (p.groups <= 2) {
-    update_lut8_small_kernel<<<grid, kSmallThreads, lut8_small_smem_bytes(), stream>>>(p);
+    const int64_t want = (total + kSmallThreads - 1) / kSmallThreads;
+    update_lut8_small_kernel<<<static_cast<int>(want < cap ? want : cap), kSmallThreads, lut8_small_smem_bytes(),
+                               stream>>>(p);
     return cudaGetLastError();
   }
-  return launch_lut8_cfg<512, 2>(p, grid, stream);
+  // one CTA per chunk of 512 * BPT blocks, at most the resident CTAs
+  const int bpt = lut8_bpt(p.tab.blk_total, sms);
+  const int64_t chunk = static_cast<int64_t>(kLut8Threads) * bpt;
+  const int64_t want = (total + chunk - 1) / chunk;
+  const int grid = static_cast<int>(want < cap ? want : cap);
+  switch (bpt) {
+    case 8: return launch_lut8_cfg<8>(p, grid, stream);
+    case 4: return launch_lut8_cfg<4>(p, grid, stream);
+    default: return launch_lut8_cfg<2>(p, grid, stream);
+  }
 }
 
 }  // namespace zo
