@@ -177,7 +177,7 @@ __device__ __forceinline__ void lut8_apply_other(const Lut8Block& k, const float
 // TMEM lanes 32 (w mod 4) .. +31 and, of their 512 columns, the 128 from
 // 128 (w / 4); a thread's block j takes 16 columns (one per element). So a CTA
 // owns BPT = 8 blocks per thread (4096 blocks, 64 K elements) while its
-// registers hold two blocks' sums at a time, and each table copy and barrier
+// registers hold one block's sums at a time, and each table copy and barrier
 // serves four times the elements of a register-only chunk of two blocks per
 // thread. The copies are what the chunk size is for: a pair's replicated
 // tables are 64 KB of shared-memory stores, against 32 KB of lookups per 1024
@@ -200,16 +200,6 @@ __device__ __forceinline__ void tm_wait_ld(float (&r)[16]) {
   asm volatile("tcgen05.wait::ld.sync.aligned;"
                : "+f"(r[0]), "+f"(r[1]), "+f"(r[2]), "+f"(r[3]), "+f"(r[4]), "+f"(r[5]), "+f"(r[6]), "+f"(r[7]),
                  "+f"(r[8]), "+f"(r[9]), "+f"(r[10]), "+f"(r[11]), "+f"(r[12]), "+f"(r[13]), "+f"(r[14]), "+f"(r[15])
-               :
-               : "memory");
-}
-
-__device__ __forceinline__ void tm_wait_ld2(float (&r)[16], float (&s)[16]) {
-  asm volatile("tcgen05.wait::ld.sync.aligned;"
-               : "+f"(r[0]), "+f"(r[1]), "+f"(r[2]), "+f"(r[3]), "+f"(r[4]), "+f"(r[5]), "+f"(r[6]), "+f"(r[7]),
-                 "+f"(r[8]), "+f"(r[9]), "+f"(r[10]), "+f"(r[11]), "+f"(r[12]), "+f"(r[13]), "+f"(r[14]), "+f"(r[15]),
-                 "+f"(s[0]), "+f"(s[1]), "+f"(s[2]), "+f"(s[3]), "+f"(s[4]), "+f"(s[5]), "+f"(s[6]), "+f"(s[7]),
-                 "+f"(s[8]), "+f"(s[9]), "+f"(s[10]), "+f"(s[11]), "+f"(s[12]), "+f"(s[13]), "+f"(s[14]), "+f"(s[15])
                :
                : "memory");
 }
@@ -285,33 +275,24 @@ __device__ __forceinline__ void lut8_block_info(const TensorTable& tab, int& t, 
   k.vec16 = k.act && k.cnt == 16 && (k.fl & kVec32) && (k.fl & kDtypeMask) != kF32;
 }
 
-// One step of a probe-group pair: this thread's blocks j and j + 1 (sums at
-// TMEM address ta and ta + 16) over group q and, when `two`, q + 1. Every lane
-// takes part (an inactive lane's sums are never applied), so the step has no
-// branch; four independent Philox calls per step keep the lanes busy while
-// the sums come in from TMEM. Per block the groups are added in order.
+// One step of a probe-group pair: one block of this thread (its sums at TMEM
+// address ta) over group q and, when `two`, q + 1, the groups added in order.
+// Every lane takes part (an inactive lane's sums are never applied), so the
+// step has no per-lane branch; the group-q Philox call runs while the sums
+// come in from TMEM.
 template <bool FIRST>
-__device__ __forceinline__ void lut8_tm_step(uint32_t ta, int64_t b0, int64_t b1, uint32_t q, bool two,
-                                             uint32_t frame, const RoundKeys& keys) {
-  float acc0[16], acc1[16];
-  if (FIRST) {
-    zero16(acc0);
-    zero16(acc1);
-  } else {
-    tm_ld16(acc0, ta);
-    tm_ld16(acc1, ta + 16u);
-  }
-  const uint4 x00 = block_bits(b0, q, keys), x10 = block_bits(b1, q, keys);
-  if (!FIRST) tm_wait_ld2(acc0, acc1);
-  lut8_lookup(acc0, x00, frame);
-  lut8_lookup(acc1, x10, frame);
-  if (two) {
-    const uint4 x01 = block_bits(b0, q + 1u, keys), x11 = block_bits(b1, q + 1u, keys);
-    lut8_lookup(acc0, x01, frame | 128u);
-    lut8_lookup(acc1, x11, frame | 128u);
-  }
-  tm_st16(ta, acc0);
-  tm_st16(ta + 16u, acc1);
+__device__ __forceinline__ void lut8_tm_step(uint32_t ta, int64_t b, uint32_t q, bool two, uint32_t frame,
+                                             const RoundKeys& keys) {
+  float acc[16];
+  if (FIRST)
+    zero16(acc);
+  else
+    tm_ld16(acc, ta);
+  const uint4 x0 = block_bits(b, q, keys);
+  if (!FIRST) tm_wait_ld(acc);
+  lut8_lookup(acc, x0, frame);
+  if (two) lut8_lookup(acc, block_bits(b, q + 1u, keys), frame | 128u);
+  tm_st16(ta, acc);
 }
 
 // Shared memory besides the two regions: coefficients (8 per group), 4-probe
@@ -402,12 +383,10 @@ __global__ void __launch_bounds__(kLut8Threads, 1) update_lut8_kernel(const __gr
         const bool two = static_cast<int>(q) + 1 < G;
         const auto run = [&](auto first) {
 #pragma unroll
-          for (int j = 0; j < BPT; j += 2) {
-            if (!((wact >> j) & 3u)) continue;  // no lane of the warp has either block
-            const int64_t b0 = tab.blk_base + vr_s[j * THREADS + threadIdx.x];
-            const int64_t b1 = tab.blk_base + vr_s[(j + 1) * THREADS + threadIdx.x];
-            lut8_tm_step<decltype(first)::value>(trow + 16u * static_cast<uint32_t>(j), b0, b1, q, two, frame,
-                                                 P.keys);
+          for (int j = 0; j < BPT; ++j) {
+            if (!((wact >> j) & 1u)) continue;  // no lane of the warp has this block
+            const int64_t b = tab.blk_base + vr_s[j * THREADS + threadIdx.x];
+            lut8_tm_step<decltype(first)::value>(trow + 16u * static_cast<uint32_t>(j), b, q, two, frame, P.keys);
           }
         };
         if (pr == 0)
