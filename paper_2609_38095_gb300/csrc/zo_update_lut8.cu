@@ -9,9 +9,10 @@
 //   T_lo[i] = ((s0 a_{8q} + s1 a_{8q+1}) + s2 a_{8q+2}) + s3 a_{8q+3}  (s_j = +1 iff bit j of i)
 // and T_hi likewise for probes 8q+4..8q+7, holds the group's fp32 partial sum
 // for every sign byte n. An element adds one looked-up value per group, groups
-// in increasing order: one byte-permute (the address), one shared load and one
-// add per eight probes. update_kernel adds exactly these partials in this
-// order (as two 4-probe lookups), so the two kernels give the same bits.
+// in increasing order: one byte-permute (the address), one shared load and
+// half a packed fp32x2 add per eight probes. update_kernel adds exactly these
+// partials in this order (as two 4-probe lookups), so the two kernels give
+// the same bits.
 //
 // Bank conflicts. 32 lanes looking up random bytes of one 256-entry table
 // would collide on the 32 shared-memory banks, so every lane reads its own
@@ -98,17 +99,30 @@ __device__ __forceinline__ void lut8_replicate(uint32_t src_t, uint32_t dst_t, i
   }
 }
 
-// Add group q's partial of the 16 elements of a block (Philox output x) to acc.
-// frame: the region's upper half-word, 128 h + 4 l in the low byte.
+// a0, a1 <- rn(a0 + b0), rn(a1 + b1): one packed fp32x2 add (sm_100 and
+// later), the same IEEE round-to-nearest sum per element as two scalar adds.
+// Used on the probe sums only; theta's own add stays scalar, so a NaN result
+// keeps the canonical encoding.
+__device__ __forceinline__ void fadd2_rn(float& a0, float& a1, float b0, float b1) {
+  asm("{\n .reg .b64 pa, pb;\n mov.b64 pa, {%0, %1};\n mov.b64 pb, {%2, %3};\n add.rn.f32x2 pa, pa, pb;\n"
+      " mov.b64 {%0, %1}, pa;\n}"
+      : "+f"(a0), "+f"(a1)
+      : "f"(b0), "f"(b1));
+}
+
+// Add group q's partial of the 16 elements of a block (Philox output x) to acc,
+// two elements per packed add. frame: the region's upper half-word, 128 h + 4 l
+// in the low byte.
 __device__ __forceinline__ void lut8_lookup(float (&acc)[16], const uint4& x, uint32_t frame) {
 #pragma unroll
   for (int m = 0; m < 4; ++m) {
     const uint32_t w = word_of(x, m);
 #pragma unroll
-    for (int j = 0; j < 4; ++j) {
+    for (int j = 0; j < 4; j += 2) {
       // bytes: frame.b0 (lane offset), w.b_j (sign byte -> row), frame.b2, frame.b3 (region)
-      const uint32_t addr = __byte_perm(w, frame, 0x7604u | (static_cast<uint32_t>(j) << 4));
-      acc[4 * m + j] = __fadd_rn(acc[4 * m + j], lds_f32(addr));
+      const uint32_t a0 = __byte_perm(w, frame, 0x7604u | (static_cast<uint32_t>(j) << 4));
+      const uint32_t a1 = __byte_perm(w, frame, 0x7604u | (static_cast<uint32_t>(j + 1) << 4));
+      fadd2_rn(acc[4 * m + j], acc[4 * m + j + 1], lds_f32(a0), lds_f32(a1));
     }
   }
 }
