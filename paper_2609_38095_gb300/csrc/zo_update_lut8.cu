@@ -499,13 +499,26 @@ __device__ __forceinline__ void small_seek(const TensorTable& tab, SmallCursor& 
   c.tp = reinterpret_cast<uint16_t*>(tab.ptr[c.t]);
 }
 
-// Sum of element e's lookups (groups in order) from the Philox words of groups 0 and 1.
+// Sums of elements e and e + 1 (e even) of a block, 0 + T8_0 [+ T8_1] each,
+// from the Philox words of groups 0 and 1, two elements per packed add.
 template <int E>
-__device__ __forceinline__ float small_sum(const uint4& x0, const uint4& x1, uint32_t frame, bool two) {
-  constexpr uint32_t sel = 0x7604u | (static_cast<uint32_t>(E & 3) << 4);
-  float acc = __fadd_rn(0.0f, lds_f32(__byte_perm(word_of(x0, E >> 2), frame, sel)));
-  if (two) acc = __fadd_rn(acc, lds_f32(__byte_perm(word_of(x1, E >> 2), frame | 128u, sel)));
-  return acc;
+__device__ __forceinline__ float2 small_sum2(const uint4& x0, const uint4& x1, uint32_t frame, bool two) {
+  constexpr uint32_t sel0 = 0x7604u | (static_cast<uint32_t>(E & 3) << 4);
+  constexpr uint32_t sel1 = 0x7604u | (static_cast<uint32_t>((E + 1) & 3) << 4);
+  float lo = 0.0f, hi = 0.0f;
+  const uint32_t w0 = word_of(x0, E >> 2);
+  fadd2_rn(lo, hi, lds_f32(__byte_perm(w0, frame, sel0)), lds_f32(__byte_perm(w0, frame, sel1)));
+  if (two) {
+    const uint32_t w1 = word_of(x1, E >> 2);
+    fadd2_rn(lo, hi, lds_f32(__byte_perm(w1, frame | 128u, sel0)), lds_f32(__byte_perm(w1, frame | 128u, sel1)));
+  }
+  return make_float2(lo, hi);
+}
+
+// theta pair + the leading perturbation's signed scales, one packed add.
+__device__ __forceinline__ void add_signed2(float2& f, const uint4& x, int i, const PerturbOp& op) {
+  fadd2_rn(f.x, f.y, __uint_as_float(op.nscale_bits ^ sign_bit(x, i, op.bit)),
+           __uint_as_float(op.nscale_bits ^ sign_bit(x, i + 1, op.bit)));
 }
 
 template <uint8_t DT>
@@ -513,21 +526,26 @@ __device__ __forceinline__ void small_block16(uint32_t (&v)[8], const uint4& x0,
                                               uint32_t frame, bool two, const UpdateParams& P, bool do_sum) {
 #pragma unroll
   for (int r = 0; r < 8; ++r) {
-    if (P.has_pre) v[r] = pre_regs16<DT>(v[r], xp, r, P.pre);
+    float2 f = unpack2<DT>(v[r]);
+    if (P.has_pre) {
+      add_signed2(f, xp, 2 * r, P.pre);
+      v[r] = pack2<DT>(f.x, f.y);  // the perturbed value is rounded to storage first
+      f = unpack2<DT>(v[r]);
+    }
     if (do_sum) {
-      const float2 f = unpack2<DT>(v[r]);
-      float lo, hi;
+      float2 acc;
       switch (r) {  // element indices must be constants for the word and byte selects
-        case 0: lo = small_sum<0>(x0, x1, frame, two); hi = small_sum<1>(x0, x1, frame, two); break;
-        case 1: lo = small_sum<2>(x0, x1, frame, two); hi = small_sum<3>(x0, x1, frame, two); break;
-        case 2: lo = small_sum<4>(x0, x1, frame, two); hi = small_sum<5>(x0, x1, frame, two); break;
-        case 3: lo = small_sum<6>(x0, x1, frame, two); hi = small_sum<7>(x0, x1, frame, two); break;
-        case 4: lo = small_sum<8>(x0, x1, frame, two); hi = small_sum<9>(x0, x1, frame, two); break;
-        case 5: lo = small_sum<10>(x0, x1, frame, two); hi = small_sum<11>(x0, x1, frame, two); break;
-        case 6: lo = small_sum<12>(x0, x1, frame, two); hi = small_sum<13>(x0, x1, frame, two); break;
-        default: lo = small_sum<14>(x0, x1, frame, two); hi = small_sum<15>(x0, x1, frame, two); break;
+        case 0: acc = small_sum2<0>(x0, x1, frame, two); break;
+        case 1: acc = small_sum2<2>(x0, x1, frame, two); break;
+        case 2: acc = small_sum2<4>(x0, x1, frame, two); break;
+        case 3: acc = small_sum2<6>(x0, x1, frame, two); break;
+        case 4: acc = small_sum2<8>(x0, x1, frame, two); break;
+        case 5: acc = small_sum2<10>(x0, x1, frame, two); break;
+        case 6: acc = small_sum2<12>(x0, x1, frame, two); break;
+        default: acc = small_sum2<14>(x0, x1, frame, two); break;
       }
-      v[r] = pack2<DT>(__fadd_rn(f.x, lo), __fadd_rn(f.y, hi));
+      fadd2_rn(f.x, f.y, acc.x, acc.y);
+      v[r] = pack2<DT>(f.x, f.y);
     }
   }
 }
