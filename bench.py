@@ -96,9 +96,19 @@ def measured_peaks():
     return {"hbm_gbs": FALLBACK_HBM_GBS, "sm_max_mhz": 2070.0}, "fallback"
 
 
-def kernel_source_hash():
+# The sources each kernel is compiled from: a traffic figure stays valid
+# while they are unchanged.
+KERNEL_SOURCES = {
+    "perturb_kernel": ("zo_device.cuh", "zo_stream_kernels.cu"),
+    "perturb2_kernel": ("zo_device.cuh", "zo_stream_kernels.cu"),
+    "perturb_pair_kernel": ("zo_device.cuh", "zo_stream_kernels.cu"),
+    "update_lut8_kernel": ("zo_device.cuh", "zo_update_lut8.cu"),
+}
+
+
+def kernel_source_hash(kernel):
     h = hashlib.sha256()
-    for f in ("zo_device.cuh", "zo_stream_kernels.cu", "zo_update_lut8.cu"):
+    for f in KERNEL_SOURCES[kernel]:
         with open(os.path.join(ROOT, "paper_2609_38095_gb300", "csrc", f), "rb") as fh:
             h.update(fh.read())
     return h.hexdigest()[:16]
@@ -111,7 +121,7 @@ def committed_traffic(kernel, config_key):
     p = os.path.join(ROOT, "profiles", "ncu_traffic.txt")
     if not os.path.exists(p):
         return None, "no ncu summary committed"
-    want = kernel_source_hash()
+    want = kernel_source_hash(kernel)
     for line in open(p):
         parts = line.split()
         if len(parts) >= 4 and parts[0] == kernel and parts[1] == config_key and parts[2] == want:
@@ -906,6 +916,12 @@ def run_zo(args):
                                             if shifted else "perturb_kernel<1, 0> (zo_perturb)", perturb_ms, n1)
         traffic, traffic_how = committed_traffic("perturb_kernel", traffic_key)
     dom_bytes = pair_bytes if pair else perturb_bytes
+    # the update's DRAM bytes (one read and one write of theta, whatever K): the
+    # 8-probe-table kernel's committed capture when it is the one this K runs
+    if args.packing == 1 and 16 < K <= 384 and not shifted:
+        upd_traffic, upd_traffic_how = committed_traffic("update_lut8_kernel", traffic_key)
+    else:
+        upd_traffic, upd_traffic_how = None, "no capture committed for the update kernel this K runs"
     # algorithmic HBM bytes of one step: every pass reads and writes theta once,
     # except the pair passes (read theta, write two copies)
     step_bytes = my_probes * pair_bytes + perturb_bytes if pair else passes * perturb_bytes
@@ -965,7 +981,8 @@ def run_zo(args):
                          "frac": step_bytes / (hbm_peak * 1e9) / (ms_per_step * 1e-3)},
             "update": {"ms": update_ms, "gparam_probe_per_s": upd_rate, "bound": "alu",
                        "peak_gparam_probe_per_s_1instr": alu_peak, "frac_alu_1instr": upd_rate / alu_peak,
-                       "GB/s": perturb_bytes / (update_ms * 1e-3) / 1e9},
+                       "GB/s": perturb_bytes / (update_ms * 1e-3) / 1e9,
+                       "traffic": upd_traffic, "traffic_source": upd_traffic_how},
             "precondition": {"ms": precond_ms},
         },
         "e2e": e2e,
