@@ -351,6 +351,39 @@ def test_update_within_tolerance(K, packing_mode):
             print(f"K={K} tensor {i}: {st}")
 
 
+@pytest.mark.parametrize("bpt,K,pre", [(8, 24, True), (8, 40, False), (4, 24, False), (4, 40, True),
+                                       (2, 64, True), (2, 200, False)])
+def test_update_every_chunk_size(bpt, K, pre):
+    """The 8-probe-table update (packing 1, 16 < K <= 384) gives each CTA a
+    chunk of 512 x BPT blocks, BPT = 8, 4 or 2 by launch size (every SM gets
+    a chunk). Lists sized for each BPT on this device, with bf16, fp16 and
+    fp32 tensors, partial last blocks, a zero-length tensor and a view off the
+    32-byte grid (its blocks skipped by the kernel and done by
+    update_shift_kernel), against the oracle element by element."""
+    sms = torch.cuda.get_device_properties(0).multi_processor_count
+    blocks = sms * 512 * bpt + 3 * 512 + 7            # just above this BPT's threshold
+    numels = [blocks * 16 - 9 * 4096 - 3001 - 17, 4096 * 9 + 5, 0, 3001, 17]
+    dtypes = [torch.bfloat16, torch.float16, torch.bfloat16, torch.float32, torch.float16]
+    host, dev = make_list(numels, dtypes, seed=bpt * 1000 + K)
+    # the fp16 tensor as a view one element into its own allocation
+    base = torch.empty(numels[1] + 1, dtype=torch.float16, device="cuda")
+    dev[1] = base[1:]
+    dev[1].copy_(to_torch(host[1], torch.float16))
+    dts = [TORCH_TO_DT[d] for d in dtypes]
+    c_np = np.random.default_rng(K + bpt).normal(0, 25, K)
+    c = torch.tensor(c_np, dtype=torch.float64, device="cuda")
+    seed, lr, eps = W.step_seed(K + bpt), 1e-3, 1e-3
+    zo.update(dev, seed, c, lr, pre=(K - 1, eps) if pre else None)
+    if pre:
+        oracle.perturb(host, dts, seed, K - 1, eps)
+    oracle.update(host, dts, seed, c_np, lr)
+    for i, (d, h, dt) in enumerate(zip(dev, host, dts)):
+        if h.size:
+            st = assert_update_close(storage_bits(d), storage_bits(h), dt, c_np, lr,
+                                     context=f"BPT={bpt} K={K} tensor {i}")
+            print(f"BPT={bpt} K={K} tensor {i}: {st}")
+
+
 def test_update_max_probes(packing_mode):
     K = zo.ZO_MAX_PROBES
     host, dev = make_list([5003, 16, 1], [torch.float32, torch.bfloat16, torch.float16], seed=77)
