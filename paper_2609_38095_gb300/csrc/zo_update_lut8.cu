@@ -475,7 +475,10 @@ __global__ void __launch_bounds__(kLut8Threads, 1) update_lut8_kernel(const __gr
 // load issued before the current block is computed, and every element takes
 // its one or two lookups and is stored at once: the same sums, in the same
 // order (0 + T8_0 [+ T8_1]), as the chunked kernel. The leading perturbation
-// reuses the Philox word of its own group when it is one of the two.
+// reuses the Philox word of its own group when it is one of the two. The group
+// count and the leading perturbation's case are template arguments: with
+// 64 registers a thread (1024 threads), the run-time flags cost 7-14 % of
+// the time of this issue-bound loop.
 // ---------------------------------------------------------------------------
 constexpr int kSmallThreads = 1024;
 size_t lut8_small_smem_bytes() { return 2 * static_cast<size_t>(kLut8Region) + 16u; }
@@ -521,13 +524,14 @@ __device__ __forceinline__ void add_signed2(float2& f, const uint4& x, int i, co
            __uint_as_float(op.nscale_bits ^ sign_bit(x, i + 1, op.bit)));
 }
 
-template <uint8_t DT>
+template <uint8_t DT, bool TWO>
 __device__ __forceinline__ void small_block16(uint32_t (&v)[8], const uint4& x0, const uint4& x1, const uint4& xp,
-                                              uint32_t frame, bool two, const UpdateParams& P, bool do_sum) {
+                                              uint32_t frame, bool pre, const UpdateParams& P, bool do_sum) {
+  constexpr bool two = TWO;
 #pragma unroll
   for (int r = 0; r < 8; ++r) {
     float2 f = unpack2<DT>(v[r]);
-    if (P.has_pre) {
+    if (pre) {
       add_signed2(f, xp, 2 * r, P.pre);
       v[r] = pack2<DT>(f.x, f.y);  // the perturbed value is rounded to storage first
       f = unpack2<DT>(v[r]);
@@ -552,6 +556,7 @@ __device__ __forceinline__ void small_block16(uint32_t (&v)[8], const uint4& x0,
 
 // Any other block of the launch: fp32, a partial last block, padding, or an
 // unaligned tensor (update_shift_kernel's).
+template <int TAG>
 __device__ __noinline__ void small_block_other(const TensorTable& tab, int t, uint32_t b, const UpdateParams& P,
                                                uint32_t frame, bool do_sum) {
   const uint32_t tb = tensor_blk_begin(tab, t);
@@ -575,6 +580,12 @@ __device__ __noinline__ void small_block_other(const TensorTable& tab, int t, ui
   lut8_apply_other(k, acc, P, do_sum);
 }
 
+// Leading perturbation of the small kernel's instantiations: on a Philox word
+// the sums also use (group 0 or 1), on its own word, or decided at run time
+// (no leading perturbation, or any).
+constexpr int kPreShared = 1, kPreOwn = 2, kPreRuntime = 3;
+
+template <int PRE, bool TWO>
 __global__ void __launch_bounds__(kSmallThreads, 1) update_lut8_small_kernel(const __grid_constant__ UpdateParams P) {
   extern __shared__ __align__(16) unsigned char smem[];
   __shared__ int skip_s;
@@ -591,7 +602,8 @@ __global__ void __launch_bounds__(kSmallThreads, 1) update_lut8_small_kernel(con
     a_s[k] = k < P.K ? __double2float_rn(P.coef_mul * P.coef[k]) : 0.0f;
   __syncthreads();
   const bool skip = skip_s != 0;
-  if (skip && !P.has_pre) return;
+  const bool has_pre = PRE == kPreRuntime ? P.has_pre : true;
+  if (skip && !has_pre) return;
   const bool do_sum = !skip;
   if (do_sum) {
     for (int e = threadIdx.x; e < 256 * G; e += kSmallThreads) {
@@ -609,9 +621,12 @@ __global__ void __launch_bounds__(kSmallThreads, 1) update_lut8_small_kernel(con
   const uint32_t total = tab.blk_total;
   const uint32_t stride = gridDim.x * kSmallThreads;
   const uint32_t frame = (region0 & 0xFFFF0000u) | ((threadIdx.x & 31u) << 2);
-  const bool two = G > 1;
+  constexpr bool two = TWO;
   // the leading perturbation's Philox word: group 0's, group 1's, or its own
-  const int pre_src = !P.has_pre ? -1 : (P.pre.ctr2 == 0u ? 0 : (P.pre.ctr2 == 1u && two ? 1 : 2));
+  // the leading perturbation's Philox word: none (-1), group 0's or group 1's (0, 1), or its own (2)
+  const int pre_src = PRE == kPreOwn ? 2
+                      : PRE == kPreShared ? (P.pre.ctr2 == 1u ? 1 : 0)
+                      : (!P.has_pre ? -1 : (P.pre.ctr2 == 0u ? 0 : (P.pre.ctr2 == 1u && two ? 1 : 2)));
   uint32_t b = blockIdx.x * kSmallThreads + threadIdx.x;
   if (b >= total) return;
   SmallCursor c;
@@ -646,12 +661,12 @@ __global__ void __launch_bounds__(kSmallThreads, 1) update_lut8_small_kernel(con
       if (pre_src == 1) xp = x1;
       if (pre_src == 2) xp = block_bits(vb, P.pre.ctr2, P.keys);
       if (dt == kBF16)
-        small_block16<kBF16>(v, x0, x1, xp, frame, two, P, do_sum);
+        small_block16<kBF16, TWO>(v, x0, x1, xp, frame, has_pre, P, do_sum);
       else
-        small_block16<kF16>(v, x0, x1, xp, frame, two, P, do_sum);
+        small_block16<kF16, TWO>(v, x0, x1, xp, frame, has_pre, P, do_sum);
       st256(p, v);
     } else {
-      small_block_other(tab, t, b, P, frame, do_sum);
+      small_block_other<2 * PRE + TWO>(tab, t, b, P, frame, do_sum);
     }
     if (bn >= total) break;
     b = bn;
@@ -685,11 +700,20 @@ bool lut8_supported(int groups, int packing) { return packing == kPacking1 && gr
 
 cudaError_t lut8_prepare(int groups, int* blocks_per_sm) {
   if (groups <= 2) {
-    cudaError_t e = cudaFuncSetAttribute(update_lut8_small_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                         static_cast<int>(lut8_small_smem_bytes()));
+    const int lim = static_cast<int>(lut8_small_smem_bytes());
+    cudaError_t e = cudaSuccess;
+    const void* kernels[] = {
+        reinterpret_cast<const void*>(update_lut8_small_kernel<kPreShared, false>),
+        reinterpret_cast<const void*>(update_lut8_small_kernel<kPreShared, true>),
+        reinterpret_cast<const void*>(update_lut8_small_kernel<kPreOwn, false>),
+        reinterpret_cast<const void*>(update_lut8_small_kernel<kPreOwn, true>),
+        reinterpret_cast<const void*>(update_lut8_small_kernel<kPreRuntime, false>),
+        reinterpret_cast<const void*>(update_lut8_small_kernel<kPreRuntime, true>)};
+    for (const void* k : kernels)
+      if (e == cudaSuccess) e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, lim);
     if (e != cudaSuccess) return e;
-    return cudaOccupancyMaxActiveBlocksPerMultiprocessor(blocks_per_sm, update_lut8_small_kernel, kSmallThreads,
-                                                         lut8_small_smem_bytes());
+    return cudaOccupancyMaxActiveBlocksPerMultiprocessor(blocks_per_sm, update_lut8_small_kernel<kPreRuntime, true>,
+                                                         kSmallThreads, lut8_small_smem_bytes());
   }
   cudaError_t e = lut8_prepare_cfg<2>(groups, blocks_per_sm);
   if (e == cudaSuccess) e = lut8_prepare_cfg<4>(groups, blocks_per_sm);
@@ -710,8 +734,26 @@ cudaError_t launch_update_lut8(const UpdateParams& p, int sms, int blocks_per_sm
   const int64_t cap = static_cast<int64_t>(sms) * blocks_per_sm;
   if (p.groups <= 2) {
     const int64_t want = (total + kSmallThreads - 1) / kSmallThreads;
-    update_lut8_small_kernel<<<static_cast<int>(want < cap ? want : cap), kSmallThreads, lut8_small_smem_bytes(),
-                               stream>>>(p);
+    const int g = static_cast<int>(want < cap ? want : cap);
+    const size_t sm = lut8_small_smem_bytes();
+    // with a leading perturbation: its Philox word one of the sums' or its own;
+    // without one, the run-time instantiation (faster there: its registers are
+    // laid out for the leading perturbation and it does not spill)
+    const bool two = p.groups == 2;
+    const int pre = !p.has_pre ? kPreRuntime
+                               : (p.pre.ctr2 == 0u || (p.pre.ctr2 == 1u && two) ? kPreShared : kPreOwn);
+    if (pre == kPreShared && two)
+      update_lut8_small_kernel<kPreShared, true><<<g, kSmallThreads, sm, stream>>>(p);
+    else if (pre == kPreShared)
+      update_lut8_small_kernel<kPreShared, false><<<g, kSmallThreads, sm, stream>>>(p);
+    else if (pre == kPreOwn && two)
+      update_lut8_small_kernel<kPreOwn, true><<<g, kSmallThreads, sm, stream>>>(p);
+    else if (pre == kPreOwn)
+      update_lut8_small_kernel<kPreOwn, false><<<g, kSmallThreads, sm, stream>>>(p);
+    else if (two)
+      update_lut8_small_kernel<kPreRuntime, true><<<g, kSmallThreads, sm, stream>>>(p);
+    else
+      update_lut8_small_kernel<kPreRuntime, false><<<g, kSmallThreads, sm, stream>>>(p);
     return cudaGetLastError();
   }
   // one CTA per chunk of 512 * BPT blocks, at most the resident CTAs

@@ -732,6 +732,28 @@ def test_update_with_leading_perturb(K, packing_mode):
         assert_update_close(storage_bits(d), storage_bits(h), dt, c_np, lr)
 
 
+@pytest.mark.parametrize("K,pre_probe", [(3, 1), (3, 9), (9, 3), (9, 40), (16, 100), (24, 200)])
+def test_update_with_leading_perturb_of_another_probe(K, pre_probe, packing_mode):
+    """The leading perturbation's probe in one of the update's own probe
+    groups (its Philox word shared with the sums) or in another group (its own
+    word), one or two groups: the same as the perturbation then the update."""
+    host, dev = make_list(MIXED_NUMELS, MIXED_DTYPES, seed=K + pre_probe)
+    dts = [TORCH_TO_DT[d] for d in MIXED_DTYPES]
+    dev2 = [t.clone() for t in dev]
+    c_np = np.random.default_rng(K + pre_probe).normal(0, 25, K)
+    c = torch.tensor(c_np, device="cuda")
+    seed, lr, eps = W.step_seed(pre_probe), 1e-3, -2e-3
+    zo.update(dev, seed, c, lr, pre=(pre_probe, eps))
+    zo.perturb(dev2, seed, pre_probe, eps)
+    zo.update(dev2, seed, c, lr)
+    for x, y in zip(dev, dev2):
+        assert torch.equal(x.view(torch.uint8), y.view(torch.uint8)) if x.numel() else True
+    oracle.perturb(host, dts, seed, pre_probe, eps)
+    oracle.update(host, dts, seed, c_np, lr)
+    for d, h, dt in zip(dev, host, dts):
+        assert_update_close(storage_bits(d), storage_bits(h), dt, c_np, lr)
+
+
 def test_update_with_leading_perturb_after_failed_preconditioner():
     """A non-finite loss skips the probe sum but never the restore."""
     host, dev = make_list(MIXED_NUMELS, MIXED_DTYPES, seed=99)
