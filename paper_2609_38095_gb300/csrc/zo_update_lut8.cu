@@ -520,8 +520,10 @@ __device__ __forceinline__ float2 small_sum2(const uint4& x0, const uint4& x1, u
 
 // theta pair + the leading perturbation's signed scales, one packed add.
 __device__ __forceinline__ void add_signed2(float2& f, const uint4& x, int i, const PerturbOp& op) {
-  fadd2_rn(f.x, f.y, __uint_as_float(op.nscale_bits ^ sign_bit(x, i, op.bit)),
-           __uint_as_float(op.nscale_bits ^ sign_bit(x, i + 1, op.bit)));
+  // the probe bit moved to bit 31 by a multiply (PerturbOp::mul): the
+  // multiply-add pipe instead of the integer ALU, the busier one here
+  fadd2_rn(f.x, f.y, __uint_as_float(op.nscale_bits ^ ((word_of(x, i >> 2) * op.mul[i & 3]) & 0x80000000u)),
+           __uint_as_float(op.nscale_bits ^ ((word_of(x, (i + 1) >> 2) * op.mul[(i + 1) & 3]) & 0x80000000u)));
 }
 
 template <uint8_t DT, bool TWO>
