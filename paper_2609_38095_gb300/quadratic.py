@@ -40,30 +40,35 @@ class QuadraticStep:
         self.c = torch.empty(self.K, dtype=torch.float64, device=dev)
         self.status = torch.zeros(1, dtype=torch.int32, device=dev)
         self.ws = torch.empty(zo.quadratic_loss_workspace_size(theta.numel()), dtype=torch.uint8, device=dev)
-
-    def loss(self, out):
-        zo.quadratic_loss(self.theta, self.a, out=out, workspace=self.ws)
+        # the loss with its arguments checked once, and the table cells it writes
+        self.loss = zo.QuadraticLoss(theta, a, self.ws)
+        row = self.losses.stride(0) * self.losses.element_size()
+        base = self.loss.out_address(self.losses)
+        self._lp = [base + k * row for k in range(self.K)]                  # L+ of probe k
+        self._lm = [base + k * row + 8 for k in range(self.K)]              # L- of probe k
+        self._l0 = base + 16                                                # L0, row 0
+        self._l0_rows = (self.losses[1:, 2], self.losses[0:1, 2].expand(self.K - 1)) if self.K > 1 else None
 
     def step(self, seed: int):
         """Enqueue one step on the current stream (nothing waits)."""
-        K, eps, L = self.K, self.eps, self.losses
-        self.loss(L[0, 2:3])                                   # clean loss L0 (Algorithm 1)
-        if K > 1:
-            L[1:, 2].copy_(L[0:1, 2].expand(K - 1))
+        K, eps = self.K, self.eps
+        self.loss(self._l0)                                    # clean loss L0 (Algorithm 1)
+        if self._l0_rows is not None:
+            self._l0_rows[0].copy_(self._l0_rows[1])           # into every row's third column
         fused = self.schedule == "fused"
         if fused:
             zo.perturb(self.plist, seed, 0, eps)
         for k in range(K):
             if not fused:
                 zo.perturb(self.plist, seed, k, eps)
-            self.loss(L[k, 0:1])                               # L+ at theta + eps z_k
+            self.loss(self._lp[k])                             # L+ at theta + eps z_k
             zo.perturb(self.plist, seed, k, -2 * eps)
-            self.loss(L[k, 1:2])                               # L- at theta - eps z_k
+            self.loss(self._lm[k])                             # L- at theta - eps z_k
             if not fused:
                 zo.perturb(self.plist, seed, k, eps)           # restore
             elif k + 1 < K:
                 zo.perturb2(self.plist, seed, k, eps, k + 1, eps)
-        zo.precondition(L, eps, out=(self.c, self.status))
+        zo.precondition(self.losses, eps, out=(self.c, self.status))
         zo.update(self.plist, seed, self.c, self.lr, status=self.status, pre=(K - 1, eps) if fused else None)
 
     def library_launches_per_step(self) -> int:

@@ -360,6 +360,39 @@ def quadratic_loss(theta, a, out=None, workspace=None):
     return out
 
 
+class QuadraticLoss:
+    """quadratic_loss with theta, a and the workspace checked once: a call
+    takes only the address of its output (a float64 on theta's device, for
+    example an element of a loss table) and enqueues the kernels. For a step
+    that evaluates the loss 2K + 1 times on the same weights."""
+
+    def __init__(self, theta, a, workspace=None):
+        n = theta.numel()
+        if a.numel() != n:
+            raise ValueError("theta and a differ in size")
+        self.device = theta.device
+        if workspace is None:
+            workspace = torch.empty(quadratic_loss_workspace_size(n), dtype=torch.uint8, device=self.device)
+        if workspace.numel() * workspace.element_size() < quadratic_loss_workspace_size(n):
+            raise ValueError("workspace too small")
+        _same_device(self.device, a=a, workspace=workspace)
+        self._keep = (theta, a, workspace)   # the addresses below stay valid while these live
+        self._args = (_dev_ptr(theta, torch.float32, "theta"), _dev_ptr(a, torch.float32, "a"), n)
+        self._ws = (_dev_ptr(workspace, what="workspace"), workspace.numel() * workspace.element_size())
+
+    def out_address(self, out):
+        """The address to pass for `out` (a float64 element on theta's device)."""
+        if not isinstance(out, torch.Tensor) or out.dtype != torch.float64 or out.numel() < 1:
+            raise ValueError("out must hold one float64")
+        _same_device(self.device, out=out)
+        return out.data_ptr()
+
+    def __call__(self, out_address: int):
+        with _on(self.device):
+            rc = _lib().zo_quadratic_loss(*self._args, ctypes.c_void_p(out_address), *self._ws, _stream(self.device))
+        _check("zo_quadratic_loss", rc)
+
+
 def quadratic_loss_static(theta, a, out=None):
     """zo_quadratic_loss_static: the same loss with the library's fixed
     scratch instead of a workspace (the call itself allocates nothing; pass

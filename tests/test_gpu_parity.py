@@ -502,6 +502,28 @@ def test_quadratic_loss(n):
     assert zo.quadratic_loss(td, ad).item() == got   # fixed order: reproducible
 
 
+def test_prepared_quadratic_loss():
+    """QuadraticLoss (arguments checked once) writes the same value as
+    quadratic_loss into any float64 cell, and rejects bad arguments."""
+    n = (1 << 20) + 7
+    td = torch.from_numpy(W.tiny_theta(n)).cuda()
+    ad = torch.from_numpy(W.tiny_curvatures(n)).cuda()
+    table = torch.full((4, 3), -1.0, dtype=torch.float64, device="cuda")
+    q = zo.QuadraticLoss(td, ad)
+    q(q.out_address(table[2, 1:2]))
+    want = zo.quadratic_loss(td, ad).item()
+    assert table[2, 1].item() == want
+    assert (table.view(-1)[torch.arange(12, device="cuda") != 7] == -1.0).all()   # nothing else written
+    with pytest.raises(ValueError):
+        zo.QuadraticLoss(td, ad[:-1])
+    with pytest.raises(ValueError):
+        zo.QuadraticLoss(td, ad, workspace=torch.empty(8, dtype=torch.uint8, device="cuda"))
+    with pytest.raises(ValueError):
+        q.out_address(torch.empty(1, dtype=torch.float32, device="cuda"))
+    with pytest.raises(TypeError):
+        zo.QuadraticLoss(td, ad.double())
+
+
 # ------------------------------------------------------- small workload, e2e
 def test_tiny_workload_lockstep():
     """Ten full steps of the small workload (d = 2^20 fp32, quadratic loss,
