@@ -52,7 +52,8 @@ LANES_PER_SM = 128
 def parse_args():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
-    ap.add_argument("--steps", type=int, default=2)
+    ap.add_argument("--steps", type=int, default=None,
+                    help="timed steps (default 2; 10 for --config tiny, the small workload's ten full steps)")
     ap.add_argument("--warmup", type=int, default=3)
     ap.add_argument("--impl", choices=["zo", "reference"], default="zo")
     ap.add_argument("--config", default="opt-30b", choices=sorted(W.BY_KEY))
@@ -85,7 +86,10 @@ def parse_args():
     ap.add_argument("--view-offset", type=int, default=0,
                     help="every parameter a view this many elements into its own allocation (e.g. 1: off the "
                          "32-byte grid, the perturbation passes run the aligned-chunk kernel)")
-    return ap.parse_args()
+    args = ap.parse_args()
+    if args.steps is None:
+        args.steps = W.TINY_STEPS if args.config == "tiny" else 2
+    return args
 
 
 def measured_peaks():
