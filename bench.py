@@ -985,6 +985,8 @@ def run_zo(args):
                          "frac": step_bytes / (hbm_peak * 1e9) / (ms_per_step * 1e-3)},
             "update": {"ms": update_ms, "gparam_probe_per_s": upd_rate, "bound": "alu",
                        "peak_gparam_probe_per_s_1instr": alu_peak, "frac_alu_1instr": upd_rate / alu_peak,
+                       # the two-instruction model (an add and a sign operation per pair)
+                       "frac_alu_2instr": upd_rate / (alu_peak / 2),
                        "GB/s": perturb_bytes / (update_ms * 1e-3) / 1e9,
                        "traffic": upd_traffic, "traffic_source": upd_traffic_how},
             "precondition": {"ms": precond_ms},
