@@ -194,8 +194,8 @@ __device__ __forceinline__ void lut8_apply_other(const Lut8Block& k, const float
 // registers hold one block's sums at a time, and each table copy and barrier
 // serves four times the elements of a register-only chunk of two blocks per
 // thread. The copies are what the chunk size is for: a pair's replicated
-// tables are 64 KB of shared-memory stores, against 32 KB of lookups per 1024
-// blocks.
+// tables are 64 KB of shared-memory stores, against 128 KB of lookups per
+// 1024 blocks.
 constexpr int kLut8Threads = 512;
 constexpr uint32_t kTmemCols = 512;
 
