@@ -272,21 +272,40 @@ __device__ __forceinline__ void lut8_replicate4(uint32_t t4, uint32_t dst_t, int
   }
 }
 
-// Block bl of the launch: its tensor (cursor t, moved forward) and place.
-__device__ __forceinline__ void lut8_block_info(const TensorTable& tab, int& t, uint32_t bl, Lut8Block& k) {
+// A thread's tensor while its blocks stay inside it: the table is read again
+// only when a block leaves it.
+struct Lut8Cursor {
+  int t;
+  uint32_t tb, te;  // first and one-past-last launch block
+  int64_t numel;
+  void* base;
+  int64_t vbase;    // virtual block of launch block bl of this tensor, minus bl
+  uint8_t fl;
+};
+
+__device__ __forceinline__ void lut8_seek(const TensorTable& tab, Lut8Cursor& c, uint32_t bl) {
+  c.t = advance_tensor(tab, c.t, bl);
+  c.tb = tensor_blk_begin(tab, c.t);
+  c.te = tab.blk_end[c.t];
+  c.numel = tab.numel[c.t];
+  c.base = reinterpret_cast<void*>(tab.ptr[c.t]);
+  c.vbase = tab.blk_base - static_cast<int64_t>(tab.vdelta[c.t]);
+  c.fl = tab.flags[c.t];
+}
+
+// Block bl of the launch (bl only grows for a cursor): its tensor and place.
+__device__ __forceinline__ void lut8_block_info(const TensorTable& tab, Lut8Cursor& c, uint32_t bl, Lut8Block& k) {
   k.act = bl < tab.blk_total;
   k.vec16 = false;
   if (!k.act) return;
-  t = advance_tensor(tab, t, bl);
-  k.fl = tab.flags[t];
-  const uint32_t tb = tensor_blk_begin(tab, t);
-  // unaligned tensors are update_shift_kernel's; blocks below tb are padding
-  k.act = !(k.fl & kShift) && bl >= tb;
-  k.b = virtual_block(tab, t, bl);
-  k.e0 = static_cast<int64_t>(bl - tb) * 16;
-  k.cnt = static_cast<int>(min(static_cast<int64_t>(16), tab.numel[t] - k.e0));
-  k.base = reinterpret_cast<void*>(tab.ptr[t]);
-  k.vec16 = k.act && k.cnt == 16 && (k.fl & kVec32) && (k.fl & kDtypeMask) != kF32;
+  if (bl >= c.te) lut8_seek(tab, c, bl);
+  k.fl = c.fl;
+  k.act = !(c.fl & kShift) && bl >= c.tb;
+  k.b = c.vbase + static_cast<int64_t>(bl);
+  k.e0 = static_cast<int64_t>(bl - c.tb) * 16;
+  k.cnt = static_cast<int>(min(static_cast<int64_t>(16), c.numel - k.e0));
+  k.base = c.base;
+  k.vec16 = k.act && k.cnt == 16 && (c.fl & kVec32) && (c.fl & kDtypeMask) != kF32;
 }
 
 // One step of a probe-group pair: one block of this thread (its sums at TMEM
@@ -374,18 +393,20 @@ __global__ void __launch_bounds__(kLut8Threads, 1) update_lut8_kernel(const __gr
   const uint32_t per_round = gridDim.x * chunk;
   const uint32_t rounds = (tab.blk_total + per_round - 1u) / per_round;
   uint32_t cur = 0;  // region holding the current pair (0 or 1)
-  int tc = 0;        // tensor cursor: the tensor of this thread's first block of the chunk
+  Lut8Cursor cur0;   // tensor cursor at this thread's first block of the chunk
+  cur0.t = 0;
+  cur0.te = 0;       // nothing cached yet: the first block seeks
 
   for (uint32_t rnd = 0; rnd < rounds; ++rnd) {
     // this thread's blocks of the chunk: cb, cb + THREADS, ..
     const uint32_t cb = (rnd * gridDim.x + blockIdx.x) * chunk + threadIdx.x;
     if (do_sum) {
       uint32_t wact = 0;  // blocks of the chunk that some lane of the warp sums
-      int t = tc;
+      Lut8Cursor c = cur0;
 #pragma unroll
       for (int j = 0; j < BPT; ++j) {
         Lut8Block k;
-        lut8_block_info(tab, t, cb + static_cast<uint32_t>(j * THREADS), k);
+        lut8_block_info(tab, c, cb + static_cast<uint32_t>(j * THREADS), k);
         vr_s[j * THREADS + threadIdx.x] = k.act ? static_cast<uint32_t>(k.b - tab.blk_base) : 0u;
         if (__any_sync(0xFFFFFFFFu, k.act)) wact |= 1u << j;
         // theta is read after all pairs: bring it into L2 meanwhile
@@ -420,12 +441,12 @@ __global__ void __launch_bounds__(kLut8Threads, 1) update_lut8_kernel(const __gr
     // Apply: each block's sums read back from TMEM and added to theta (in L2
     // by now). Full aligned 16-bit blocks here; the rare others (fp32, partial
     // last blocks) in a loop of their own, which keeps their code out of this one.
-    int t = tc;
+    Lut8Cursor c = cur0;
     bool others = false;
 #pragma unroll 1
     for (int j = 0; j < BPT; ++j) {
       Lut8Block k;
-      lut8_block_info(tab, t, cb + static_cast<uint32_t>(j * THREADS), k);
+      lut8_block_info(tab, c, cb + static_cast<uint32_t>(j * THREADS), k);
       others |= k.act && !k.vec16;
       uint32_t v[8];
       if (k.vec16) ld256(static_cast<uint16_t*>(k.base) + k.e0, v);
@@ -443,11 +464,11 @@ __global__ void __launch_bounds__(kLut8Threads, 1) update_lut8_kernel(const __gr
       }
     }
     if (__any_sync(0xFFFFFFFFu, others)) {
-      t = tc;
+      Lut8Cursor c2 = cur0;
 #pragma unroll 1
       for (int j = 0; j < BPT; ++j) {
         Lut8Block k;
-        lut8_block_info(tab, t, cb + static_cast<uint32_t>(j * THREADS), k);
+        lut8_block_info(tab, c2, cb + static_cast<uint32_t>(j * THREADS), k);
         const bool mine = k.act && !k.vec16;
         float acc[16];
         zero16(acc);
@@ -455,7 +476,7 @@ __global__ void __launch_bounds__(kLut8Threads, 1) update_lut8_kernel(const __gr
         if (mine) lut8_apply_other(k, acc, P, do_sum);
       }
     }
-    tc = t;
+    cur0 = c;
   }
   if (do_sum) {
     tm_fence_before();
