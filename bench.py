@@ -350,6 +350,25 @@ def param_set(args):
     return ps
 
 
+def stream_config(ps, args, world):
+    """The `config` of a parameter-set workload: the same dict on both arms
+    (how each arm does the work is in its own top-level keys)."""
+    pp = bool(getattr(args, "probe_parallel", False))
+    return {"workload": ps.name, "K": ps.K, "d": ps.d, "tensors": len(ps.numels), "packing": args.packing,
+            "storage": {W.DT_F16: "fp16", W.DT_BF16: "bf16"}.get(ps.dtype, "fp32"),
+            "eps": ps.eps, "lr": ps.eps, "parallelism": f"probe-parallel{world}" if pp else f"replicas{world}",
+            **({"view_offset": args.view_offset} if args.view_offset else {}),
+            "l2": "inputs larger than L2 (every pass streams the whole parameter set)"}
+
+
+def tiny_config(ps, args, world):
+    """The `config` of the small workload, the same dict on both arms."""
+    return {"workload": ps.name, "K": ps.K, "d": ps.d, "eps": ps.eps, "lr": W.TINY_LR,
+            "loss": "quadratic 1/2 sum a_i theta_i^2, a_i log-uniform in [1e-2, 1e2]",
+            "parallelism": f"replicas{world}",
+            "l2": f"flushed before every timed step ({L2_FLUSH_BYTES >> 20} MB write outside the events)"}
+
+
 def run_reference(args):
     rank = int(os.environ.get("RANK", "0"))
     if rank != 0:
@@ -361,8 +380,10 @@ def run_reference(args):
         "impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": args.gpus,
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": dt * 1e3, "higher_is_better": True,
         "scaling": "weak", "vs_baseline": None, "dtype": "f32", "data": "synthetic",
-        "config": {"workload": ps.name, "K": ps.K, "d": ps.d, "packing": args.packing, "sample_weights": M},
-        "cpu_baseline": {"value": value, "unit": UNIT, "cores": cores, "kind": "oracle", "sample": sample},
+        "config": stream_config(ps, args, args.gpus),
+        "schedule": f"Algorithm 1 order ({3 * ps.K} perturb passes, the preconditioner, the fused update) on a sample",
+        "cpu_baseline": {"value": value, "unit": UNIT, "cores": cores, "kind": "oracle", "sample": sample,
+                         "extrapolated": True, "sample_weights": M, "cpu_model": cpu_model()},
         "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
     }
     print(json.dumps(line), flush=True)
@@ -500,7 +521,8 @@ def run_tiny(args):
             "impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": args.gpus,
             "steps": args.steps, "warmup": 0, "ms_per_step": st_s * 1e3, "higher_is_better": True,
             "scaling": "weak", "vs_baseline": None, "dtype": "f32", "data": "synthetic",
-            "config": {"workload": ps.name, "K": ps.K, "d": ps.d, "lr": W.TINY_LR, "eps": ps.eps},
+            "config": tiny_config(ps, args, args.gpus),
+            "schedule": "Algorithm 1 order, the oracle's full steps",
             "cpu_baseline": {"value": value, "unit": UNIT, "cores": cores, "kind": "oracle",
                              "sample": f"the whole workload, {args.steps} full steps", "cpu_model": cpu_model()},
             "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}), flush=True)
@@ -592,10 +614,8 @@ def run_tiny(args):
         "metric": METRIC, "value": world * d * K / (ms_per_step * 1e-3) / 1e9, "unit": UNIT, "n_gpus": world,
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms_per_step, "higher_is_better": True,
         "scaling": "weak", "vs_baseline": None, "dtype": "f32", "data": "synthetic",
-        "config": {"workload": ps.name, "K": K, "d": d, "eps": eps, "lr": lr, "schedule": schedule,
-                   "loss": "quadratic 1/2 sum a_i theta_i^2 on the device, a_i log-uniform in [1e-2, 1e2]",
-                   "parallelism": f"replicas{world}",
-                   "l2": f"flushed before every timed step ({L2_FLUSH_BYTES >> 20} MB write outside the events)"},
+        "config": tiny_config(ps, args, world),
+        "schedule": schedule,
         "roofline": {"bound": "hbm", "kernel": "whole step (launch-bound: every kernel moves 8 MB or less)",
                      "achieved": achieved, "peak": hbm_peak, "unit": "GB/s", "frac": achieved / hbm_peak,
                      "traffic": None, "traffic_source": "not captured for the small workload",
@@ -708,7 +728,6 @@ def run_zo(args):
     K, eps, d = ps.K, ps.eps, ps.d
     params = W.allocate_params(ps, device=dev, view_offset=args.view_offset)
     plist = zo.ParamList(params)
-    n_tensors = len(params)
     shifted = any(t.data_ptr() % 32 for t in params)   # the perturbation passes use perturb_shift_kernel
 
     def like_param(t):
@@ -962,15 +981,10 @@ def run_zo(args):
         "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
         "warmup": args.warmup, "ms_per_step": ms_per_step, "higher_is_better": True,
         "scaling": "strong" if pp else "weak", "vs_baseline": None, "dtype": "f32", "data": "synthetic",
-        "config": {"workload": ps.name, "K": K, "d": d, "tensors": n_tensors, "packing": args.packing,
-                   "schedule": (f"probe-parallel pair schedule ({passes} passes over the weights per step on each "
-                                f"of {world} ranks, the K x 3 loss table all-gathered)" if pp else
-                                f"{args.schedule} ({passes} passes over the weights per step)"),
-                   "storage": "fp16" if
-                   ps.dtype == W.DT_F16 else ("bf16" if ps.dtype == W.DT_BF16 else "fp32"),
-                   "eps": eps, "lr": eps, "parallelism": f"probe-parallel{world}" if pp else f"replicas{world}",
-                   **({"view_offset": args.view_offset} if args.view_offset else {}),
-                   "l2": "inputs larger than L2 (every pass streams the whole parameter set)"},
+        "config": stream_config(ps, args, world),
+        "schedule": (f"probe-parallel pair schedule ({passes} passes over the weights per step on each "
+                     f"of {world} ranks, the K x 3 loss table all-gathered)" if pp else
+                     f"{args.schedule} ({passes} passes over the weights per step)"),
         "roofline": {"bound": "hbm", "kernel": dom_kernel, "achieved": dom_achieved, "peak": hbm_peak,
                      "unit": "GB/s", "frac": dom_achieved / hbm_peak, "traffic": traffic, "traffic_source": traffic_how,
                      "peak_source": f"{peak_kind} hbm_gbs", "bytes_per_launch": dom_bytes,

@@ -131,7 +131,8 @@ def assert_update_close(got_bits, want_bits, dt, c, lr, context=""):
                                [(int(i), hex(int(gb[i])), hex(int(wb[i])), int(ulp[i])) for i in far[:5]])
     # in the band (every element for fp32 storage) the derived bound; equal
     # infinities pass (their difference is NaN)
-    bad = np.nonzero(band & ~((np.abs(g - w) <= bound) | (gb == wb)))[0]
+    with np.errstate(invalid="ignore"):
+        bad = np.nonzero(band & ~((np.abs(g - w) <= bound) | (gb == wb)))[0]
     assert bad.size == 0, (context, [(int(i), g[i], w[i], bound[i]) for i in bad[:5]])
     return {"n": int(gb.size + np.sum(nan_w)), "equal": int(np.sum(gb == wb) + np.sum(nan_w)),
             "max_ulp": int(ulp.max()) if ulp.size else 0, "band": int(np.sum(band)) if dt != W.DT_F32 else 0}

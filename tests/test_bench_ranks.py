@@ -81,6 +81,10 @@ def test_reference_arm_line_on_cpu(capsys, monkeypatch):
         assert key in d, key
     assert d["cpu_baseline"]["kind"] == "oracle" and d["cpu_baseline"]["value"] == d["value"]
     assert d["e2e"] == {"value": d["value"], "unit": d["unit"], "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}
+    # the same config dict as the device arm prints (built by the same function)
+    args = bench.parse_args()
+    assert d["config"] == bench.stream_config(bench.param_set(args), args, 1)
+    assert d["config"]["workload"] == "opt-1.3b-shape-bf16" and d["config"]["tensors"] == 388
 
 
 def test_reference_arm_small_workload_on_cpu(capsys, monkeypatch):
@@ -94,6 +98,8 @@ def test_reference_arm_small_workload_on_cpu(capsys, monkeypatch):
     d = json.loads(capsys.readouterr().out.strip().splitlines()[-1])
     assert d["impl"] == "reference" and d["value"] > 0 and d["config"]["d"] == 1 << 20
     assert d["cpu_baseline"]["cores"] == 2 and d["e2e"]["value"] == d["value"]
+    args = bench.parse_args()
+    assert d["config"] == bench.tiny_config(bench.param_set(args), args, 1)
 
 
 def test_cpu_model_and_single_thread_oracle():
