@@ -15,7 +15,8 @@ from paper_2609_38095_gb300 import build as zo_build
 from paper_2609_38095_gb300 import workloads as W
 from paper_2609_38095_gb300 import zo
 
-from gpu_helpers import (TORCH_TO_DT, assert_update_close, storage_bits, storage_np, to_torch, ulp_distance16)
+from gpu_helpers import (TORCH_TO_DT, assert_update_close, bits_to_f64, storage_bits, storage_np, to_torch,
+                         ulp_distance16)
 
 pytestmark = pytest.mark.gpu
 
@@ -382,6 +383,51 @@ def test_update_every_chunk_size(bpt, K, pre):
             st = assert_update_close(storage_bits(d), storage_bits(h), dt, c_np, lr,
                                      context=f"BPT={bpt} K={K} tensor {i}")
             print(f"BPT={bpt} K={K} tensor {i}: {st}")
+
+
+@pytest.mark.parametrize("n_alias", [32, 45])
+@pytest.mark.parametrize("K,pre", [(16, True), (24, True), (40, False)])
+def test_update_beyond_2_32_blocks(n_alias, K, pre):
+    """Tensors whose Philox block counter has a non-zero high word (virtual
+    index >= 2^36). One 2^31-element bf16 tensor (4 GB) listed n_alias times
+    fills the index space below them. A launch holds fewer than 2^31 blocks
+    (15 of these entries), so with 32 entries the checked tensors share a
+    launch that starts below block 2^32 and ends above it (the general step);
+    with 45 their launch starts above it (one high word for the whole launch:
+    the split Philox of the 8-probe-table update). K = 16 takes the small-K
+    kernel, 24 and 40 the chunked one with a last pair of one group. The
+    aliased entries are updated concurrently and end with arbitrary values;
+    only the checked tensors (bf16, a fp16 view off the 32-byte grid, fp32)
+    are compared, element by element, with the oracle at their virtual
+    indices."""
+    free, _ = torch.cuda.mem_get_info()
+    if free < 6 << 30:
+        pytest.skip("needs 6 GB of device memory")
+    big = torch.zeros(1 << 31, dtype=torch.bfloat16, device="cuda")
+    try:
+        numels = [4096 + 7, 1000, 333]
+        dtypes = [torch.bfloat16, torch.float16, torch.float32]
+        host, dev = make_list(numels, dtypes, seed=n_alias * 100 + K)
+        base = torch.empty(numels[1] + 1, dtype=torch.float16, device="cuda")
+        dev[1] = base[1:]
+        dev[1].copy_(to_torch(host[1], torch.float16))
+        dts = [TORCH_TO_DT[d] for d in dtypes]
+        S = oracle.virtual_offsets([big.numel()] * n_alias + numels)[n_alias:]
+        assert S[0] == n_alias << 31 and S[0] >= 1 << 36
+        c_np = np.random.default_rng(K + n_alias).normal(0, 25, K)
+        c = torch.tensor(c_np, dtype=torch.float64, device="cuda")
+        seed, lr, eps = W.step_seed(K + n_alias), 1e-3, 1e-3
+        zo.update([big] * n_alias + dev, seed, c, lr, pre=(K - 1, eps) if pre else None)
+        for i, (d, h, dt) in enumerate(zip(dev, host, dts)):
+            g = np.uint64(S[i]) + np.arange(h.size, dtype=np.uint64)
+            theta = bits_to_f64(storage_bits(h), dt).astype(np.float32)
+            if pre:
+                theta = bits_to_f64(oracle.perturb_elements(dt, g, theta, seed, K - 1, eps), dt).astype(np.float32)
+            want = oracle.update_elements(dt, g, theta, seed, c_np, lr)
+            assert_update_close(storage_bits(d), want, dt, c_np, lr, context=f"{n_alias} entries K={K} tensor {i}")
+    finally:
+        del big
+        torch.cuda.empty_cache()
 
 
 def test_update_max_probes(packing_mode):
