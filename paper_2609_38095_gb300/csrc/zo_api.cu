@@ -436,7 +436,9 @@ int run_perturb(const zo_tensor* params, int32_t n, PerturbParams& pp, DeviceInf
   int loop = zo::kLoopBlocks, bps = d->perturb_bps, slot = -1;
   uint64_t key = 0;
   if (pp.nops == 2) {
-    key = list_key(params, n);
+    // probes in two groups of 8 (two Philox calls per block) run a kernel of
+    // their own, so they get a configuration choice of their own
+    key = list_key(params, n) ^ (pp.op[0].ctr2 != pp.op[1].ctr2 ? 0x9E3779B97F4A7C15ull : 0ull);
     const int c = g_two_op_tuner.pick(key, s, &slot);
     loop = kTwoOpLoop[c];
     bps = d->two_op_bps[c];

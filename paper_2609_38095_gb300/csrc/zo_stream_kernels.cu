@@ -43,14 +43,27 @@ __device__ __forceinline__ float add_signed_mul(float th, const uint4& x, int i,
 }
 
 // Sixteen 16-bit weights in registers (element 2r in the low half of v[r]).
-template <uint8_t DT, int NOPS>
+// CROSS: a two-op pass whose probes fall in two groups of 8 (two Philox calls
+// per block, one pass in eight of the fused schedule). Its adds are packed
+// fp32x2 adds, the same round-to-nearest sum per element: with the second
+// Philox call the loop is issue-bound and the packed adds take it from 20.5
+// to 18.9 ms on the OPT-30B-shaped set, while the one-group pass, bound by
+// HBM, is 1 % slower with them, so it keeps scalar adds.
+template <uint8_t DT, int NOPS, bool CROSS = false>
 __device__ __forceinline__ void perturb_regs16(uint32_t (&v)[8], const uint4 (&x)[2], const PerturbOp (&op)[2]) {
 #pragma unroll
   for (int r = 0; r < 8; ++r) {
 #pragma unroll
     for (int o = 0; o < NOPS; ++o) {
-      const float2 f = unpack2<DT>(v[r]);
-      v[r] = pack2<DT>(add_signed_mul(f.x, x[o], 2 * r, op[o]), add_signed_mul(f.y, x[o], 2 * r + 1, op[o]));
+      if constexpr (CROSS) {
+        float2 f = unpack2<DT>(v[r]);
+        fadd2_rn(f.x, f.y, __uint_as_float(op[o].nscale_bits ^ sign_bit_mul(x[o], 2 * r, op[o])),
+                 __uint_as_float(op[o].nscale_bits ^ sign_bit_mul(x[o], 2 * r + 1, op[o])));
+        v[r] = pack2<DT>(f.x, f.y);
+      } else {
+        const float2 f = unpack2<DT>(v[r]);
+        v[r] = pack2<DT>(add_signed_mul(f.x, x[o], 2 * r, op[o]), add_signed_mul(f.y, x[o], 2 * r + 1, op[o]));
+      }
     }
   }
 }
@@ -139,7 +152,7 @@ __device__ __noinline__ void perturb_block_other(const TensorTable& tab, int t, 
 // software-pipelined loop (the next block's 256-bit load is issued before the
 // current block is computed and stored, so two loads per thread stay in
 // flight; the pass is HBM-bound and needs the bytes in flight).
-template <int NOPS, uint8_t DT>
+template <int NOPS, uint8_t DT, bool CROSS = false>
 __device__ __forceinline__ void perturb_run16(uint16_t* p, uint32_t n, size_t pstride, int64_t vb,
                                               uint32_t stride, const PerturbOp (&op)[2], bool same_ctr,
                                               const RoundKeys& keys) {
@@ -152,8 +165,8 @@ __device__ __forceinline__ void perturb_run16(uint16_t* p, uint32_t n, size_t ps
     uint4 x[2];
     x[0] = block_bits(vb, op[0].ctr2, keys);
     x[1] = x[0];
-    if (NOPS == 2 && !same_ctr) x[1] = block_bits(vb, op[1].ctr2, keys);
-    perturb_regs16<DT, NOPS>(v, x, op);
+    if (NOPS == 2 && (CROSS || !same_ctr)) x[1] = block_bits(vb, op[1].ctr2, keys);
+    perturb_regs16<DT, NOPS, CROSS>(v, x, op);
     st256(p, v);
     p = pn;
     vb += stride;
@@ -184,7 +197,7 @@ __device__ __forceinline__ void* block_addr(const Cursor& c, uint32_t b, int kin
   return reinterpret_cast<char*>(c.tp) + static_cast<size_t>(b - c.tb) * bytes;
 }
 
-template <int NOPS, bool F32V>
+template <int NOPS, bool F32V, bool CROSS = false>
 __device__ __forceinline__ void perturb_blocks(const PerturbParams& P, const PerturbOp (&op)[2], bool same_ctr) {
   const TensorTable& tab = P.tab;
   const uint32_t blk_total = tab.blk_total;
@@ -218,12 +231,12 @@ __device__ __forceinline__ void perturb_blocks(const PerturbParams& P, const Per
     uint4 x[2];
     x[0] = block_bits(vb, op[0].ctr2, P.keys);
     x[1] = x[0];
-    if (NOPS == 2 && !same_ctr) x[1] = block_bits(vb, op[1].ctr2, P.keys);
+    if (NOPS == 2 && (CROSS || !same_ctr)) x[1] = block_bits(vb, op[1].ctr2, P.keys);
     if (kind == kBlock16) {
       if (dt == kBF16)
-        perturb_regs16<kBF16, NOPS>(v, x, op);
+        perturb_regs16<kBF16, NOPS, CROSS>(v, x, op);
       else
-        perturb_regs16<kF16, NOPS>(v, x, op);
+        perturb_regs16<kF16, NOPS, CROSS>(v, x, op);
       st256(p, v);
     } else if (F32V && kind == kBlock32) {
 #pragma unroll
@@ -234,7 +247,9 @@ __device__ __forceinline__ void perturb_blocks(const PerturbParams& P, const Per
       st256(p, v);
       st256(static_cast<char*>(p) + 32, w);
     } else {
-      perturb_block_other<NOPS, F32V ? 2 : kLoopBlocks>(tab, t, b, x[0], x[1], op[0], op[1]);
+      // each kernel its own copy of the out-of-line routine
+      perturb_block_other<NOPS, F32V ? 2 : (CROSS ? kLoopBlocks + 8 : kLoopBlocks)>(tab, t, b, x[0], x[1], op[0],
+                                                                                   op[1]);
     }
     if (bn >= blk_total) break;
     b = bn;
@@ -255,7 +270,7 @@ __device__ __forceinline__ void perturb_blocks(const PerturbParams& P, const Per
 // the full, aligned 16-bit region of its current tensor they go through the
 // tight loop of perturb_run16; any other block (fp32, a partial last block,
 // an unaligned tensor) is handled on its own.
-template <int NOPS, int TAG>
+template <int NOPS, int TAG, bool CROSS = false>
 __device__ __forceinline__ void perturb_runs_range(const PerturbParams& P, const PerturbOp (&op)[2], bool same_ctr,
                                                    uint32_t b, uint32_t end, uint32_t stride) {
   const TensorTable& tab = P.tab;
@@ -274,9 +289,9 @@ __device__ __forceinline__ void perturb_runs_range(const PerturbParams& P, const
       uint16_t* p = c.tp + static_cast<size_t>(b - c.tb) * 16;
       const size_t pstride = static_cast<size_t>(stride) * 16;
       if (c.dt == kBF16)
-        perturb_run16<NOPS, kBF16>(p, n, pstride, vb, stride, op, same_ctr, P.keys);
+        perturb_run16<NOPS, kBF16, CROSS>(p, n, pstride, vb, stride, op, same_ctr, P.keys);
       else
-        perturb_run16<NOPS, kF16>(p, n, pstride, vb, stride, op, same_ctr, P.keys);
+        perturb_run16<NOPS, kF16, CROSS>(p, n, pstride, vb, stride, op, same_ctr, P.keys);
       b += n * stride;
     } else {
       uint4 x[2];
@@ -292,21 +307,22 @@ __device__ __forceinline__ void perturb_runs_range(const PerturbParams& P, const
 // Grid-stride by runs. Fewer instructions per block than perturb_blocks, but
 // the lanes of a warp leave a run up to one iteration apart, which costs
 // most where runs are short (tensors of a few blocks per thread).
-template <int NOPS>
+template <int NOPS, bool CROSS = false>
 __device__ __forceinline__ void perturb_runs(const PerturbParams& P, const PerturbOp (&op)[2], bool same_ctr) {
   const uint32_t stride = gridDim.x * blockDim.x;
-  perturb_runs_range<NOPS, kLoopRuns>(P, op, same_ctr, blockIdx.x * blockDim.x + threadIdx.x, P.tab.blk_total,
-                                      stride);
+  perturb_runs_range<NOPS, CROSS ? kLoopRuns + 8 : kLoopRuns, CROSS>(
+      P, op, same_ctr, blockIdx.x * blockDim.x + threadIdx.x, P.tab.blk_total, stride);
 }
 
-// LOOP selects perturb_blocks (kLoopBlocks) or perturb_runs (kLoopRuns). The
+// LOOP selects perturb_blocks (kLoopBlocks) or perturb_runs (kLoopRuns);
+// CROSS marks a two-op launch whose probes fall in two groups of 8. The
 // single-op pass (zo_perturb) always walks block by block (4.99 ms against
 // 5.56 ms by runs on the Qwen3-8B-shaped set, equal elsewhere). For the two-op
 // pass (zo_perturb2) the faster loop and grid depend on the parameter list
 // (OPT-30B-shaped: runs with 3 blocks per SM 18.54 ms, per block with 4
 // 18.72 ms; Qwen3-8B-shaped: 5.96 ms against 5.27 ms), so the host times the
 // candidates on the caller's own list; all give the same bits.
-template <int NOPS, int LOOP, bool F32V = false>
+template <int NOPS, int LOOP, bool F32V = false, bool CROSS = false>
 __global__ void __launch_bounds__(256) perturb_kernel(const __grid_constant__ PerturbParams P) {
   if (P.status != nullptr && *P.status != 0) return;
   PerturbOp op[2] = {P.op[0], P.op[1]};
@@ -314,9 +330,9 @@ __global__ void __launch_bounds__(256) perturb_kernel(const __grid_constant__ Pe
     op[0].nscale_bits = __float_as_uint(__double2float_rn(P.coef_mul * P.coef[P.probe])) ^ 0x80000000u;
   const bool same_ctr = op[1].ctr2 == op[0].ctr2;
   if (LOOP == kLoopBlocks)
-    perturb_blocks<NOPS, F32V>(P, op, same_ctr);
+    perturb_blocks<NOPS, F32V, CROSS>(P, op, same_ctr);
   else
-    perturb_runs<NOPS>(P, op, same_ctr);
+    perturb_runs<NOPS, CROSS>(P, op, same_ctr);
 }
 
 // ---------------------------------------------------------------------------
@@ -1145,12 +1161,17 @@ __global__ void probe_signs_kernel(RoundKeys keys, uint32_t q, uint32_t j, int64
 namespace zo {
 
 cudaError_t launch_perturb(const PerturbParams& p, int grid, int loop, bool f32v, cudaStream_t stream) {
+  const bool cross = p.nops == 2 && p.op[0].ctr2 != p.op[1].ctr2;
   if (p.nops == 1 && f32v)
     perturb_kernel<1, kLoopBlocks, true><<<grid, kThreads, 0, stream>>>(p);
   else if (p.nops == 1)
     perturb_kernel<1, kLoopBlocks><<<grid, kThreads, 0, stream>>>(p);
+  else if (loop == kLoopRuns && cross)
+    perturb_kernel<2, kLoopRuns, false, true><<<grid, kThreads, 0, stream>>>(p);
   else if (loop == kLoopRuns)
     perturb_kernel<2, kLoopRuns><<<grid, kThreads, 0, stream>>>(p);
+  else if (cross)
+    perturb_kernel<2, kLoopBlocks, false, true><<<grid, kThreads, 0, stream>>>(p);
   else
     perturb_kernel<2, kLoopBlocks><<<grid, kThreads, 0, stream>>>(p);
   return cudaGetLastError();

@@ -99,17 +99,6 @@ __device__ __forceinline__ void lut8_replicate(uint32_t src_t, uint32_t dst_t, i
   }
 }
 
-// a0, a1 <- rn(a0 + b0), rn(a1 + b1): one packed fp32x2 add (sm_100 and
-// later), the same IEEE round-to-nearest sum per element as two scalar adds.
-// Used on the probe sums only; theta's own add stays scalar, so a NaN result
-// keeps the canonical encoding.
-__device__ __forceinline__ void fadd2_rn(float& a0, float& a1, float b0, float b1) {
-  asm("{\n .reg .b64 pa, pb;\n mov.b64 pa, {%0, %1};\n mov.b64 pb, {%2, %3};\n add.rn.f32x2 pa, pa, pb;\n"
-      " mov.b64 {%0, %1}, pa;\n}"
-      : "+f"(a0), "+f"(a1)
-      : "f"(b0), "f"(b1));
-}
-
 // Add group q's partial of the 16 elements of a block (Philox output x) to acc,
 // two elements per packed add. frame: the region's upper half-word, 128 h + 4 l
 // in the low byte.

@@ -386,6 +386,48 @@ def test_update_every_chunk_size(bpt, K, pre):
 
 
 @pytest.mark.parametrize("n_alias", [32, 45])
+def test_perturb_beyond_2_32_blocks(n_alias):
+    """The perturbation passes on tensors whose Philox block counter has a
+    non-zero high word (virtual index >= 2^36), laid out as in
+    test_update_beyond_2_32_blocks: with 32 aliased 2^31-element entries in
+    front, the checked tensors' launch straddles block 2^32; with 45 it
+    starts above it. A single pass, a two-op pass in one group of 8 and one
+    across two groups (the two-group kernel), each bit-exact with the oracle
+    at the checked tensors' virtual indices."""
+    free, _ = torch.cuda.mem_get_info()
+    if free < 6 << 30:
+        pytest.skip("needs 6 GB of device memory")
+    big = torch.zeros(1 << 31, dtype=torch.bfloat16, device="cuda")
+    try:
+        numels = [4096 + 7, 1000, 333]
+        dtypes = [torch.bfloat16, torch.float16, torch.float32]
+        host, dev = make_list(numels, dtypes, seed=n_alias)
+        base = torch.empty(numels[1] + 1, dtype=torch.float16, device="cuda")
+        dev[1] = base[1:]
+        dev[1].copy_(to_torch(host[1], torch.float16))
+        dts = [TORCH_TO_DT[d] for d in dtypes]
+        S = oracle.virtual_offsets([big.numel()] * n_alias + numels)[n_alias:]
+        assert S[0] >= 1 << 36
+        seed, eps = W.step_seed(n_alias), 1e-3
+        plist = zo.ParamList([big] * n_alias + dev)
+        theta = [bits_to_f64(storage_bits(h), dt).astype(np.float32) for h, dt in zip(host, dts)]
+        for ops in (((5, -2 * eps),), ((5, eps), (6, eps)), ((7, eps), (8, eps))):
+            if len(ops) == 1:
+                zo.perturb(plist, seed, ops[0][0], ops[0][1])
+            else:
+                zo.perturb2(plist, seed, ops[0][0], ops[0][1], ops[1][0], ops[1][1])
+            for i, (d, dt) in enumerate(zip(dev, dts)):
+                g = np.uint64(S[i]) + np.arange(numels[i], dtype=np.uint64)
+                for k, sc in ops:
+                    want = oracle.perturb_elements(dt, g, theta[i], seed, k, sc)
+                    theta[i] = bits_to_f64(want, dt).astype(np.float32)
+                np.testing.assert_array_equal(storage_bits(d), want, err_msg=f"{n_alias} entries {ops} tensor {i}")
+    finally:
+        del big
+        torch.cuda.empty_cache()
+
+
+@pytest.mark.parametrize("n_alias", [32, 45])
 @pytest.mark.parametrize("K,pre", [(16, True), (24, True), (40, False)])
 def test_update_beyond_2_32_blocks(n_alias, K, pre):
     """Tensors whose Philox block counter has a non-zero high word (virtual
