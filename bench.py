@@ -70,11 +70,13 @@ def parse_args():
                     help="keep the nvidia-smi clock samples of the timed region in this file")
     ap.add_argument("--packing", type=int, default=1, choices=[1, 8],
                     help="generated bits per (weight, probe): 1 (the paper's bit packing) or 8")
-    ap.add_argument("--schedule", default="fused", choices=["fused", "alg1", "pair"],
-                    help="fused: each restore is folded into the next probe's +eps pass and the last one into "
-                         "the update (2K+1 passes); alg1: Algorithm 1's +eps, -2eps, +eps per probe (3K+1); "
-                         "pair: theta +- eps z_k written out of place by one pass per probe into two extra "
-                         "copies of the weights (K+1 passes, 3 copies in device memory)")
+    ap.add_argument("--schedule", default=None, choices=["fused", "alg1", "pair", "onepass"],
+                    help="fused (default): each restore is folded into the next probe's +eps pass and the last "
+                         "one into the update (2K+1 passes); alg1: Algorithm 1's +eps, -2eps, +eps per probe "
+                         "(3K+1); pair: theta +- eps z_k written out of place by one pass per probe into two extra "
+                         "copies of the weights (K+1 passes, 3 copies in device memory); onepass (--config tiny "
+                         "only, its default): the fused schedule with each pass and the loss after it in one "
+                         "launch")
     ap.add_argument("--probe-parallel", action="store_true",
                     help="the probe-parallel step over the ranks (probe k on rank k mod R, the loss table "
                          "all-gathered, every rank updates); implies the pair schedule")
@@ -90,6 +92,12 @@ def parse_args():
     args = ap.parse_args()
     if args.steps is None:
         args.steps = W.TINY_STEPS if args.config == "tiny" else 2
+    if args.schedule is None:
+        args.schedule = "onepass" if args.config == "tiny" else "fused"
+    if args.schedule == "onepass" and args.config != "tiny":
+        ap.error("--schedule onepass needs --config tiny (the loss it fuses is the small workload's)")
+    if args.schedule == "pair" and args.config == "tiny":
+        ap.error("--config tiny runs the onepass, fused or alg1 schedule")
     return args
 
 
@@ -534,7 +542,7 @@ def run_tiny(args):
         dist.init_process_group("nccl", device_id=dev)
     ps = param_set(args)
     K, eps, lr, d = ps.K, ps.eps, W.TINY_LR, ps.d
-    schedule = "alg1" if args.schedule == "alg1" else "fused"
+    schedule = args.schedule
     theta = torch.from_numpy(W.tiny_theta()).to(dev)
     a = torch.from_numpy(W.tiny_curvatures()).to(dev)
     q = QuadraticStep(theta, a, K, eps, lr, schedule=schedule)
@@ -559,7 +567,10 @@ def run_tiny(args):
     clk = clocks.stop()
     ms_per_step = max_over_ranks(sum(a_.elapsed_time(b_) for a_, b_ in ev) / args.steps, world, dev)
     launches = q.library_launches_per_step()
-    calls = 2 * K + 1 + (2 * K if schedule == "fused" else 3 * K) + 2     # C-ABI calls per step
+    if schedule == "onepass":
+        calls = 2 * K + 1 + 2                                                # C-ABI calls per step
+    else:
+        calls = 2 * K + 1 + (2 * K if schedule == "fused" else 3 * K) + 2
     host_us_per_call = 1e6 * statistics.median(host_s) / calls
     # the same step replayed from a CUDA graph (no host cost per call)
     graph_ms = None
@@ -605,10 +616,32 @@ def run_tiny(args):
     peaks, peak_kind = measured_peaks()
     hbm_peak = float(peaks.get("hbm_gbs", FALLBACK_HBM_GBS))
     # bytes the step must move: each weight pass reads and writes theta, each
-    # loss reads theta and a
-    passes = 2 * K + 1 if schedule == "fused" else 3 * K + 1
-    step_bytes = passes * 2 * d * 4 + (2 * K + 1) * 2 * d * 4
+    # loss reads theta and a (onepass: a pass that perturbs and evaluates
+    # reads theta and a and writes theta)
+    if schedule == "onepass":
+        step_bytes = 2 * K * 3 * d * 4 + 2 * d * 4 + 2 * d * 4
+    else:
+        passes = 2 * K + 1 if schedule == "fused" else 3 * K + 1
+        step_bytes = passes * 2 * d * 4 + (2 * K + 1) * 2 * d * 4
     achieved = step_bytes / (ms_per_step * 1e-3) / 1e9
+    # the fused schedule (separate perturbation and loss launches) on the same
+    # workload, for comparison with onepass
+    other_us = None
+    if schedule == "onepass":
+        th2 = torch.from_numpy(W.tiny_theta()).to(dev)
+        q2 = QuadraticStep(th2, a, K, eps, lr, schedule="fused")
+        for s_ in range(args.warmup):
+            q2.step(W.step_seed(s_))
+        ev2 = []
+        for i in range(args.steps):
+            flush.zero_()
+            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            e0.record(stream)
+            q2.step(W.step_seed(args.warmup + i))
+            e1.record(stream)
+            ev2.append((e0, e1))
+        torch.cuda.synchronize(dev)
+        other_us = 1e3 * sum(x.elapsed_time(y) for x, y in ev2) / len(ev2)
     cpu = None if args.no_cpu_baseline or world > 1 else tiny_cpu_baseline(args, K, eps, lr, args.steps)
     line = {
         "metric": METRIC, "value": world * d * K / (ms_per_step * 1e-3) / 1e9, "unit": UNIT, "n_gpus": world,
@@ -621,9 +654,11 @@ def run_tiny(args):
                      "traffic": None, "traffic_source": "not captured for the small workload",
                      "peak_source": f"{peak_kind} hbm_gbs", "bytes_per_step": step_bytes},
         "tiny": {"us_per_step": ms_per_step * 1e3, "library_launches_per_step": launches,
-                 "torch_launches_per_step": 1 if K > 1 else 0, "abi_calls_per_step": calls,
+                 "torch_launches_per_step": 1 if K > 1 and schedule != "onepass" else 0,
+                 "abi_calls_per_step": calls,
                  "host_us_per_call": host_us_per_call, "host_us_per_step": 1e6 * statistics.median(host_s),
-                 "graph_replay_us_per_step": graph_ms * 1e3 if graph_ms is not None else None},
+                 "graph_replay_us_per_step": graph_ms * 1e3 if graph_ms is not None else None,
+                 "fused_schedule_us_per_step": other_us},
         "e2e": {"value": world * d * K / e2e_s / 1e9, "unit": UNIT, "h2d_bytes_per_step": 0,
                 "d2h_bytes_per_step": 12, "ms_per_step": e2e_s * 1e3},
         "gpu_launches": launches * args.steps,

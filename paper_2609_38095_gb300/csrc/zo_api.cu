@@ -594,7 +594,7 @@ const char* zo_status_string(int status) {
 
 const char* zo_last_cuda_error(void) { return g_last_cuda_error; }
 
-int zo_version(void) { return 10300; }
+int zo_version(void) { return 10400; }
 
 int zo_set_packing(int32_t bits_per_value) {
   if (bits_per_value != zo::kPacking1 && bits_per_value != zo::kPacking8) return ZO_ERR_ARG;
@@ -867,6 +867,38 @@ int zo_quadratic_loss(const float* theta, const float* a, int64_t n, double* out
   cudaError_t e = zo::launch_quadratic_loss(theta, a, n, out, static_cast<double*>(workspace), zo::kMaxLossPartials,
                                             d->sms, static_cast<cudaStream_t>(stream));
   return e == cudaSuccess ? ZO_OK : cuda_fail(e, "quadratic_loss");
+}
+
+int64_t zo_perturb_quadratic_loss_workspace_size(int64_t n) {
+  (void)n;
+  // the partials, then the ticket counter (8 bytes keep the size a multiple of 8)
+  return static_cast<int64_t>(zo::kMaxQuadPassPartials) * static_cast<int64_t>(sizeof(double)) + 8;
+}
+
+int zo_perturb_quadratic_loss(float* theta, const float* a, int64_t n, uint64_t seed, int32_t packing, int32_t nops,
+                              uint32_t probe_a, float scale_a, uint32_t probe_b, float scale_b, double* out,
+                              int32_t out_copies, int64_t out_stride, void* workspace, int64_t workspace_bytes,
+                              void* stream) {
+  if (n < 0 || out == nullptr || (n > 0 && (theta == nullptr || a == nullptr))) return ZO_ERR_ARG;
+  if (nops < 0 || nops > 2 || out_copies < 1 || out_stride < 1) return ZO_ERR_ARG;
+  if (packing != 0 && packing != zo::kPacking1 && packing != zo::kPacking8) return ZO_ERR_ARG;
+  if ((nops >= 1 && !std::isfinite(scale_a)) || (nops == 2 && !std::isfinite(scale_b))) return ZO_ERR_ARG;
+  if (reinterpret_cast<uintptr_t>(theta) % sizeof(float) != 0 || reinterpret_cast<uintptr_t>(a) % sizeof(float) != 0)
+    return ZO_ERR_ALIGN;
+  if (workspace == nullptr || workspace_bytes < zo_perturb_quadratic_loss_workspace_size(n)) return ZO_ERR_WORKSPACE;
+  if (reinterpret_cast<uintptr_t>(workspace) % sizeof(double) != 0) return ZO_ERR_ALIGN;
+  DeviceInfo* d = nullptr;
+  int rc = device_info(&d);
+  if (rc != ZO_OK) return rc;
+  const int pk = packing != 0 ? packing : g_packing.load();
+  const zo::RoundKeys keys = expand_keys(seed);
+  const zo::PerturbOp ops[2] = {make_op(probe_a, scale_a, pk), make_op(probe_b, scale_b, pk)};
+  double* partial = static_cast<double*>(workspace);
+  uint32_t* ticket = reinterpret_cast<uint32_t*>(partial + zo::kMaxQuadPassPartials);
+  cudaError_t e = zo::launch_perturb_quad_loss(theta, a, n, keys, ops, nops, out, out_copies, out_stride, partial,
+                                               ticket, zo::kMaxQuadPassPartials, d->sms,
+                                               static_cast<cudaStream_t>(stream));
+  return e == cudaSuccess ? ZO_OK : cuda_fail(e, "perturb_quad_loss");
 }
 
 int zo_quadratic_loss_static(const float* theta, const float* a, int64_t n, double* out, void* stream) {

@@ -14,6 +14,7 @@ constexpr int kPrecondRelative = 2;   // ZO_PRECOND_RELATIVE_CURVATURE
 constexpr int kThreads = 256;         // threads per block of the streaming kernels
 constexpr int kMaxLossPartials = 2048;
 constexpr int kStaticLossPartials = 4096;   // fixed scratch of the allocation-free loss (32 KB)
+constexpr int kMaxQuadPassPartials = 4096;  // CTAs of the one-pass perturbation + loss
 constexpr int64_t kStaticLossSlice = 2048;  // elements per partial in that variant
 
 // f32v: the launch holds 32-byte aligned fp32 tensors (single-op kernel only).
@@ -48,5 +49,11 @@ cudaError_t launch_quadratic_loss(const float* theta, const float* a, int64_t n,
                                   int max_partials, int num_sms, cudaStream_t stream);
 cudaError_t launch_quadratic_loss_static(const float* theta, const float* a, int64_t n, double* out,
                                          cudaStream_t stream);
+// ops: nops (0, 1 or 2) perturbations; partial: max_partials doubles; ticket:
+// a zeroed counter, zeroed again by the launch.
+cudaError_t launch_perturb_quad_loss(float* theta, const float* a, int64_t n, const RoundKeys& keys,
+                                     const PerturbOp* ops, int nops, double* out, int out_copies, int64_t out_stride,
+                                     double* partial, uint32_t* ticket, int max_partials, int num_sms,
+                                     cudaStream_t stream);
 
 }  // namespace zo

@@ -114,11 +114,183 @@ __global__ void __launch_bounds__(256) quad_loss_final_kernel(const double* __re
   if (threadIdx.x == 0) *out = __dmul_rn(0.5, bs);
 }
 
+// ---------------------------------------------------------------------------
+// One forward point of the small quadratic workload in one pass: nops (0, 1
+// or 2) perturbations of theta, applied exactly as zo_perturb / zo_perturb2
+// apply them to an fp32 tensor (one fp32 add each), then the loss
+// f(theta') = 1/2 sum a_i theta'_i^2 of the perturbed weights (Algorithm 1's
+// ApplyPackedPerturbation followed by the forward pass, which for this
+// workload is the reduction itself).
+//
+// A thread owns whole 16-element Philox blocks (grid-stride; theta is the
+// parameter list's only tensor, so element i has virtual index i). Each term
+// a_i theta_i^2 is formed without rounding as a pair of fp32 values
+// (Dekker's exact product by fused multiply-add: a t = p + pe, p t = q + qe,
+// term = q + fma(pe, t, qe), the last add carrying a relative error of about
+// 2^-48) and summed into the thread's fp32 pair (s, sl) with Knuth's exact
+// two-sum. Terms outside the range where those products are exact
+// (|p| or |q| below 2^-100 or from 2^126 up, infinities, NaN) are added in
+// fp64 instead, as (double)a * ((double)t * (double)t). So the fp64 pipe,
+// slow on this GPU, sees a few operations per thread instead of five per
+// weight. The thread's value (s + sl in fp64, plus its fp64 part) is folded
+// with the same fixed-order block sum as the loss above into one partial per
+// CTA; the CTA that finishes last (a ticket counter in the workspace, reset
+// by that CTA) folds the partials in index order and writes the result to
+// out[j * out_stride], j < out_copies. No CTA waits for another. For a given
+// grid the order of every sum is fixed: bit-reproducible.
+// ---------------------------------------------------------------------------
+// theta + scale z for element i of a block, fp32 storage: the probe bit moved
+// to the sign by a multiply (PerturbOp::mul), as in the streaming passes.
+__device__ __forceinline__ float add_signed_mul_f32(float th, const uint4& x, int i, const PerturbOp& op) {
+  return __fadd_rn(th, __uint_as_float(op.nscale_bits ^ ((word_of(x, i >> 2) * op.mul[i & 3]) & 0x80000000u)));
+}
+
+struct QuadPassParams {
+  float* theta;
+  const float* a;
+  int64_t n;
+  RoundKeys keys;
+  PerturbOp op[2];
+  double* partial;      // one per CTA
+  uint32_t* ticket;     // zero before the launch; the last CTA zeroes it again
+  double* out;
+  int32_t out_copies;
+  int64_t out_stride;
+};
+
+struct DsSum {  // s + sl, an unevaluated fp32 pair
+  float s = 0.0f, sl = 0.0f;
+};
+
+__device__ __forceinline__ void quad_term(DsSum& ds, double& dsum, float av, float t) {
+  const float p = __fmul_rn(av, t);
+  const float pe = __fmaf_rn(av, t, -p);      // a t - p, exact
+  const float q = __fmul_rn(p, t);
+  const float qe = __fmaf_rn(p, t, -q);       // p t - q, exact
+  const float ap = fabsf(p), aq = fabsf(q);
+  if (ap >= 0x1p-100f && ap < 0x1p126f && aq >= 0x1p-100f && aq < 0x1p126f) {
+    const float r = __fmaf_rn(pe, t, qe);     // the term's low part
+    const float s = __fadd_rn(ds.s, q);       // two-sum of ds.s and q
+    const float bb = __fsub_rn(s, ds.s);
+    const float e = __fadd_rn(__fsub_rn(ds.s, __fsub_rn(s, bb)), __fsub_rn(q, bb));
+    ds.sl = __fadd_rn(ds.sl, __fadd_rn(e, r));
+    ds.s = s;
+  } else {
+    const double td = t;
+    dsum = __dadd_rn(dsum, __dmul_rn(static_cast<double>(av), __dmul_rn(td, td)));
+  }
+}
+
+template <int NOPS, bool VEC>
+__global__ void __launch_bounds__(256) perturb_quad_loss_kernel(const __grid_constant__ QuadPassParams P) {
+  __shared__ double warp_sums[8];
+  __shared__ bool last_s;
+  DsSum ds;
+  double dsum = 0.0;
+  const int64_t nb = (P.n + 15) / 16;
+  const int64_t stride = static_cast<int64_t>(gridDim.x) * blockDim.x;
+  const bool same_ctr = P.op[1].ctr2 == P.op[0].ctr2;
+  for (int64_t b = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; b < nb; b += stride) {
+    const int64_t e0 = b * 16;
+    const int cnt = static_cast<int>(min(static_cast<int64_t>(16), P.n - e0));
+    float t[16], av[16];
+    if (VEC && cnt == 16) {
+      const float4* tp = reinterpret_cast<const float4*>(P.theta + e0);
+      const float4* ap = reinterpret_cast<const float4*>(P.a + e0);
+#pragma unroll
+      for (int j = 0; j < 4; ++j) {
+        const float4 x = tp[j], y = ap[j];
+        t[4 * j] = x.x; t[4 * j + 1] = x.y; t[4 * j + 2] = x.z; t[4 * j + 3] = x.w;
+        av[4 * j] = y.x; av[4 * j + 1] = y.y; av[4 * j + 2] = y.z; av[4 * j + 3] = y.w;
+      }
+    } else {
+#pragma unroll
+      for (int i = 0; i < 16; ++i) {
+        t[i] = i < cnt ? P.theta[e0 + i] : 0.0f;
+        av[i] = i < cnt ? P.a[e0 + i] : 0.0f;
+      }
+    }
+    if (NOPS >= 1) {
+      const uint4 x0 = block_bits(b, P.op[0].ctr2, P.keys);
+      uint4 x1 = x0;
+      if (NOPS == 2 && !same_ctr) x1 = block_bits(b, P.op[1].ctr2, P.keys);
+#pragma unroll
+      for (int i = 0; i < 16; ++i) {
+        t[i] = add_signed_mul_f32(t[i], x0, i, P.op[0]);
+        if (NOPS == 2) t[i] = add_signed_mul_f32(t[i], x1, i, P.op[1]);
+      }
+      if (VEC && cnt == 16) {
+        float4* tp = reinterpret_cast<float4*>(P.theta + e0);
+#pragma unroll
+        for (int j = 0; j < 4; ++j) tp[j] = make_float4(t[4 * j], t[4 * j + 1], t[4 * j + 2], t[4 * j + 3]);
+      } else {
+#pragma unroll
+        for (int i = 0; i < 16; ++i)
+          if (i < cnt) P.theta[e0 + i] = t[i];
+      }
+    }
+#pragma unroll
+    for (int i = 0; i < 16; ++i)
+      if (i < cnt) quad_term(ds, dsum, av[i], t[i]);
+  }
+  const double mine = __dadd_rn(__dadd_rn(static_cast<double>(ds.s), static_cast<double>(ds.sl)), dsum);
+  const double bs = block_sum(mine, warp_sums);
+  if (threadIdx.x == 0) {
+    P.partial[blockIdx.x] = bs;
+    __threadfence();  // the partial is visible before the ticket counts it
+    last_s = atomicAdd(P.ticket, 1u) == gridDim.x - 1u;
+  }
+  __syncthreads();
+  if (!last_s) return;
+  __threadfence();
+  double s = 0.0;
+  for (int i = threadIdx.x; i < static_cast<int>(gridDim.x); i += blockDim.x) s = __dadd_rn(s, __ldcg(P.partial + i));
+  const double total = block_sum(s, warp_sums);
+  if (threadIdx.x == 0) {
+    const double f = __dmul_rn(0.5, total);
+    for (int j = 0; j < P.out_copies; ++j) P.out[static_cast<int64_t>(j) * P.out_stride] = f;
+    *P.ticket = 0u;
+  }
+}
+
 cudaError_t launch_precondition(const double* losses, int K, double eps, double alpha, double lambda_reg,
                                 int flags, double* c, double* w, double* curv, int32_t* status,
                                 cudaStream_t stream) {
   const int threads = ((K + 31) / 32) * 32;
   precondition_kernel<<<1, threads, 0, stream>>>(losses, K, eps, alpha, lambda_reg, flags, c, w, curv, status);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_perturb_quad_loss(float* theta, const float* a, int64_t n, const RoundKeys& keys,
+                                     const PerturbOp* ops, int nops, double* out, int out_copies, int64_t out_stride,
+                                     double* partial, uint32_t* ticket, int max_partials, int num_sms,
+                                     cudaStream_t stream) {
+  QuadPassParams P;
+  P.theta = theta;
+  P.a = a;
+  P.n = n;
+  P.keys = keys;
+  P.op[0] = ops[0];
+  P.op[1] = nops == 2 ? ops[1] : ops[0];
+  P.partial = partial;
+  P.ticket = ticket;
+  P.out = out;
+  P.out_copies = out_copies;
+  P.out_stride = out_stride;
+  const int threads = 256;
+  const int64_t want = ((n + 15) / 16 + threads - 1) / threads;
+  int64_t cap = static_cast<int64_t>(num_sms) * 8;
+  if (cap > max_partials) cap = max_partials;
+  const int grid = static_cast<int>(want < 1 ? 1 : (want > cap ? cap : want));
+  const bool vec = reinterpret_cast<uintptr_t>(theta) % 16 == 0 && reinterpret_cast<uintptr_t>(a) % 16 == 0;
+  switch (nops * 2 + (vec ? 1 : 0)) {
+    case 0: perturb_quad_loss_kernel<0, false><<<grid, threads, 0, stream>>>(P); break;
+    case 1: perturb_quad_loss_kernel<0, true><<<grid, threads, 0, stream>>>(P); break;
+    case 2: perturb_quad_loss_kernel<1, false><<<grid, threads, 0, stream>>>(P); break;
+    case 3: perturb_quad_loss_kernel<1, true><<<grid, threads, 0, stream>>>(P); break;
+    case 4: perturb_quad_loss_kernel<2, false><<<grid, threads, 0, stream>>>(P); break;
+    default: perturb_quad_loss_kernel<2, true><<<grid, threads, 0, stream>>>(P); break;
+  }
   return cudaGetLastError();
 }
 

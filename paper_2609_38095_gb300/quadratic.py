@@ -9,16 +9,23 @@ a call of the C ABI; the only other device work is the copy of L0 into the
 table's third column (K doubles).
 
 Schedules (the weights at every forward point and after the step are the
-same bits in both):
-  fused  the restore of probe k and the +eps of probe k+1 in one pass
-         (zo_perturb2), the last restore inside the update pass (zo_update_ex)
-  alg1   Algorithm 1's +eps, -2 eps, +eps passes per probe, then the update
+same bits in all three):
+  onepass  the fused schedule with every perturbation pass and the loss that
+           follows it in one launch (zo_perturb_quadratic_loss): 2K + 1
+           launches for the forward points, then the preconditioner and the
+           update
+  fused    the restore of probe k and the +eps of probe k+1 in one pass
+           (zo_perturb2), the last restore inside the update pass
+           (zo_update_ex); each loss a call of zo_quadratic_loss
+  alg1     Algorithm 1's +eps, -2 eps, +eps passes per probe, then the update
+The losses of onepass differ from the other two by rounding only (each loss
+term carried in fp32 pairs instead of fp64).
 """
 import torch
 
 from . import zo
 
-SCHEDULES = ("fused", "alg1")
+SCHEDULES = ("onepass", "fused", "alg1")
 
 
 class QuadraticStep:
@@ -42,6 +49,7 @@ class QuadraticStep:
         self.ws = torch.empty(zo.quadratic_loss_workspace_size(theta.numel()), dtype=torch.uint8, device=dev)
         # the loss with its arguments checked once, and the table cells it writes
         self.loss = zo.QuadraticLoss(theta, a, self.ws)
+        self.onepass = zo.QuadraticPass(theta, a) if schedule == "onepass" else None
         row = self.losses.stride(0) * self.losses.element_size()
         base = self.loss.out_address(self.losses)
         self._lp = [base + k * row for k in range(self.K)]                  # L+ of probe k
@@ -52,6 +60,17 @@ class QuadraticStep:
     def step(self, seed: int):
         """Enqueue one step on the current stream (nothing waits)."""
         K, eps = self.K, self.eps
+        if self.onepass is not None:
+            q = self.onepass
+            q(seed, (), self._l0, copies=K, stride=3)              # clean loss L0 into every row
+            q(seed, ((0, eps),), self._lp[0])                      # L+ of probe 0
+            for k in range(K):
+                q(seed, ((k, -2 * eps),), self._lm[k])             # L- at theta - eps z_k
+                if k + 1 < K:                                      # restore k, +eps of k + 1, L+ of k + 1
+                    q(seed, ((k, eps), (k + 1, eps)), self._lp[k + 1])
+            zo.precondition(self.losses, eps, out=(self.c, self.status))
+            zo.update(self.plist, seed, self.c, self.lr, status=self.status, pre=(K - 1, eps))
+            return
         self.loss(self._l0)                                    # clean loss L0 (Algorithm 1)
         if self._l0_rows is not None:
             self._l0_rows[0].copy_(self._l0_rows[1])           # into every row's third column
@@ -72,9 +91,11 @@ class QuadraticStep:
         zo.update(self.plist, seed, self.c, self.lr, status=self.status, pre=(K - 1, eps) if fused else None)
 
     def library_launches_per_step(self) -> int:
-        """Kernels of this library one step launches (the loss is two: partial
-        sums, then their fold)."""
+        """Kernels of this library one step launches (with zo_quadratic_loss
+        the loss is two: partial sums, then their fold)."""
         K = self.K
+        if self.schedule == "onepass":
+            return 2 * K + 1 + 2
         losses = 2 * (2 * K + 1)
         passes = 2 * K if self.schedule == "fused" else 3 * K
         return losses + passes + 2

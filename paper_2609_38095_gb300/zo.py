@@ -30,7 +30,8 @@ DTYPE_CODE = {torch.float32: 0, torch.bfloat16: 1, torch.float16: 2}
 EXPORTS = ["zo_status_string", "zo_last_cuda_error", "zo_version", "zo_set_packing", "zo_get_packing",
            "zo_perturb", "zo_perturb2", "zo_perturb_pair", "zo_precondition",
            "zo_precondition_ex", "zo_update", "zo_update_ex", "zo_update_sequential", "zo_probe_bytes", "zo_probe_signs",
-           "zo_quadratic_loss_workspace_size", "zo_quadratic_loss", "zo_quadratic_loss_static"]
+           "zo_quadratic_loss_workspace_size", "zo_quadratic_loss", "zo_quadratic_loss_static",
+           "zo_perturb_quadratic_loss_workspace_size", "zo_perturb_quadratic_loss"]
 ZO_QUADRATIC_LOSS_STATIC_MAX_N = 8388608
 
 
@@ -79,6 +80,9 @@ def _lib():
             "zo_quadratic_loss_workspace_size": ([i64], i64),
             "zo_quadratic_loss": ([vp, vp, i64, vp, vp, i64, vp], c.c_int),
             "zo_quadratic_loss_static": ([vp, vp, i64, vp, vp], c.c_int),
+            "zo_perturb_quadratic_loss_workspace_size": ([i64], i64),
+            "zo_perturb_quadratic_loss": ([vp, vp, i64, u64, i32, i32, u32, f32, u32, f32, vp, i32, i64, vp, i64, vp],
+                                          c.c_int),
         }
         for name, (args, res) in sig.items():
             f = getattr(L, name)
@@ -410,4 +414,71 @@ def quadratic_loss_static(theta, a, out=None):
         rc = _lib().zo_quadratic_loss_static(_dev_ptr(theta, torch.float32, "theta"), _dev_ptr(a, torch.float32, "a"),
                                              n, _dev_ptr(out, torch.float64, "out"), _stream(dev))
     _check("zo_quadratic_loss_static", rc)
+    return out
+
+
+def perturb_quadratic_loss_workspace_size(n: int) -> int:
+    return _lib().zo_perturb_quadratic_loss_workspace_size(n)
+
+
+def _quad_ops(ops):
+    ops = list(ops)
+    if len(ops) > 2:
+        raise ValueError("at most two perturbations per pass")
+    pa, sa = ops[0] if ops else (0, 0.0)
+    pb, sb = ops[1] if len(ops) == 2 else (0, 0.0)
+    return len(ops), int(pa), float(sa), int(pb), float(sb)
+
+
+class QuadraticPass:
+    """zo_perturb_quadratic_loss with theta, a and the workspace checked once:
+    one forward point of the small workload per call -- up to two
+    perturbations of theta (as perturb / perturb2 apply them) and the loss of
+    the result, in one pass. The workspace is allocated zero-filled here, as
+    the call requires. packing: None follows the process default."""
+
+    def __init__(self, theta, a, workspace=None, packing=None):
+        n = theta.numel()
+        if a.numel() != n:
+            raise ValueError("theta and a differ in size")
+        if packing not in (None, 1, 8):
+            raise ValueError("packing must be None, 1 or 8")
+        self.device = theta.device
+        size = perturb_quadratic_loss_workspace_size(n)
+        if workspace is None:
+            workspace = torch.zeros(size, dtype=torch.uint8, device=self.device)
+        if workspace.numel() * workspace.element_size() < size:
+            raise ValueError("workspace too small")
+        _same_device(self.device, a=a, workspace=workspace)
+        self._keep = (theta, a, workspace)
+        self._args = (_dev_ptr(theta, torch.float32, "theta"), _dev_ptr(a, torch.float32, "a"), n)
+        self._ws = (_dev_ptr(workspace, what="workspace"), workspace.numel() * workspace.element_size())
+        self.packing = packing or 0
+
+    def out_address(self, out):
+        """The address to pass for `out` (float64 elements on theta's device)."""
+        if not isinstance(out, torch.Tensor) or out.dtype != torch.float64 or out.numel() < 1:
+            raise ValueError("out must hold float64 elements")
+        _same_device(self.device, out=out)
+        return out.data_ptr()
+
+    def __call__(self, seed: int, ops, out_address: int, copies: int = 1, stride: int = 1):
+        """ops: a list of at most two (probe, scale) pairs applied in order;
+        the loss goes to copies float64 cells stride elements apart."""
+        nops, pa, sa, pb, sb = _quad_ops(ops)
+        with _on(self.device):
+            rc = _lib().zo_perturb_quadratic_loss(*self._args, seed, self.packing, nops, pa, sa, pb, sb,
+                                                  ctypes.c_void_p(out_address), copies, stride, *self._ws,
+                                                  _stream(self.device))
+        _check("zo_perturb_quadratic_loss", rc)
+
+
+def perturb_quadratic_loss(theta, a, seed: int, ops, out=None, workspace=None, packing=None):
+    """One pass: theta <- theta + scale z_probe for each (probe, scale) of ops
+    (at most two, in order), then out[0] <- 1/2 sum a_i theta_i^2 of the
+    result (zo_perturb_quadratic_loss). Returns out (a float64 tensor)."""
+    if out is None:
+        out = torch.empty(1, dtype=torch.float64, device=theta.device)
+    q = QuadraticPass(theta, a, workspace=workspace, packing=packing)
+    q(seed, ops, q.out_address(out))
     return out

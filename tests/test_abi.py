@@ -34,7 +34,7 @@ def test_exports_every_declared_symbol(L):
 
 
 def test_version_and_strings(L):
-    assert zo.version() == 10300
+    assert zo.version() == 10400
     for s in (0, -1, -2, -3, -4, -5, -6, -7):
         assert zo.status_string(s).startswith("ZO_")
     assert "unknown" in zo.status_string(99)
@@ -160,6 +160,30 @@ def test_static_loss_validation(L):
     assert f(p, p, zo.ZO_QUADRATIC_LOSS_STATIC_MAX_N + 1, p, None) == zo.ZO_ERR_WORKSPACE
 
 
+def test_perturb_quadratic_loss_validation(L):
+    """zo_perturb_quadratic_loss rejects bad arguments on the host, before
+    any CUDA call (the pointers here are never dereferenced)."""
+    p = ctypes.c_void_p(FAKE)
+    f = L.zo_perturb_quadratic_loss
+    ws = L.zo_perturb_quadratic_loss_workspace_size(1 << 20)
+    assert ws >= 8 and ws % 8 == 0
+
+    def call(n=16, packing=0, nops=1, sa=1e-3, sb=1e-3, out=p, copies=1, stride=1, theta=p, a=p, w=p, wb=ws):
+        return f(theta, a, n, 1, packing, nops, 0, sa, 1, sb, out, copies, stride, w, wb, None)
+
+    assert call(n=-1) == zo.ZO_ERR_ARG
+    assert call(nops=3) == zo.ZO_ERR_ARG and call(nops=-1) == zo.ZO_ERR_ARG
+    assert call(sa=float("nan")) == zo.ZO_ERR_ARG
+    assert call(nops=2, sb=float("inf")) == zo.ZO_ERR_ARG
+    assert call(copies=0) == zo.ZO_ERR_ARG and call(stride=0) == zo.ZO_ERR_ARG
+    assert call(out=None) == zo.ZO_ERR_ARG and call(theta=None) == zo.ZO_ERR_ARG
+    assert call(packing=2) == zo.ZO_ERR_ARG
+    assert call(theta=ctypes.c_void_p(FAKE + 2)) == zo.ZO_ERR_ALIGN
+    assert call(a=ctypes.c_void_p(FAKE + 1)) == zo.ZO_ERR_ALIGN
+    assert call(w=None) == zo.ZO_ERR_WORKSPACE and call(wb=ws - 8) == zo.ZO_ERR_WORKSPACE
+    assert call(w=ctypes.c_void_p(FAKE + 4)) == zo.ZO_ERR_ALIGN
+
+
 def test_packing_switch(L):
     assert zo.get_packing() == 1
     assert L.zo_set_packing(3) == zo.ZO_ERR_ARG
@@ -203,7 +227,7 @@ def test_header_is_plain_c_and_links_from_c(tmp_path, L):
         "#include <stdio.h>\n#include <string.h>\n#include \"zo.h\"\n"
         "int main(void) {\n"
         "  zo_tensor t = {0, 0, ZO_BF16, 0};\n"
-        "  if (zo_version() != 10300) return 1;\n"
+        "  if (zo_version() != 10400) return 1;\n"
         "  if (strncmp(zo_status_string(ZO_ERR_ARG), \"ZO_ERR_ARG\", 10) != 0) return 2;\n"
         "  if (zo_perturb(&t, -1, 1, 0, 1e-3f, NULL) != ZO_ERR_ARG) return 3;\n"
         "  if (zo_set_packing(3) != ZO_ERR_ARG) return 4;\n"

@@ -73,14 +73,15 @@ def rel_diff(got, want):
     return [float(np.max(np.abs(g - w) / np.abs(w))) for g, w in zip(got, want)]
 
 
-def test_free_running_trajectory_matches_the_oracle():
+@pytest.mark.parametrize("schedule", ["fused", "onepass"])
+def test_free_running_trajectory_matches_the_oracle(schedule):
     ps = W.TINY
     K, eps, lr = ps.K, ps.eps, W.TINY_LR
     want, _ = oracle_trajectory(W.TINY_STEPS, K, eps, lr)
-    got, _ = device_trajectory(W.TINY_STEPS, K, eps, lr, "fused")
+    got, _ = device_trajectory(W.TINY_STEPS, K, eps, lr, schedule)
     rel = rel_diff(got, want)
     growth = [w[0, 2] / want[0][0, 2] for w in want]
-    print("free-running small workload, lr = 1e-2: relative loss drift per step",
+    print(f"free-running small workload ({schedule}), lr = 1e-2: relative loss drift per step",
           " ".join(f"{r:.1e}" for r in rel), "; loss growth", " ".join(f"{g:.1e}" for g in growth))
     stable = [s for s, g in enumerate(growth) if g < 1e5]
     assert len(stable) >= 3
@@ -91,14 +92,15 @@ def test_free_running_trajectory_matches_the_oracle():
     assert got[-1][0, 2] > got[0][0, 2] and want[-1][0, 2] > want[0][0, 2]
 
 
-def test_free_running_trajectory_at_a_stable_step_size():
+@pytest.mark.parametrize("schedule", ["fused", "onepass"])
+def test_free_running_trajectory_at_a_stable_step_size(schedule):
     ps = W.TINY
     K, eps, lr = ps.K, ps.eps, 1e-5
     want, _ = oracle_trajectory(W.TINY_STEPS, K, eps, lr)
-    got, _ = device_trajectory(W.TINY_STEPS, K, eps, lr, "fused")
+    got, _ = device_trajectory(W.TINY_STEPS, K, eps, lr, schedule)
     for s, (g, w) in enumerate(zip(got, want)):
         np.testing.assert_allclose(g, w, rtol=1e-5, err_msg=f"step {s}")
-    print("free-running small workload, lr = 1e-5: relative loss drift per step",
+    print(f"free-running small workload ({schedule}), lr = 1e-5: relative loss drift per step",
           " ".join(f"{r:.1e}" for r in rel_diff(got, want)))
 
 
