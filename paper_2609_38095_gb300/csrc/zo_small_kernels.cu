@@ -130,14 +130,16 @@ __global__ void __launch_bounds__(256) quad_loss_final_kernel(const double* __re
 // 2^-48) and summed into the thread's fp32 pair (s, sl) with Knuth's exact
 // two-sum. Terms outside the range where those products are exact
 // (|p| or |q| below 2^-100 or from 2^126 up, infinities, NaN) are added in
-// fp64 instead, as (double)a * ((double)t * (double)t). So the fp64 pipe,
-// slow on this GPU, sees a few operations per thread instead of five per
-// weight. The thread's value (s + sl in fp64, plus its fp64 part) is folded
-// with the same fixed-order block sum as the loss above into one partial per
-// CTA; the CTA that finishes last (a ticket counter in the workspace, reset
-// by that CTA) folds the partials in index order and writes the result to
-// out[j * out_stride], j < out_copies. No CTA waits for another. For a given
-// grid the order of every sum is fixed: bit-reproducible.
+// fp64 instead, as (double)a * ((double)t * (double)t), behind a branch that
+// is rarely taken: the fp64 pipe is slow on this GPU, and a predicated-off
+// fp64 instruction still occupies it, so the loss above (five fp64
+// operations per weight) takes 17 us on 2^20 weights. The pairs are summed
+// over each warp's shuffle tree and converted to fp64 per warp, the warps
+// added in order into one partial per CTA; the CTA that finishes last (a
+// ticket counter in the workspace, reset by that CTA) folds the partials in
+// index order and writes the result to out[j * out_stride], j < out_copies.
+// No CTA waits for another. For a given grid the order of every sum is
+// fixed: bit-reproducible.
 // ---------------------------------------------------------------------------
 // theta + scale z for element i of a block, fp32 storage: the probe bit moved
 // to the sign by a multiply (PerturbOp::mul), as in the streaming passes.
@@ -162,23 +164,56 @@ struct DsSum {  // s + sl, an unevaluated fp32 pair
   float s = 0.0f, sl = 0.0f;
 };
 
-__device__ __forceinline__ void quad_term(DsSum& ds, double& dsum, float av, float t) {
+// ds += (q + r) by Knuth's two-sum of ds.s and q; the rounding error and r
+// go to the low part.
+__device__ __forceinline__ void ds_add(DsSum& ds, float q, float r) {
+  const float s = __fadd_rn(ds.s, q);
+  const float bb = __fsub_rn(s, ds.s);
+  const float e = __fadd_rn(__fsub_rn(ds.s, __fsub_rn(s, bb)), __fsub_rn(q, bb));
+  ds.sl = __fadd_rn(ds.sl, __fadd_rn(e, r));
+  ds.s = s;
+}
+
+// The term a t^2 as q + r (see above); false when it leaves the range where
+// the fp32 products are exact (then q = r = 0 and the caller adds it in fp64).
+// Branch-free: the slow fp64 pipe is only reached through the caller's
+// rarely taken branch.
+__device__ __forceinline__ bool quad_term_ds(float av, float t, float& q, float& r) {
   const float p = __fmul_rn(av, t);
   const float pe = __fmaf_rn(av, t, -p);      // a t - p, exact
-  const float q = __fmul_rn(p, t);
-  const float qe = __fmaf_rn(p, t, -q);       // p t - q, exact
-  const float ap = fabsf(p), aq = fabsf(q);
-  if (ap >= 0x1p-100f && ap < 0x1p126f && aq >= 0x1p-100f && aq < 0x1p126f) {
-    const float r = __fmaf_rn(pe, t, qe);     // the term's low part
-    const float s = __fadd_rn(ds.s, q);       // two-sum of ds.s and q
-    const float bb = __fsub_rn(s, ds.s);
-    const float e = __fadd_rn(__fsub_rn(ds.s, __fsub_rn(s, bb)), __fsub_rn(q, bb));
-    ds.sl = __fadd_rn(ds.sl, __fadd_rn(e, r));
-    ds.s = s;
-  } else {
-    const double td = t;
-    dsum = __dadd_rn(dsum, __dmul_rn(static_cast<double>(av), __dmul_rn(td, td)));
+  const float q0 = __fmul_rn(p, t);
+  const float qe = __fmaf_rn(p, t, -q0);      // p t - q, exact
+  const float ap = fabsf(p), aq = fabsf(q0);
+  const bool ok = ap >= 0x1p-100f && ap < 0x1p126f && aq >= 0x1p-100f && aq < 0x1p126f;
+  q = ok ? q0 : 0.0f;
+  r = ok ? __fmaf_rn(pe, t, qe) : 0.0f;       // the term's low part
+  return ok;
+}
+
+// Sum of the CTA's fp32 pairs and fp64 parts, in a fixed order: pairs over
+// each warp's shuffle tree (lane l takes lane l + off), converted to fp64 per
+// warp with the warp's fp64 parts (shuffled only when one is non-zero), then
+// the warps in index order. Returns the sum in thread 0.
+__device__ __forceinline__ double block_sum_ds(DsSum ds, double dsum, double* warp_sums) {
+#pragma unroll
+  for (int off = 16; off > 0; off >>= 1) {
+    DsSum o;
+    o.s = __shfl_down_sync(0xFFFFFFFFu, ds.s, off);
+    o.sl = __shfl_down_sync(0xFFFFFFFFu, ds.sl, off);
+    ds_add(ds, o.s, o.sl);
   }
+  if (__any_sync(0xFFFFFFFFu, dsum != 0.0)) {
+#pragma unroll
+    for (int off = 16; off > 0; off >>= 1) dsum = __dadd_rn(dsum, __shfl_down_sync(0xFFFFFFFFu, dsum, off));
+  }
+  const int lane = threadIdx.x & 31, wid = threadIdx.x >> 5;
+  if (lane == 0) warp_sums[wid] = __dadd_rn(__dadd_rn(static_cast<double>(ds.s), static_cast<double>(ds.sl)), dsum);
+  __syncthreads();
+  double s = 0.0;
+  if (threadIdx.x == 0) {
+    for (int i = 0; i < static_cast<int>(blockDim.x >> 5); ++i) s = __dadd_rn(s, warp_sums[i]);
+  }
+  return s;
 }
 
 template <int NOPS, bool VEC>
@@ -229,12 +264,24 @@ __global__ void __launch_bounds__(256) perturb_quad_loss_kernel(const __grid_con
           if (i < cnt) P.theta[e0 + i] = t[i];
       }
     }
+    uint32_t wide = 0;  // terms that go to fp64
 #pragma unroll
-    for (int i = 0; i < 16; ++i)
-      if (i < cnt) quad_term(ds, dsum, av[i], t[i]);
+    for (int i = 0; i < 16; ++i) {
+      float q, r;
+      const bool ok = quad_term_ds(av[i], t[i], q, r);  // padding: a = t = 0, q = r = 0
+      ds_add(ds, q, r);
+      if (!ok && i < cnt) wide |= 1u << i;
+    }
+    if (wide != 0u) {
+#pragma unroll
+      for (int i = 0; i < 16; ++i)
+        if ((wide >> i) & 1u) {
+          const double td = t[i];
+          dsum = __dadd_rn(dsum, __dmul_rn(static_cast<double>(av[i]), __dmul_rn(td, td)));
+        }
+    }
   }
-  const double mine = __dadd_rn(__dadd_rn(static_cast<double>(ds.s), static_cast<double>(ds.sl)), dsum);
-  const double bs = block_sum(mine, warp_sums);
+  const double bs = block_sum_ds(ds, dsum, warp_sums);
   if (threadIdx.x == 0) {
     P.partial[blockIdx.x] = bs;
     __threadfence();  // the partial is visible before the ticket counts it
