@@ -256,13 +256,14 @@ int grid_for(int64_t blocks, int sms, int bps) {
 // the same bits; which is fastest depends on the tensor sizes (measured: runs
 // with 3 blocks per SM on the OPT-30B-shaped set, one block per iteration with
 // 4 on the Qwen3-8B-shaped one, runs with 4 on the OPT-1.3B-shaped one, the
-// spread between candidates from 1 % to 12 %). The first kTrials calls on a
-// list (keyed by its sizes, dtypes, alignments and device) run the candidates
-// in turn, kRounds times each, each call between two events on the caller's
-// stream; once all those events have completed (polled, never waited for),
-// later calls use the candidate with the shortest time. Calls made while the
-// stream is being captured into a graph, or before a decision, use
-// candidate 0.
+// spread between candidates from 1 % to 12 %). The first calls on a list
+// (keyed by its sizes, dtypes, alignments and device, and by whether the two
+// probes fall in one group of 8 or in two) run the candidates in turn, three
+// rounds each (one for the two-group calls), each call between two events on
+// the caller's stream; once all those events have completed (polled, never
+// waited for), later calls use the candidate with the shortest time (the
+// shortest of its rounds). Calls made while the stream is being captured
+// into a graph, or before a decision, use candidate 0.
 // After a failed runtime call of this file's own bookkeeping (events, capture
 // query): reset the thread's last error only when it is that call's error, so
 // an unrelated error the caller has not collected yet stays pending.
@@ -274,7 +275,7 @@ class TwoOpTuner {
  public:
   // Candidate for this call; *slot receives the trial index when the call's
   // launches must be bracketed by that trial's events, else -1.
-  int pick(uint64_t key, cudaStream_t s, int* slot) {
+  int pick(uint64_t key, int rounds, cudaStream_t s, int* slot) {
     *slot = -1;
     cudaStreamCaptureStatus cap = cudaStreamCaptureStatusNone;
     const cudaError_t ce = cudaStreamIsCapturing(s, &cap);
@@ -283,12 +284,12 @@ class TwoOpTuner {
       return 0;
     }
     std::lock_guard<std::mutex> lock(mu_);
-    Entry* e = find(key);
+    Entry* e = find(key, rounds);
     if (e == nullptr) return 0;
     if (e->chosen >= 0) return e->chosen;
     decide(*e);
     if (e->chosen >= 0) return e->chosen;
-    if (e->next < kTrials) {
+    if (e->next < e->trials) {
       *slot = e->next++;
       return *slot % kTwoOpCandidates;
     }
@@ -297,7 +298,7 @@ class TwoOpTuner {
 
   void record(uint64_t key, int slot, int which, cudaStream_t s) {
     std::lock_guard<std::mutex> lock(mu_);
-    Entry* e = find(key);
+    Entry* e = find(key, 0);
     if (e == nullptr || e->ev[slot][which] == nullptr) return;
     const cudaError_t er = cudaEventRecord(e->ev[slot][which], s);
     if (er != cudaSuccess) {
@@ -307,25 +308,29 @@ class TwoOpTuner {
   }
 
  private:
-  static constexpr int kRounds = 3;
-  static constexpr int kTrials = kRounds * kTwoOpCandidates;
+  static constexpr int kMaxRounds = 3;
+  static constexpr int kTrials = kMaxRounds * kTwoOpCandidates;
 
   struct Entry {
     uint64_t key = 0;
     int chosen = -1;
     int next = 0;  // next trial; trial i runs candidate i % kTwoOpCandidates
+    int trials = kTrials;
     bool failed = false;
     cudaEvent_t ev[kTrials][2] = {};
   };
 
-  // Entry of `key`, created with its events on first use (nullptr when the
-  // table is full or events cannot be created: then candidate 0 is used).
-  Entry* find(uint64_t key) {
+  // Entry of `key`, created with its events on first use with `rounds` trial
+  // rounds (1..kMaxRounds; rounds = 0 only looks up). nullptr when absent and
+  // not created, the table is full, or events cannot be created: then
+  // candidate 0 is used.
+  Entry* find(uint64_t key, int rounds) {
     for (Entry& e : entries_)
       if (e.key == key) return &e;
-    if (entries_.size() >= kMaxEntries) return nullptr;
+    if (rounds < 1 || entries_.size() >= kMaxEntries) return nullptr;
     Entry e;
     e.key = key;
+    e.trials = (rounds < kMaxRounds ? rounds : kMaxRounds) * kTwoOpCandidates;
     for (auto& pair : e.ev)
       for (cudaEvent_t& ev : pair)
         if (const cudaError_t ec = cudaEventCreate(&ev); ec != cudaSuccess) {
@@ -341,9 +346,9 @@ class TwoOpTuner {
       e.chosen = 0;
       return;
     }
-    if (e.next < kTrials) return;
+    if (e.next < e.trials) return;
     float best[kTwoOpCandidates];
-    for (int i = 0; i < kTrials; ++i) {
+    for (int i = 0; i < e.trials; ++i) {
       if (const cudaError_t q = cudaEventQuery(e.ev[i][1]); q != cudaSuccess) {  // not done yet (or failed)
         clear_own_error(q);
         return;
@@ -437,9 +442,13 @@ int run_perturb(const zo_tensor* params, int32_t n, PerturbParams& pp, DeviceInf
   uint64_t key = 0;
   if (pp.nops == 2) {
     // probes in two groups of 8 (two Philox calls per block) run a kernel of
-    // their own, so they get a configuration choice of their own
-    key = list_key(params, n) ^ (pp.op[0].ctr2 != pp.op[1].ctr2 ? 0x9E3779B97F4A7C15ull : 0ull);
-    const int c = g_two_op_tuner.pick(key, s, &slot);
+    // their own, so they get a configuration choice of their own, timed one
+    // round per candidate: such calls come once per 8 probes, and three
+    // rounds would leave a K = 16 step still timing candidates after a few
+    // steps
+    const bool cross = pp.op[0].ctr2 != pp.op[1].ctr2;
+    key = list_key(params, n) ^ (cross ? 0x9E3779B97F4A7C15ull : 0ull);
+    const int c = g_two_op_tuner.pick(key, cross ? 1 : 3, s, &slot);
     loop = kTwoOpLoop[c];
     bps = d->two_op_bps[c];
   }

@@ -692,10 +692,12 @@ def test_perturb2_is_two_perturbs(a, b, packing_mode):
 
 
 def test_perturb2_every_tuned_configuration():
-    """zo_perturb2 times its three candidate configurations (three rounds) on
-    the first nine calls for a parameter list, then keeps the fastest: 12
-    calls on one list run every candidate and the chosen one, each bit-exact
-    with the oracle."""
+    """zo_perturb2 times its three candidate configurations on the first nine
+    calls for a parameter list with both probes in one group of 8 (three
+    rounds), and on the first three with the probes in two groups (one
+    round, a kernel of its own), then keeps the fastest of each: 12 calls of
+    the first kind and 6 of the second on one list run every candidate and
+    the chosen one, each bit-exact with the oracle."""
     rng = np.random.default_rng(606)
     numels = [int(x) for x in rng.integers(1, 70000, 40)] + [4096 * 300, 17]
     dtypes = [DTS[int(x)] for x in rng.integers(0, 3, len(numels))]
@@ -703,8 +705,8 @@ def test_perturb2_every_tuned_configuration():
     dts = [TORCH_TO_DT[d] for d in dtypes]
     plist = zo.ParamList(dev)
     seed = W.step_seed(606)
-    for call in range(12):
-        a, b = 2 * call + 7, 2 * call + 8
+    pairs = [(8 * c + 1, 8 * c + 2) for c in range(12)] + [(8 * c + 7, 8 * c + 8) for c in range(6)]
+    for call, (a, b) in enumerate(pairs):
         zo.perturb2(plist, seed, a, 1e-3, b, -1e-3)
         oracle.perturb(host, dts, seed, a, 1e-3)
         oracle.perturb(host, dts, seed, b, -1e-3)
