@@ -198,3 +198,32 @@ def test_tiny_workload_onepass_lockstep():
         np.testing.assert_allclose(cg, c_same, rtol=1e-12)
         oracle.update(host, [W.DT_F32], seed, cg, lr)
         assert_update_close(storage_bits(theta), storage_bits(host[0]), W.DT_F32, cg, lr, context=f"step {step}")
+
+
+def test_tiny_onepass_step_replayed_from_a_cuda_graph():
+    """The onepass step only enqueues work (its workspace counter is left at
+    zero by every launch), so a captured step replays correctly: two replays
+    from the same start give the eager step's losses, coefficients and
+    weights bit for bit."""
+    ps = W.TINY
+    start = W.tiny_theta()
+    a = torch.from_numpy(W.tiny_curvatures()).cuda()
+    theta = torch.from_numpy(start.copy()).cuda()
+    q = QuadraticStep(theta, a, ps.K, ps.eps, W.TINY_LR, schedule="onepass")
+    q.step(W.step_seed(5))
+    torch.cuda.synchronize()
+    want = (q.losses.clone(), q.c.clone(), theta.clone())
+    theta.copy_(torch.from_numpy(start))
+    side = torch.cuda.Stream()
+    side.wait_stream(torch.cuda.current_stream())
+    with torch.cuda.stream(side):
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g, stream=side):
+            q.step(W.step_seed(5))
+    torch.cuda.current_stream().wait_stream(side)
+    for _ in range(2):
+        theta.copy_(torch.from_numpy(start))
+        g.replay()
+        torch.cuda.synchronize()
+        assert torch.equal(q.losses, want[0]) and torch.equal(q.c, want[1])
+        assert torch.equal(theta.view(torch.int32), want[2].view(torch.int32))
