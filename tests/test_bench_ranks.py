@@ -179,3 +179,18 @@ def test_probe_parallel_step_gloo_two_ranks():
         for a, b in zip(two[r][3], one[0][3]):
             view = np.uint32 if a.dtype == np.float32 else np.uint16
             np.testing.assert_array_equal(a.view(view), b.view(view))
+
+
+def test_schedule_defaults_and_combinations(monkeypatch):
+    """The parameter sets default to the fused schedule and the small
+    workload to onepass; onepass needs --config tiny, which does not run the
+    pair schedule."""
+    for argv, want in ((["bench.py"], "fused"), (["bench.py", "--config", "tiny"], "onepass"),
+                       (["bench.py", "--config", "tiny", "--schedule", "fused"], "fused"),
+                       (["bench.py", "--config", "opt-1.3b", "--schedule", "alg1"], "alg1")):
+        monkeypatch.setattr(sys, "argv", argv)
+        assert bench.parse_args().schedule == want, argv
+    for argv in (["bench.py", "--schedule", "onepass"], ["bench.py", "--config", "tiny", "--schedule", "pair"]):
+        monkeypatch.setattr(sys, "argv", argv)
+        with pytest.raises(SystemExit):
+            bench.parse_args()
